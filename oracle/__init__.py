@@ -1,0 +1,37 @@
+"""Float64 CPU oracle for the block-diffusion commit step.
+
+TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and
+``bench.py`` (its ``cpu_baseline`` leg and its ``--impl reference`` arm) may
+import this package. The CUDA library and its Python binding never import it,
+and it imports nothing from them: the two share no code.
+
+Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
+(closed forms, a 50-digit brute force, invariants, a logsumexp cross-check and
+hand-derived commit-rule cases). The only reading that no paper number can pin
+is which blocks may take the top-1 fallback: that is an input (the caller's
+``block_flags``), not a computation of the oracle.
+"""
+
+from .commit_oracle import (
+    ACTIVE,
+    FALLBACK_ELIGIBLE,
+    commit_block,
+    commit_step,
+    decode_bf16,
+    decode_e4m3,
+    lm_head_logits,
+    row_confidence,
+    weights_f64,
+)
+
+__all__ = [
+    "ACTIVE",
+    "FALLBACK_ELIGIBLE",
+    "commit_block",
+    "commit_step",
+    "decode_bf16",
+    "decode_e4m3",
+    "lm_head_logits",
+    "row_confidence",
+    "weights_f64",
+]

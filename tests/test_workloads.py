@@ -1,0 +1,66 @@
+"""The seeded input generator: shapes, dtypes, reproducibility, planted boosts."""
+
+import numpy as np
+import pytest
+import torch
+
+from workloads import ACTIVE, CONFIGS, FALLBACK_ELIGIBLE, generate, scaled
+
+
+def test_five_workloads_have_the_stated_shapes():
+    shapes = [(c.n_seq, c.n_slots, c.block_len, c.d, c.V, len(c.tau)) for c in CONFIGS]
+    assert shapes == [
+        (1, 1, 32, 256, 4096, 1),
+        (8, 2, 32, 2048, 151936, 4),
+        (32, 4, 32, 2048, 157184, 8),
+        (64, 4, 64, 4096, 151936, 16),
+        (256, 8, 64, 5120, 157184, 16),
+    ]
+    assert CONFIGS[1].tau == (0.7, 0.8, 0.9, 0.95)
+    for c in CONFIGS[2:]:
+        assert 0.95 in c.tau and list(c.tau) == sorted(c.tau)
+    assert CONFIGS[2].tau[0] == 0.5 and CONFIGS[2].tau[-1] == pytest.approx(0.98)
+    assert CONFIGS[3].tau[0] == pytest.approx(0.3) and CONFIGS[3].tau[-1] == pytest.approx(0.99)
+
+
+def test_tiny_is_seeded_and_reproducible():
+    a = generate(CONFIGS[0])
+    b = generate(CONFIGS[0])
+    assert torch.equal(a.hidden, b.hidden) and torch.equal(a.weight, b.weight)
+    assert a.hidden.dtype == torch.float32 and a.weight.shape == (4096, 256)
+    assert int(a.pos_masked.sum()) == 32
+    assert a.block_flags.tolist() == [ACTIVE | FALLBACK_ELIGIBLE]
+
+
+def test_tiny_plants_plus_eight_on_half_the_positions():
+    wl = generate(CONFIGS[0])
+    h = wl.hidden.double()
+    w = wl.weight.double()
+    logits = h @ w.T
+    # a planted position has one logit about 8 above its N(0, 1) value, so its
+    # top-2 gap is large; unplanted positions have the small gaps of the two
+    # largest of 4096 normal draws
+    top2 = logits.topk(2, dim=1).values
+    planted = ((top2[:, 0] - top2[:, 1]) > 1.5).sum().item()
+    assert planted == 16
+
+
+def test_scaled_bf16_and_e4m3_variants():
+    c = scaled(CONFIGS[4], n_seq=2, n_slots=2, d=128, V=1000)
+    wl = generate(c)
+    assert wl.weight.dtype == torch.float8_e4m3fn and wl.weight_scale.shape == (1000,)
+    deq = wl.weight.float() * wl.weight_scale[:, None]
+    assert torch.all(deq.abs().amax(dim=1) > 0)
+    # the largest code of every row is 448 (absmax / 448 scaling)
+    assert torch.all(wl.weight.float().abs().amax(dim=1) == 448.0)
+    assert wl.hidden.dtype == torch.bfloat16
+    flags = wl.block_flags.view(2, 2)
+    assert flags[:, 0].tolist() == [ACTIVE | FALLBACK_ELIGIBLE] * 2
+    assert flags[:, 1].tolist() == [ACTIVE] * 2
+
+
+def test_mask_fraction_is_close_to_the_stated_rate():
+    c = scaled(CONFIGS[1], d=8, V=64)
+    wl = generate(c)
+    frac = wl.pos_masked.float().mean().item()
+    assert abs(frac - 0.6) < 0.07

@@ -1,0 +1,174 @@
+"""Draw one synthetic commit-step input from a seeded torch CPU generator.
+
+Draw order (fixed, so a seed names one input): the masked-position flags,
+then the hidden states, then the LM-head weights, then the planted boosts.
+
+A planted boost of size b on vocabulary entry v at position p moves the
+hidden state along that entry's weight row,
+    h_p <- h_p + b * w_v / ||w_v||^2      (fp32, then rounded to the stored dtype)
+which raises that position's logit for v by about b.  It is part of building
+the input only: whatever values end up stored are what both the oracle and
+the CUDA library read.
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass
+from typing import Optional, Tuple
+
+import torch
+
+from .configs import WorkloadConfig
+
+ACTIVE = 1  # block_flags bit 0: the slot holds an active block
+FALLBACK_ELIGIBLE = 2  # block_flags bit 1: the block may take the top-1 fallback
+
+_TORCH_DTYPE = {"f32": torch.float32, "bf16": torch.bfloat16}
+
+
+@dataclass
+class Workload:
+    cfg: WorkloadConfig
+    hidden: torch.Tensor  # [P, d], float32 or bfloat16
+    weight: torch.Tensor  # [V, d], float32, bfloat16 or float8_e4m3fn
+    weight_scale: Optional[torch.Tensor]  # [V] float32 for e4m3 weights, else None
+    pos_masked: torch.Tensor  # [P] uint8, 1 = still masked
+    block_flags: torch.Tensor  # [n_seq * n_slots] uint8
+    tau: Tuple[float, ...]
+    mask_token_id: int
+
+    @property
+    def P(self) -> int:
+        return self.cfg.P
+
+    def to(self, device) -> "Workload":
+        return Workload(
+            cfg=self.cfg,
+            hidden=self.hidden.to(device),
+            weight=self.weight.to(device),
+            weight_scale=None if self.weight_scale is None else self.weight_scale.to(device),
+            pos_masked=self.pos_masked.to(device),
+            block_flags=self.block_flags.to(device),
+            tau=self.tau,
+            mask_token_id=self.mask_token_id,
+        )
+
+
+def block_flags_for(cfg: WorkloadConfig) -> torch.Tensor:
+    flags = torch.zeros(cfg.n_seq, cfg.n_slots, dtype=torch.uint8)
+    if cfg.active == "all":
+        flags[:, :] = ACTIVE
+    elif cfg.active == "first_half":
+        flags[:, : max(1, cfg.n_slots // 2)] = ACTIVE
+    else:
+        raise ValueError(cfg.active)
+    if cfg.fallback == "oldest":
+        flags[:, 0] |= FALLBACK_ELIGIBLE
+    elif cfg.fallback == "all":
+        flags |= FALLBACK_ELIGIBLE
+    elif cfg.fallback != "none":
+        raise ValueError(cfg.fallback)
+    # eligibility only means something for active blocks
+    flags[(flags & ACTIVE) == 0] = 0
+    return flags.reshape(-1).contiguous()
+
+
+def _realised_rows(weight_stored: torch.Tensor, scale: Optional[torch.Tensor], rows: torch.Tensor) -> torch.Tensor:
+    w = weight_stored[rows].float()
+    if scale is not None:
+        w = w * scale[rows, None]
+    return w
+
+
+def generate(cfg: WorkloadConfig) -> Workload:
+    """Build the seeded input of ``cfg`` on the host (CPU tensors)."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(cfg.seed)
+    P, d, V = cfg.P, cfg.d, cfg.V
+
+    # 1. masked-position flags
+    if cfg.mask_frac >= 1.0:
+        pos_masked = torch.ones(P, dtype=torch.uint8)
+    elif cfg.mask_frac <= 0.0:
+        pos_masked = torch.zeros(P, dtype=torch.uint8)
+    else:
+        pos_masked = (torch.rand(P, generator=g) < cfg.mask_frac).to(torch.uint8)
+    block_flags = block_flags_for(cfg)
+
+    # 2. hidden states, N(0, 1)
+    hidden = torch.randn(P, d, generator=g, dtype=torch.float32)
+
+    # 3. LM-head weights, N(0, 1/d), stored [V, d]
+    weight = torch.randn(V, d, generator=g, dtype=torch.float32)
+    weight.mul_(1.0 / math.sqrt(d))
+    scale = None
+    if cfg.weight_dtype == "f32":
+        stored = weight
+    elif cfg.weight_dtype == "bf16":
+        stored = weight.to(torch.bfloat16)
+    elif cfg.weight_dtype == "e4m3":
+        # per-output-channel scale from the row's absolute maximum; 448 is the
+        # largest finite e4m3 value; conversion rounds to nearest even
+        absmax = weight.abs().amax(dim=1)
+        scale = (absmax / 448.0).to(torch.float32)
+        stored = torch.empty(V, d, dtype=torch.float8_e4m3fn)
+        step = 8192
+        for r0 in range(0, V, step):
+            r1 = min(V, r0 + step)
+            stored[r0:r1] = (weight[r0:r1] / scale[r0:r1, None]).to(torch.float8_e4m3fn)
+    else:
+        raise ValueError(cfg.weight_dtype)
+    del weight
+
+    # 4. planted boosts
+    if cfg.boost != "none":
+        _plant(cfg, g, hidden, stored, scale)
+
+    hidden = hidden.to(_TORCH_DTYPE[cfg.hidden_dtype]).contiguous()
+    return Workload(
+        cfg=cfg,
+        hidden=hidden,
+        weight=stored.contiguous(),
+        weight_scale=scale,
+        pos_masked=pos_masked,
+        block_flags=block_flags,
+        tau=tuple(float(t) for t in cfg.tau),
+        mask_token_id=cfg.mask_token_id,
+    )
+
+
+def _plant(cfg, g, hidden, stored, scale):
+    P, V = cfg.P, cfg.V
+    if cfg.boost == "fixed_half":
+        n = int(round(P * cfg.boost_frac))
+        pos = torch.randperm(P, generator=g)[:n]
+        cols = torch.randint(0, V, (n,), generator=g)
+        b = torch.full((n,), float(cfg.boost_lo))
+        _add(hidden, stored, scale, pos, cols, b)
+        return
+    u = torch.rand(P, generator=g)
+    b = cfg.boost_lo + (cfg.boost_hi - cfg.boost_lo) * torch.rand(P, generator=g)
+    col1 = torch.randint(0, V, (P,), generator=g)
+    col2 = torch.randint(0, V - 1, (P,), generator=g)
+    col2 = col2 + (col2 >= col1).to(col2.dtype)  # distinct from col1
+    if cfg.boost == "single":
+        pos = torch.nonzero(u < cfg.boost_frac).reshape(-1)
+        _add(hidden, stored, scale, pos, col1[pos], b[pos])
+    elif cfg.boost == "tied_mix":
+        tied = torch.nonzero(u < 0.3).reshape(-1)
+        single = torch.nonzero((u >= 0.3) & (u < 0.6)).reshape(-1)
+        _add(hidden, stored, scale, tied, col1[tied], b[tied])
+        _add(hidden, stored, scale, tied, col2[tied], b[tied])
+        _add(hidden, stored, scale, single, col1[single], b[single])
+    else:
+        raise ValueError(cfg.boost)
+
+
+def _add(hidden, stored, scale, pos, cols, b, chunk=4096):
+    for i in range(0, pos.numel(), chunk):
+        p = pos[i : i + chunk]
+        c = cols[i : i + chunk]
+        w = _realised_rows(stored, scale, c)
+        nrm2 = (w * w).sum(dim=1, keepdim=True)
+        hidden[p] += b[i : i + chunk, None] * w / nrm2
