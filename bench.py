@@ -1,0 +1,453 @@
+"""Throughput of the fused commit step (LM head + mask-suppressed softmax
+confidence + multi-threshold commit) on GB300, as masked positions per second.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--config NAME] [--graph]
+
+One step = one bd_commit_step over one window of the workload (compaction,
+packing, LM head with the online softmax epilogue, merge and commit for the
+whole threshold grid). With N > 1 (torchrun, one rank per GPU) every rank
+runs its own independent window: the step shards by sequence with no data
+exchange, so scaling is weak. Rank 0 prints one JSON line.
+
+The reference arm (--impl reference) times the float64 CPU oracle on the
+host cores, one bounded sample of whole blocks per step.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from workloads import CONFIGS, by_name, generate  # noqa: E402
+
+DEFAULT_CONFIG = CONFIGS[1].name
+METRIC = "masked positions/s through fused LM-head+confidence+commit"
+UNIT = "positions/s"
+KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_tc.cu", "paper_2609_33887_gb300/csrc/common.cuh"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_tc_traffic.txt")
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default=DEFAULT_CONFIG)
+    ap.add_argument("--graph", action="store_true", help="replay each step as a captured CUDA graph")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# --------------------------------------------------------------- helpers --
+def timing_events(n, stream):
+    """n (begin, end) pairs of timing events whose CUDA handles exist (torch
+    creates them lazily, at the first record)."""
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for a, b in evs:
+        a.record(stream)
+        b.record(stream)
+    return evs
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained"), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def kernel_hash():
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(config_name):
+    """DRAM bytes per LM-head launch from a committed ncu summary, if it was
+    taken on the current kernel source for this workload; else None."""
+    if not os.path.exists(TRAFFIC_FILE):
+        return None
+    rec = {}
+    with open(TRAFFIC_FILE) as f:
+        for line in f:
+            if ":" in line and not line.startswith("#"):
+                k, v = line.split(":", 1)
+                rec[k.strip()] = v.strip()
+    if rec.get("kernel_sha256_16") != kernel_hash() or rec.get("workload") != config_name:
+        return None
+    try:
+        return float(rec["dram_bytes_per_launch"])
+    except (KeyError, ValueError):
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        import tempfile
+
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.FIELDS, "--format=csv,noheader,nounits",
+                 "-lms", "50"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.1)
+        self.proc.terminate()
+        self.proc.wait()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        mx = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower().startswith("active")})
+        loaded = [x for x in sm if mx and x >= 0.3 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows),
+                "power_w_max": max((float(r[3]) for r in rows if r[3].replace(".", "").isdigit()), default=None)}
+
+
+def algorithmic(cfg, n_masked):
+    """Algorithmic work of one step: 2*N*d*V FLOPs, and the bytes the method
+    must move: the head once, the masked hidden rows, 12 B of outputs and 1 B
+    of mask per position (logits are never stored)."""
+    wbytes = {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype]
+    hbytes = {"f32": 4, "bf16": 2}[cfg.hidden_dtype]
+    flops = 2.0 * n_masked * cfg.d * cfg.V
+    bytes_ = cfg.V * cfg.d * wbytes + (cfg.V * 4 if cfg.weight_dtype == "e4m3" else 0) \
+        + n_masked * cfg.d * hbytes + cfg.P * 13
+    return flops, bytes_
+
+
+# ----------------------------------------------------------- oracle timing --
+def oracle_sample_time(wl, n_blocks, seed=7, w64=None):
+    """Time the oracle on a sample of whole blocks; returns (seconds, masked positions)."""
+    import oracle
+    from workloads.rawio import dtype_tag, raw_numpy
+
+    cfg = wl.cfg
+    rng = np.random.default_rng(seed)
+    blocks = sorted(rng.choice(cfg.n_blocks, size=min(n_blocks, cfg.n_blocks), replace=False).tolist())
+    if w64 is None:
+        w64 = oracle.weights_f64(raw_numpy(wl.weight), dtype_tag(wl.weight),
+                                 None if wl.weight_scale is None else raw_numpy(wl.weight_scale))
+    hid = raw_numpy(wl.hidden)
+    pm = raw_numpy(wl.pos_masked)
+    bf = raw_numpy(wl.block_flags)
+    t0 = time.perf_counter()
+    out = oracle.commit_step(hid, dtype_tag(wl.hidden), w64, "f64", None, pm, bf, cfg.n_seq, cfg.n_slots,
+                             cfg.block_len, wl.mask_token_id, wl.tau, blocks=blocks)
+    dt = time.perf_counter() - t0
+    return dt, int((out["tokens"] >= 0).sum()), blocks, w64
+
+
+def cores_used():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+# ---------------------------------------------------------- reference arm --
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    cfg = by_name(args.config)
+    wl = generate(cfg)
+    # per step: whole blocks, sized so that warmup + steps stay within a few minutes
+    _, _, _, w64 = oracle_sample_time(wl, 1)
+    t1, n1, _, _ = oracle_sample_time(wl, 1, w64=w64)
+    budget = 150.0
+    per_step = budget / max(1, args.steps + args.warmup)
+    n_blocks = max(1, min(cfg.n_blocks, int(per_step / max(t1, 1e-3))))
+    for i in range(args.warmup):
+        oracle_sample_time(wl, n_blocks, seed=100 + i, w64=w64)
+    tot_t, tot_n = 0.0, 0
+    for i in range(args.steps):
+        dt, n, _, _ = oracle_sample_time(wl, n_blocks, seed=1000 + i, w64=w64)
+        tot_t += dt
+        tot_n += n
+    value = tot_n / tot_t if tot_t > 0 else 0.0
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
+                   "d": cfg.d, "V": cfg.V, "T": len(cfg.tau)},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                         "sample": f"{n_blocks} whole block(s) per step of {cfg.name}; head decoded to float64 "
+                                   "once, outside the timed steps"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------- our arm --
+def run_ours(args):
+    import paper_2609_33887_gb300 as bdc
+    from paper_2609_33887_gb300 import bdcommit as B
+
+    rank, world, local = dist_env()
+    if not torch.cuda.is_available():
+        raise SystemExit("bench.py needs a CUDA device (no CPU fallback)")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    pg = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=dev)
+        pg = dist
+    bdc.load_library()
+
+    cfg = by_name(args.config)
+    # each rank serves its own window (independent sequences): weak scaling
+    from dataclasses import replace
+
+    wl_host = generate(replace(cfg, seed=cfg.seed + 1000 * rank) if rank else cfg)
+    wl = wl_host.to(dev)
+    P, T = cfg.P, len(cfg.tau)
+    n_masked = int(((wl_host.pos_masked != 0) &
+                    (torch.repeat_interleave(wl_host.block_flags & 1, cfg.block_len) != 0)).sum())
+    stream = torch.cuda.current_stream()
+    ws_bytes = bdc.bd_workspace_size(wl.hidden, wl.weight, wl.weight_scale, wl.pos_masked, wl.block_flags,
+                                     cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau)
+    workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
+    tokens = torch.empty(P, dtype=torch.int32, device=dev)
+    conf = torch.empty(P, dtype=torch.float32, device=dev)
+    commit = torch.empty(P, dtype=torch.int32, device=dev)
+    counts = torch.empty((cfg.n_seq, T), dtype=torch.int32, device=dev)
+
+    def step(h=None, ev=None):
+        rc = B.bd_commit_step_ex(wl.hidden if h is None else h, wl.weight, wl.weight_scale, wl.pos_masked,
+                                 wl.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
+                                 cfg.tau, tokens, conf, commit, stream=stream, workspace=workspace,
+                                 out_counts=counts, lmhead_events=ev)
+        if rc != 0:
+            raise B.BdError(rc)
+
+    launches_per_step = 4 + (1 if cfg.weight_dtype == "e4m3" else 0)
+    K, W = args.steps, args.warmup
+    for _ in range(W):
+        step()
+    torch.cuda.synchronize()
+    st = B.bd_get_device_status(stream)
+    if st != 0:
+        raise B.BdError(st, "warm-up")
+
+    graph = None
+    if args.graph:
+        graph = torch.cuda.CUDAGraph()
+        ev_g = timing_events(1, stream)[0]
+        with torch.cuda.graph(graph, stream=stream):
+            step(ev=ev_g)
+        graph.replay()
+        torch.cuda.synchronize()
+
+    # ---- device-resident timed region
+    evs = timing_events(K, stream)
+    lm_ms = []
+    vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x]
+    sampler = ClockSampler(vis[local] if local < len(vis) else str(local))
+    sampler.start()
+    if pg:
+        pg.barrier()
+    torch.cuda.synchronize()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    if graph is None:
+        for i in range(K):
+            step(ev=evs[i])
+    else:
+        for i in range(K):
+            graph.replay()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    clocks = sampler.stop()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    if graph is None:
+        lm_ms = [a.elapsed_time(b) for a, b in evs]
+    else:
+        # one extra replay timed alone for the LM-head events inside the graph
+        lm_ms = []
+        for _ in range(min(K, 50)):
+            graph.replay()
+            torch.cuda.synchronize()
+            lm_ms.append(ev_g[0].elapsed_time(ev_g[1]))
+    st = B.bd_get_device_status(stream)
+    if st != 0:
+        raise B.BdError(st, "timed region")
+    if pg:
+        t = torch.tensor([elapsed_ms], device=dev)
+        pg.all_reduce(t, op=pg.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+        nm = torch.tensor([float(n_masked)], device=dev)
+        pg.all_reduce(nm, op=pg.ReduceOp.SUM)
+        total_masked = float(nm.item())
+    else:
+        total_masked = float(n_masked)
+    ms_per_step = elapsed_ms / K
+    value = total_masked * K / (elapsed_ms / 1e3)
+
+    # ---- end to end through the public call with host buffers
+    e2e = None
+    if not args.no_e2e:
+        h_host = wl_host.hidden.pin_memory()
+        pm_host = wl_host.pos_masked.pin_memory()
+        bf_host = wl_host.block_flags.pin_memory()
+        out_host = [torch.empty(P, dtype=torch.int32).pin_memory(), torch.empty(P, dtype=torch.float32).pin_memory(),
+                    torch.empty(P, dtype=torch.int32).pin_memory(),
+                    torch.empty((cfg.n_seq, T), dtype=torch.int32).pin_memory()]
+        h_dev = torch.empty_like(wl.hidden)
+
+        def e2e_step():
+            h_dev.copy_(h_host, non_blocking=True)
+            wl.pos_masked.copy_(pm_host, non_blocking=True)
+            wl.block_flags.copy_(bf_host, non_blocking=True)
+            step(h=h_dev)
+            for o, d_ in zip(out_host, (tokens, conf, commit, counts)):
+                o.copy_(d_, non_blocking=True)
+
+        for _ in range(W):
+            e2e_step()
+        torch.cuda.synchronize()
+        if pg:
+            pg.barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(K):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e_ms = e0.elapsed_time(e1)
+        if pg:
+            t = torch.tensor([e_ms], device=dev)
+            pg.all_reduce(t, op=pg.ReduceOp.MAX)
+            e_ms = float(t.item())
+        h2d = h_host.numel() * h_host.element_size() + pm_host.numel() + bf_host.numel()
+        d2h = sum(o.numel() * o.element_size() for o in out_host)
+        e2e = {"value": total_masked * K / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h),
+               "note": "pinned host hidden states + mask state in, tokens/conf/commit/counts out, per step; "
+                       "LM-head weights stay resident in HBM"}
+
+    # ---- roofline of the dominant kernel (LM head)
+    hbm_gbs, tc_tflops, tc_sus, peak_src = peaks()
+    flops, abytes = algorithmic(cfg, n_masked)
+    lm_avg_s = statistics.mean(lm_ms) / 1e3
+    t_tc = flops / (tc_tflops * 1e12)
+    t_hbm = abytes / (hbm_gbs * 1e9)
+    traffic = recorded_traffic(cfg.name)
+    if t_tc >= t_hbm:
+        achieved = flops / lm_avg_s / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": tc_tflops, "unit": "TFLOP/s",
+                "frac": achieved / tc_tflops, "traffic": traffic,
+                "peak_source": f"bf16_tflops (burst) of {peak_src}",
+                "frac_of_sustained": (achieved / tc_sus) if tc_sus else None}
+    else:
+        achieved = abytes / lm_avg_s / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
+                "frac": achieved / hbm_gbs, "traffic": traffic, "peak_source": f"hbm_gbs of {peak_src}"}
+    roof["lmhead_ms_avg"] = lmhead_ms = statistics.mean(lm_ms)
+    roof["hbm_view"] = {"algorithmic_bytes": abytes, "achieved_gbs": abytes / lm_avg_s / 1e9,
+                        "frac": abytes / lm_avg_s / 1e9 / hbm_gbs}
+    roof["algorithmic_flops"] = flops
+    roof["kernel_sha256_16"] = kernel_hash()
+
+    # ---- CPU baseline: the oracle on a bounded sample, rank 0 at N = 1 only
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        dt, n, blocks, w64 = oracle_sample_time(wl_host, 2)
+        target = 15.0
+        nb = max(1, min(cfg.n_blocks, int(2 * target / max(dt, 1e-3))))
+        dt, n, blocks, _ = oracle_sample_time(wl_host, nb, w64=w64)
+        cpu = {"value": n / dt, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+               "sample": f"{len(blocks)} whole blocks ({n} masked positions) of {cfg.name}, {dt:.1f} s; "
+                         "head decoded to float64 once outside the timed call"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
+            "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if cfg.weight_dtype == "bf16" else ("e4m3xbf16" if cfg.weight_dtype == "e4m3" else "f32"),
+            "data": "synthetic",
+            "config": {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
+                       "masked_positions_per_rank": n_masked, "d": cfg.d, "V": cfg.V, "T": len(cfg.tau),
+                       "parallelism": f"independent windows x{world}", "graph": bool(args.graph),
+                       "l2": "inputs larger than L2 (the LM head is %.0f MB, read every step)"
+                             % (cfg.V * cfg.d * {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype] / 1e6)},
+            "roofline": roof,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step * K,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    if pg:
+        pg.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

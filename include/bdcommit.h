@@ -1,0 +1,194 @@
+/*
+ * bdcommit: the per-forward commit step of a multi-block diffusion LM engine
+ * on one GB300 (sm_103a).
+ *
+ * One call takes the final hidden state of every position in the engine's
+ * window of block slots, and for every still-masked position of every active
+ * block:
+ *   1. projects it through the LM head          logits = W_head . h
+ *   2. reads the mask-suppressed softmax         conf = max_v softmax(logits)_v,
+ *      that the engine commits from                token = argmax_v (lowest v on ties)
+ *      (App. B.1, "Entropy of the deeper blocks")
+ *   3. applies the accept threshold              commit when conf >= tau
+ *      ("at or above the accept threshold", Sec. 3.1 and App. B.1), with the
+ *      per-block top-1 fallback when no position clears it (App. B.2,
+ *      self-distillation protocol), once for every tau of a grid, so one
+ *      forward scores a whole grid of operating points (App. F.3).
+ * Logits never reach device memory: the LM-head kernel reduces each row to a
+ * running (max, sum of exponentials, argmax) while it multiplies.
+ *
+ * Conventions for every entry point below
+ *   - All tensors are caller-owned. Device pointers must stay valid until the
+ *     work queued on the stream has finished; the library keeps no reference.
+ *   - Calls are asynchronous on the given stream and never synchronise the
+ *     host, except bd_get_device_status (documented there).
+ *   - Return value: 0 (BD_OK) or a negative bd_status. Argument checks happen
+ *     before any CUDA call, so a rejected call has queued nothing. The library
+ *     never traps, aborts or exits.
+ *   - Position p of the window is p = (s * n_slots + b) * block_len + j for
+ *     sequence s, slot b and offset j in the block.
+ */
+#ifndef BDCOMMIT_H
+#define BDCOMMIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---------------------------------------------------------------- status */
+typedef enum {
+  BD_OK = 0,
+  BD_ERR_NULL = -1,      /* a required pointer is NULL */
+  BD_ERR_SHAPE = -2,     /* sizes disagree or are out of range */
+  BD_ERR_DTYPE = -3,     /* unsupported dtype or dtype combination */
+  BD_ERR_ALIGN = -4,     /* pointer or row stride misaligned (see bd_weight) */
+  BD_ERR_TAU = -5,       /* T outside 1..32, NULL grid, or a NaN threshold */
+  BD_ERR_WORKSPACE = -6, /* caller workspace smaller than bd_workspace_size */
+  BD_ERR_CUDA = -7,      /* a CUDA runtime call or kernel launch failed */
+  BD_ERR_TIMEOUT = -8,   /* a bounded device-side wait gave up (see bd_get_device_status) */
+  BD_ERR_DEVICE = -9,    /* the current device cannot run this library (needs sm_103) */
+  BD_ERR_ARG = -10       /* other invalid argument (mask_token_id, variant, flags) */
+} bd_status;
+
+/* ----------------------------------------------------------------- dtypes */
+typedef enum {
+  BD_F32 = 0,  /* IEEE binary32 */
+  BD_BF16 = 1, /* bfloat16 */
+  BD_E4M3 = 2  /* FP8 E4M3 (OCP "fn" variant: no infinities), weights only */
+} bd_dtype;
+
+/* Block flag bits (bd_mask_state.block_flags). */
+#define BD_BLOCK_ACTIVE 1u            /* the slot holds an active block (App. F) */
+#define BD_BLOCK_FALLBACK_ELIGIBLE 2u /* the block may take the top-1 fallback (App. B.2) */
+
+/* Hidden states of the whole window: [rows, cols] row-major, device memory.
+ *   rows  = P = n_seq * n_slots * block_len (every slot, placeholders too:
+ *           the engine forwards the whole window, App. F)
+ *   cols  = d, the model width
+ *   ld    = elements between consecutive rows (>= cols)
+ *   dtype = BD_F32 or BD_BF16. With BD_BF16 the pointer must be 16-byte
+ *           aligned and ld * 2 a multiple of 16. */
+typedef struct {
+  const void* data;
+  int32_t dtype;
+  int64_t rows;
+  int64_t cols;
+  int64_t ld;
+} bd_hidden;
+
+/* LM-head weights [vocab, dim] row-major (one row per vocabulary entry, the
+ * K-major layout of an nn.Linear head), device memory.
+ *   dtype BD_F32  : with BD_F32 hidden states (exact fp32 SIMT path).
+ *   dtype BD_BF16 : with BD_BF16 hidden states (tensor-core path).
+ *   dtype BD_E4M3 : with BD_BF16 hidden states; `scale` is a device float32
+ *                   array [vocab] and the weight of row v is code * scale[v]
+ *                   (per-output-channel scaling, the FP8 precision lever).
+ *   For BD_BF16 / BD_E4M3 the pointer must be 16-byte aligned and
+ *   ld * element size a multiple of 16 (TMA row stride rule). */
+typedef struct {
+  const void* data;
+  int32_t dtype;
+  int64_t vocab;
+  int64_t dim;
+  int64_t ld;
+  const float* scale; /* required iff dtype == BD_E4M3, else ignored */
+} bd_weight;
+
+/* Which positions are still masked and which slots hold active blocks
+ * (the engine's fixed-slot block buffer, App. F). Device memory.
+ *   pos_masked [n_seq * n_slots * block_len] : 1 = still masked, 0 = resolved
+ *   block_flags[n_seq * n_slots]             : BD_BLOCK_* bits
+ *   block_len in 1..64 (the paper's engine uses 32)
+ *   mask_token_id: -1 = no suppression; else in [0, vocab): that entry is
+ *                  removed from the softmax and can never be the token. */
+typedef struct {
+  int32_t n_seq;
+  int32_t n_slots;
+  int32_t block_len;
+  int32_t mask_token_id;
+  const uint8_t* pos_masked;
+  const uint8_t* block_flags;
+} bd_mask_state;
+
+/* Threshold grid: HOST array tau[0..T-1], 1 <= T <= 32, no NaN. Bit k of a
+ * position's commit mask answers "does this position commit at tau[k]". The
+ * values are copied at call time; the array may be reused immediately. */
+typedef struct {
+  const float* tau;
+  int32_t T;
+} bd_tau_grid;
+
+/* Execution options.
+ *   stream          : a cudaStream_t (NULL = the legacy default stream).
+ *   workspace       : device scratch of at least bd_workspace_size bytes,
+ *                     256-byte aligned; NULL = a library-owned buffer for the
+ *                     current device, grown with cudaMalloc on demand (not
+ *                     allowed inside CUDA graph capture: pass your own then).
+ *                     One workspace must not be used by two calls that can
+ *                     run at the same time.
+ *   out_counts      : optional device int32 [n_seq * T]; receives, per
+ *                     sequence and threshold, the number of committed
+ *                     positions (the numerator of tokens per forward, Sec. 2.1).
+ *   lmhead_event_begin / lmhead_event_end : optional cudaEvent_t recorded on
+ *                     the stream right before and after the LM-head kernel,
+ *                     for timing it alone.
+ *   variant         : 0 = automatic; 1 = force the fp32-FMA SIMT LM-head
+ *                     kernel; 2 = force the tensor-core kernel (BF16/E4M3 only).
+ *   flags           : reserved, must be 0. */
+typedef struct {
+  void* stream;
+  void* workspace;
+  size_t workspace_bytes;
+  int32_t* out_counts;
+  void* lmhead_event_begin;
+  void* lmhead_event_end;
+  int32_t variant;
+  int32_t flags;
+} bd_exec;
+
+/* The commit step (Sec. 3.1, App. B.1, B.2, F) on the default stream with the
+ * library-owned workspace. Outputs, all device arrays of P entries and all
+ * fully written:
+ *   out_tokens[p] : argmax token of a masked position of an active block, else -1
+ *   out_conf[p]   : its confidence (max softmax probability, in (0, 1]), else 0
+ *   out_commit[p] : bit k set <=> the position commits at tau[k], else 0 */
+int bd_commit_step(const bd_hidden* hidden, const bd_weight* weight,
+                   const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
+                   int32_t* out_tokens, float* out_conf, uint32_t* out_commit);
+
+/* Same as bd_commit_step with explicit execution options (exec may be NULL). */
+int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight,
+                      const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
+                      int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+                      const bd_exec* exec);
+
+/* Bytes of device workspace a call with these arguments needs (0 if the
+ * arguments are invalid). Depends on sizes, dtypes and the current device's
+ * SM count only, not on the data. */
+size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
+                         const bd_mask_state* mask_state, const bd_tau_grid* tau_grid);
+
+/* Synchronises `stream` (a cudaStream_t, NULL = legacy default), then returns
+ * and clears the device-side status of the current device: BD_OK, or
+ * BD_ERR_TIMEOUT if a kernel's bounded wait gave up since the last call (its
+ * outputs are then invalid), or BD_ERR_CUDA if the synchronisation failed. */
+int bd_get_device_status(void* stream);
+
+/* Static English text for a status code. Never NULL. */
+const char* bd_status_string(int status);
+
+/* Frees the library-owned workspaces and status words of every device.
+ * No call may be in flight. */
+int bd_shutdown(void);
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+int bd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BDCOMMIT_H */

@@ -82,7 +82,11 @@ def weights_f64(raw: np.ndarray, dtype: str, scale: Optional[np.ndarray] = None)
     f32 and bf16 rows are used as stored. e4m3 rows are the stored code times
     the row's (output channel's) float32 scale, i.e. exactly the dequantised
     weights the library is handed, not the matrix before quantisation.
+    "f64" rows are values already decoded by this function (a caller that
+    evaluates many samples of one head decodes it once).
     """
+    if dtype == "f64":
+        return np.asarray(raw, dtype=np.float64)
     if dtype == "f32":
         return np.asarray(raw, dtype=np.float32).astype(np.float64)
     if dtype == "bf16":

@@ -1,0 +1,40 @@
+"""GB300-native (sm_103a) commit step of a multi-block diffusion LM engine.
+
+The work happens in libbdcommit.so (include/bdcommit.h); this package holds
+its CUDA sources (csrc/), the in-tree build step (build.py) and the ctypes
+binding (bdcommit.py).
+"""
+
+from . import bdcommit
+from .bdcommit import (
+    BD_BLOCK_ACTIVE,
+    BD_BLOCK_FALLBACK_ELIGIBLE,
+    BD_OK,
+    BdError,
+    bd_commit_step,
+    bd_commit_step_ex,
+    bd_get_device_status,
+    bd_shutdown,
+    bd_status_string,
+    bd_version,
+    bd_workspace_size,
+    commit_step,
+    load_library,
+)
+
+__all__ = [
+    "BD_BLOCK_ACTIVE",
+    "BD_BLOCK_FALLBACK_ELIGIBLE",
+    "BD_OK",
+    "BdError",
+    "bd_commit_step",
+    "bd_commit_step_ex",
+    "bd_get_device_status",
+    "bd_shutdown",
+    "bd_status_string",
+    "bd_version",
+    "bd_workspace_size",
+    "bdcommit",
+    "commit_step",
+    "load_library",
+]

@@ -1,0 +1,238 @@
+"""ctypes binding of libbdcommit (include/bdcommit.h).
+
+Argument marshalling only: torch tensors (device memory, streams) become the
+plain pointers and sizes of the C ABI, and every step of the commit step runs
+in the library's CUDA kernels. There is no fallback: if the shared library is
+missing or cannot be loaded, every entry point raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int, c_int32, c_int64, c_size_t, c_void_p
+from typing import Optional, Sequence
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libbdcommit.so")
+
+# status codes (bd_status)
+BD_OK = 0
+BD_ERR_NULL = -1
+BD_ERR_SHAPE = -2
+BD_ERR_DTYPE = -3
+BD_ERR_ALIGN = -4
+BD_ERR_TAU = -5
+BD_ERR_WORKSPACE = -6
+BD_ERR_CUDA = -7
+BD_ERR_TIMEOUT = -8
+BD_ERR_DEVICE = -9
+BD_ERR_ARG = -10
+
+# dtypes (bd_dtype)
+BD_F32 = 0
+BD_BF16 = 1
+BD_E4M3 = 2
+
+BD_BLOCK_ACTIVE = 1
+BD_BLOCK_FALLBACK_ELIGIBLE = 2
+
+VARIANT_AUTO = 0
+VARIANT_SIMT = 1
+VARIANT_TC = 2
+
+
+class bd_hidden(ctypes.Structure):
+    _fields_ = [("data", c_void_p), ("dtype", c_int32), ("rows", c_int64), ("cols", c_int64), ("ld", c_int64)]
+
+
+class bd_weight(ctypes.Structure):
+    _fields_ = [("data", c_void_p), ("dtype", c_int32), ("vocab", c_int64), ("dim", c_int64), ("ld", c_int64),
+                ("scale", c_void_p)]
+
+
+class bd_mask_state(ctypes.Structure):
+    _fields_ = [("n_seq", c_int32), ("n_slots", c_int32), ("block_len", c_int32), ("mask_token_id", c_int32),
+                ("pos_masked", c_void_p), ("block_flags", c_void_p)]
+
+
+class bd_tau_grid(ctypes.Structure):
+    _fields_ = [("tau", POINTER(c_float)), ("T", c_int32)]
+
+
+class bd_exec(ctypes.Structure):
+    _fields_ = [("stream", c_void_p), ("workspace", c_void_p), ("workspace_bytes", c_size_t),
+                ("out_counts", c_void_p), ("lmhead_event_begin", c_void_p), ("lmhead_event_end", c_void_p),
+                ("variant", c_int32), ("flags", c_int32)]
+
+
+class BdError(RuntimeError):
+    def __init__(self, status: int, where: str = "bd_commit_step"):
+        self.status = status
+        super().__init__(f"{where} failed: {status} ({bd_status_string(status)})")
+
+
+_lib = None
+
+
+def load_library(path: Optional[str] = None) -> ctypes.CDLL:
+    """Load libbdcommit.so (built in-tree by paper_2609_33887_gb300/build.py)."""
+    global _lib
+    if _lib is not None and path is None:
+        return _lib
+    p = path or LIB_PATH
+    if not os.path.exists(p):
+        raise RuntimeError(f"libbdcommit.so not found at {p}: build it first "
+                           "(python -c 'import __graft_entry__ as g; g.build()')")
+    lib = ctypes.CDLL(p)
+    sig = {
+        "bd_commit_step": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                   POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p]),
+        "bd_commit_step_ex": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                      POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, POINTER(bd_exec)]),
+        "bd_workspace_size": (c_size_t, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                         POINTER(bd_tau_grid)]),
+        "bd_get_device_status": (c_int, [c_void_p]),
+        "bd_status_string": (ctypes.c_char_p, [c_int]),
+        "bd_shutdown": (c_int, []),
+        "bd_version": (c_int, []),
+    }
+    for name, (res, args) in sig.items():
+        fn = getattr(lib, name)
+        fn.restype = res
+        fn.argtypes = args
+    if path is None:
+        _lib = lib
+    return lib
+
+
+# ------------------------------------------------------------ marshalling --
+_DT = {torch.float32: BD_F32, torch.bfloat16: BD_BF16, torch.float8_e4m3fn: BD_E4M3}
+
+
+def _ptr(t: Optional[torch.Tensor]) -> Optional[int]:
+    return None if t is None else t.data_ptr()
+
+
+def make_hidden(hidden: torch.Tensor) -> bd_hidden:
+    if hidden.dim() != 2 or hidden.stride(1) != 1:
+        raise ValueError("hidden must be a 2-D tensor with contiguous rows")
+    return bd_hidden(_ptr(hidden), _DT[hidden.dtype], hidden.shape[0], hidden.shape[1], hidden.stride(0))
+
+
+def make_weight(weight: torch.Tensor, scale: Optional[torch.Tensor] = None) -> bd_weight:
+    if weight.dim() != 2 or weight.stride(1) != 1:
+        raise ValueError("weight must be a 2-D [vocab, dim] tensor with contiguous rows")
+    return bd_weight(_ptr(weight), _DT[weight.dtype], weight.shape[0], weight.shape[1], weight.stride(0),
+                     _ptr(scale))
+
+
+def make_mask_state(pos_masked: torch.Tensor, block_flags: torch.Tensor, n_seq: int, n_slots: int,
+                    block_len: int, mask_token_id: int = -1) -> bd_mask_state:
+    if pos_masked.dtype != torch.uint8 or block_flags.dtype != torch.uint8:
+        raise ValueError("pos_masked and block_flags must be uint8")
+    if not (pos_masked.is_contiguous() and block_flags.is_contiguous()):
+        raise ValueError("pos_masked and block_flags must be contiguous")
+    return bd_mask_state(n_seq, n_slots, block_len, mask_token_id, _ptr(pos_masked), _ptr(block_flags))
+
+
+def make_tau_grid(tau: Sequence[float]):
+    arr = (c_float * max(1, len(tau)))(*[float(t) for t in tau])
+    return bd_tau_grid(ctypes.cast(arr, POINTER(c_float)), len(tau)), arr
+
+
+def _stream_handle(stream) -> Optional[int]:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+# ------------------------------------------------------------ entry points --
+def bd_status_string(status: int) -> str:
+    return load_library().bd_status_string(int(status)).decode()
+
+
+def bd_version() -> int:
+    return int(load_library().bd_version())
+
+
+def bd_shutdown() -> int:
+    return int(load_library().bd_shutdown())
+
+
+def bd_get_device_status(stream=None) -> int:
+    return int(load_library().bd_get_device_status(_stream_handle(stream)))
+
+
+def bd_workspace_size(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                      mask_token_id, tau) -> int:
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    return int(load_library().bd_workspace_size(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms),
+                                                ctypes.byref(tg)))
+
+
+def bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                      mask_token_id, tau, out_tokens, out_conf, out_commit, *, stream=None, workspace=None,
+                      out_counts=None, lmhead_events=None, variant=VARIANT_AUTO) -> int:
+    """Queue one commit step on `stream` (default: torch's current stream).
+
+    All tensors are device tensors; `tau` is a host sequence of floats.
+    Returns the bd_status code (0 on success)."""
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    ex = bd_exec()
+    ex.stream = _stream_handle(stream)
+    if workspace is not None:
+        ex.workspace = workspace.data_ptr()
+        ex.workspace_bytes = workspace.numel() * workspace.element_size()
+    ex.out_counts = _ptr(out_counts)
+    if lmhead_events is not None:
+        ex.lmhead_event_begin = lmhead_events[0].cuda_event
+        ex.lmhead_event_end = lmhead_events[1].cuda_event
+    ex.variant = variant
+    ex.flags = 0
+    return int(load_library().bd_commit_step_ex(
+        ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+        _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit), ctypes.byref(ex)))
+
+
+def bd_commit_step(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                   mask_token_id, tau, out_tokens, out_conf, out_commit) -> int:
+    """bd_commit_step: default stream, library-owned workspace."""
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    return int(load_library().bd_commit_step(
+        ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+        _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit)))
+
+
+def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_len, tau, *,
+                weight_scale=None, mask_token_id=-1, stream=None, workspace=None, counts=False,
+                variant=VARIANT_AUTO, lmhead_events=None):
+    """Allocate the outputs on the hidden states' device, queue the step, raise on error.
+
+    Returns (tokens int32 [P], conf float32 [P], commit int32 [P] holding the
+    uint32 bit masks, counts int32 [n_seq, T] or None)."""
+    P = n_seq * n_slots * block_len
+    dev = hidden.device
+    tokens = torch.empty(P, dtype=torch.int32, device=dev)
+    conf = torch.empty(P, dtype=torch.float32, device=dev)
+    commit = torch.empty(P, dtype=torch.int32, device=dev)
+    cnt = torch.empty((n_seq, len(tau)), dtype=torch.int32, device=dev) if counts else None
+    rc = bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                           mask_token_id, tau, tokens, conf, commit, stream=stream, workspace=workspace,
+                           out_counts=cnt, lmhead_events=lmhead_events, variant=variant)
+    if rc != BD_OK:
+        raise BdError(rc)
+    return tokens, conf, commit, cnt

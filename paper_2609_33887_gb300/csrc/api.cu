@@ -1,0 +1,419 @@
+// Host side of the C ABI declared in include/bdcommit.h: argument checks,
+// the workspace plan, TMA descriptors and the launch sequence of one commit
+// step on the caller's stream.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/bdcommit.h"
+#include "kernels.h"
+
+namespace {
+
+using bd::BandPlan;
+
+constexpr int MAX_DEVICES = 64;
+constexpr int64_t MAX_POSITIONS = int64_t(1) << 24;
+constexpr int64_t MAX_VOCAB = int64_t(1) << 30;
+constexpr int64_t MAX_DIM = int64_t(1) << 20;
+
+struct DevCtx {
+  bool ready = false;
+  int sm_count = 0;
+  uint32_t* status = nullptr;  // device status word (bd::DEV_* bits)
+  void* ws = nullptr;          // library-owned workspace
+  size_t ws_bytes = 0;
+};
+
+std::mutex g_mu;
+DevCtx g_dev[MAX_DEVICES];
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+int device_ctx(DevCtx** out, int* dev_out = nullptr) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BD_ERR_CUDA;
+  if (dev < 0 || dev >= MAX_DEVICES) return BD_ERR_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  DevCtx& c = g_dev[dev];
+  if (!c.ready) {
+    int maj = 0, mnr = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&mnr, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return BD_ERR_CUDA;
+    if (maj != 10 || mnr != 3) return BD_ERR_DEVICE;  // the kernels are built for sm_103a only
+    if (g_encode == nullptr) {
+      cudaDriverEntryPointQueryResult q;
+      void* fn = nullptr;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return BD_ERR_CUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    if (cudaMalloc(&c.status, 256) != cudaSuccess) return BD_ERR_CUDA;
+    if (cudaMemset(c.status, 0, 256) != cudaSuccess) return BD_ERR_CUDA;
+    c.sm_count = sms;
+    c.ready = true;
+  }
+  *out = &c;
+  if (dev_out) *dev_out = dev;
+  return BD_OK;
+}
+
+// ---------------------------------------------------------------- checks --
+struct Call {
+  int64_t P, d, V;
+  int n_seq, n_slots, L, n_blocks, mask_id, T;
+  int hdt, wdt;
+  bool tc;          // tensor-core LM head
+  int64_t ldh, ldw;
+  int64_t ldc;      // packed hidden rows (bf16), elements
+  int64_t ldq;      // decoded e4m3 head (bf16), elements
+};
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }
+
+int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
+
+int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, const bd_tau_grid* tg,
+               int variant, Call* c) {
+  if (!h || !w || !ms || !tg) return BD_ERR_NULL;
+  if (!tg->tau) return BD_ERR_TAU;
+  if (tg->T < 1 || tg->T > 32) return BD_ERR_TAU;
+  for (int k = 0; k < tg->T; ++k)
+    if (std::isnan(tg->tau[k])) return BD_ERR_TAU;
+  if (variant < 0 || variant > 2) return BD_ERR_ARG;
+  if (ms->n_seq < 0 || ms->n_slots < 1 || ms->block_len < 1 || ms->block_len > 64) return BD_ERR_SHAPE;
+  const int64_t n_blocks = int64_t(ms->n_seq) * ms->n_slots;
+  const int64_t P = n_blocks * ms->block_len;
+  if (P > MAX_POSITIONS) return BD_ERR_SHAPE;
+  if (h->rows != P) return BD_ERR_SHAPE;
+  if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
+  if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
+  if (h->ld < h->cols || w->ld < w->dim) return BD_ERR_SHAPE;
+  if (ms->mask_token_id < -1 || ms->mask_token_id >= w->vocab) return BD_ERR_ARG;
+  if (ms->mask_token_id >= 0 && w->vocab < 2) return BD_ERR_SHAPE;  // nothing left to predict
+  const int hdt = h->dtype, wdt = w->dtype;
+  const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
+  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3);
+  if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
+  const bool tc = variant == 2 || (variant == 0 && combo_bf16);
+  if (tc && !combo_bf16) return BD_ERR_DTYPE;
+  if (P > 0) {
+    if (!h->data || !w->data || !ms->pos_masked || !ms->block_flags) return BD_ERR_NULL;
+    if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
+  }
+  if (tc) {
+    if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
+    if (!aligned(w->data, 16) || (w->ld * esize(wdt)) % 16 != 0) return BD_ERR_ALIGN;
+  } else {
+    if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
+  }
+  if (w->scale && wdt == BD_E4M3 && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  c->P = P;
+  c->d = w->dim;
+  c->V = w->vocab;
+  c->n_seq = ms->n_seq;
+  c->n_slots = ms->n_slots;
+  c->L = ms->block_len;
+  c->n_blocks = static_cast<int>(n_blocks);
+  c->mask_id = ms->mask_token_id;
+  c->T = tg->T;
+  c->hdt = hdt;
+  c->wdt = wdt;
+  c->tc = tc;
+  c->ldh = h->ld;
+  c->ldw = w->ld;
+  c->ldc = round_up(c->d, 8);
+  c->ldq = round_up(c->d, 8);
+  return BD_OK;
+}
+
+// ------------------------------------------------------------- the plan --
+int env_int(const char* name, int dflt, int lo, int hi) {
+  const char* s = std::getenv(name);
+  if (!s || !*s) return dflt;
+  int v = std::atoi(s);
+  return v < lo ? lo : v > hi ? hi : v;
+}
+
+BandPlan make_plan(const Call& c, int sm_count) {
+  BandPlan p;
+  if (c.tc) {
+    p.BM = bd::TC_BM;
+    p.BN = bd::TC_BN;
+    p.G = sm_count;
+    p.GM = env_int("BD_TC_GM", 8, 1, sm_count);
+  } else {
+    p.BM = bd::SIMT_BM;
+    p.BN = bd::SIMT_BN;
+    p.G = 2 * sm_count;
+    p.GM = 8;
+  }
+  p.n_vt = static_cast<int>((c.V + p.BN - 1) / p.BN);
+  return p;
+}
+
+struct Layout {
+  size_t hdr, idx, rowpos, pm, ps, pa, hc, wq, total;
+};
+
+Layout make_layout(const Call& c, const BandPlan& p) {
+  Layout l{};
+  size_t off = 0;
+  auto take = [&off](size_t bytes, size_t align) {
+    off = (off + align - 1) / align * align;
+    size_t o = off;
+    off += bytes;
+    return o;
+  };
+  const size_t P = static_cast<size_t>(c.P);
+  const size_t slots = static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
+  l.hdr = take(256, 256);
+  l.idx = take(4 * P, 256);
+  l.rowpos = take(4 * P, 256);
+  l.pm = take(4 * slots * P, 256);
+  l.ps = take(4 * slots * P, 256);
+  l.pa = take(4 * slots * P, 256);
+  l.hc = c.tc ? take(2 * static_cast<size_t>(c.ldc) * P, 1024) : 0;
+  l.wq = (c.tc && c.wdt == BD_E4M3) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
+  l.total = (off + 255) / 256 * 256;
+  return l;
+}
+
+bool encode_bf16_2d(CUtensorMap* m, const void* base, int64_t inner, int64_t rows, int64_t ld_elems,
+                    uint32_t box_inner, uint32_t box_rows) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld_elems * 2)};
+  cuuint32_t box[2] = {box_inner, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+int cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return BD_OK;
+  if (e == cudaErrorNoKernelImageForDevice || e == cudaErrorInvalidDeviceFunction) return BD_ERR_DEVICE;
+  return BD_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+int bd_version(void) { return 100; }
+
+const char* bd_status_string(int status) {
+  switch (status) {
+    case BD_OK: return "ok";
+    case BD_ERR_NULL: return "a required pointer is NULL";
+    case BD_ERR_SHAPE: return "sizes disagree or are out of range";
+    case BD_ERR_DTYPE: return "unsupported dtype or dtype combination";
+    case BD_ERR_ALIGN: return "pointer or row stride misaligned";
+    case BD_ERR_TAU: return "invalid threshold grid (T outside 1..32, NULL or NaN)";
+    case BD_ERR_WORKSPACE: return "workspace too small";
+    case BD_ERR_CUDA: return "a CUDA call or kernel launch failed";
+    case BD_ERR_TIMEOUT: return "a bounded device-side wait gave up";
+    case BD_ERR_DEVICE: return "the current device cannot run this library (needs sm_103)";
+    case BD_ERR_ARG: return "invalid argument";
+    default: return "unknown status";
+  }
+}
+
+size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                         const bd_tau_grid* tau_grid) {
+  Call c;
+  if (check_args(hidden, weight, mask_state, tau_grid, 0, &c) != BD_OK) return 0;
+  DevCtx* ctx = nullptr;
+  if (device_ctx(&ctx) != BD_OK) return 0;
+  return make_layout(c, make_plan(c, ctx->sm_count)).total;
+}
+
+int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                      const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+                      const bd_exec* exec) {
+  const int variant = exec ? exec->variant : 0;
+  if (exec && exec->flags != 0) return BD_ERR_ARG;
+  Call c;
+  int rc = check_args(hidden, weight, mask_state, tau_grid, variant, &c);
+  if (rc != BD_OK) return rc;
+  if (c.P == 0) return BD_OK;
+  if (!out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
+  if (!aligned(out_tokens, 4) || !aligned(out_conf, 4) || !aligned(out_commit, 4)) return BD_ERR_ALIGN;
+  if (exec && exec->out_counts && !aligned(exec->out_counts, 4)) return BD_ERR_ALIGN;
+  if (exec && exec->workspace && !aligned(exec->workspace, 256)) return BD_ERR_ALIGN;
+
+  DevCtx* ctx = nullptr;
+  rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  const BandPlan plan = make_plan(c, ctx->sm_count);
+  const Layout lay = make_layout(c, plan);
+
+  uint8_t* ws = nullptr;
+  if (exec && exec->workspace) {
+    if (exec->workspace_bytes < lay.total) return BD_ERR_WORKSPACE;
+    ws = static_cast<uint8_t*>(exec->workspace);
+  } else {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (ctx->ws_bytes < lay.total) {
+      if (ctx->ws) cudaFree(ctx->ws);  // synchronises the device: no call can still use it
+      ctx->ws = nullptr;
+      ctx->ws_bytes = 0;
+      if (cudaMalloc(&ctx->ws, lay.total) != cudaSuccess) return BD_ERR_CUDA;
+      ctx->ws_bytes = lay.total;
+    }
+    ws = static_cast<uint8_t*>(ctx->ws);
+  }
+
+  cudaStream_t st = static_cast<cudaStream_t>(exec ? exec->stream : nullptr);
+  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
+  int* idx = reinterpret_cast<int*>(ws + lay.idx);
+  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
+  float* pm = reinterpret_cast<float*>(ws + lay.pm);
+  float* ps = reinterpret_cast<float*>(ws + lay.ps);
+  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+  const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+
+  // a0: compaction of the masked positions of active blocks
+  rc = cuda_status(bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows,
+                                      st));
+  if (rc != BD_OK) return rc;
+
+  CUtensorMap tmA, tmB;
+  if (c.tc) {
+    void* hc = ws + lay.hc;
+    rc = cuda_status(bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, ctx->sm_count, st));
+    if (rc != BD_OK) return rc;
+    const void* wsrc = weight->data;
+    int64_t wld = c.ldw;
+    if (c.wdt == BD_E4M3) {
+      void* wq = ws + lay.wq;
+      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
+                                               ctx->sm_count, st));
+      if (rc != BD_OK) return rc;
+      wsrc = wq;
+      wld = c.ldq;
+    }
+    if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
+    if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
+  }
+
+  if (exec && exec->out_counts) {
+    if (cudaMemsetAsync(exec->out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
+      return BD_ERR_CUDA;
+  }
+
+  // a1 + a2: LM head with the online softmax epilogue
+  if (exec && exec->lmhead_event_begin &&
+      cudaEventRecord(static_cast<cudaEvent_t>(exec->lmhead_event_begin), st) != cudaSuccess)
+    return BD_ERR_CUDA;
+  if (c.tc) {
+    bd::TcArgs a;
+    a.n_rows = n_rows;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    a.status = ctx->status;
+    rc = cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
+  } else {
+    bd::SimtArgs a;
+    a.hidden = hidden->data;
+    a.ldh = c.ldh;
+    a.hdtype = c.hdt;
+    a.w = weight->data;
+    a.ldw = c.ldw;
+    a.wdtype = c.wdt;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.idx = idx;
+    a.n_rows = n_rows;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    rc = cuda_status(bd::launch_lmhead_simt(a, st));
+  }
+  if (rc != BD_OK) return rc;
+  if (exec && exec->lmhead_event_end &&
+      cudaEventRecord(static_cast<cudaEvent_t>(exec->lmhead_event_end), st) != cudaSuccess)
+    return BD_ERR_CUDA;
+
+  // a3 + a4: merge and the multi-threshold commit
+  bd::CommitArgs ca;
+  ca.pos_masked = mask_state->pos_masked;
+  ca.block_flags = mask_state->block_flags;
+  ca.rowpos = rowpos;
+  ca.n_rows = n_rows;
+  ca.plan = plan;
+  ca.P = P;
+  ca.part_m = pm;
+  ca.part_s = ps;
+  ca.part_a = pa;
+  ca.n_blocks = c.n_blocks;
+  ca.n_slots = c.n_slots;
+  ca.block_len = c.L;
+  std::memset(&ca.taus, 0, sizeof(ca.taus));
+  for (int k = 0; k < c.T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
+  ca.taus.T = c.T;
+  ca.out_tokens = out_tokens;
+  ca.out_conf = out_conf;
+  ca.out_commit = out_commit;
+  ca.out_counts = exec ? exec->out_counts : nullptr;
+  return cuda_status(bd::launch_merge_commit(ca, st));
+}
+
+int bd_commit_step(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                   const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit) {
+  return bd_commit_step_ex(hidden, weight, mask_state, tau_grid, out_tokens, out_conf, out_commit, nullptr);
+}
+
+int bd_get_device_status(void* stream) {
+  DevCtx* ctx = nullptr;
+  int rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return BD_ERR_CUDA;
+  uint32_t word = 0;
+  if (cudaMemcpy(&word, ctx->status, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return BD_ERR_CUDA;
+  if (word != 0 && cudaMemset(ctx->status, 0, sizeof(word)) != cudaSuccess) return BD_ERR_CUDA;
+  if (word & bd::DEV_TIMEOUT) return BD_ERR_TIMEOUT;
+  return BD_OK;
+}
+
+int bd_shutdown(void) {
+  std::lock_guard<std::mutex> lk(g_mu);
+  int cur = 0;
+  if (cudaGetDevice(&cur) != cudaSuccess) return BD_ERR_CUDA;
+  int rc = BD_OK;
+  for (int dev = 0; dev < MAX_DEVICES; ++dev) {
+    DevCtx& c = g_dev[dev];
+    if (!c.ready) continue;
+    if (cudaSetDevice(dev) != cudaSuccess) {
+      rc = BD_ERR_CUDA;
+      continue;
+    }
+    if (c.ws) cudaFree(c.ws);
+    if (c.status) cudaFree(c.status);
+    c = DevCtx();
+  }
+  cudaSetDevice(cur);
+  return rc;
+}
+
+}  // extern "C"

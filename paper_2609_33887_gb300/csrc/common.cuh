@@ -1,0 +1,337 @@
+// Device-side helpers shared by the kernels of libbdcommit: the vocabulary
+// work plan, PTX wrappers for mbarriers, TMA, tcgen05 (UMMA + tensor memory),
+// bounded waits and the online softmax combine.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+
+namespace bd {
+
+// Device status bits, OR-ed into the library's status word.
+constexpr uint32_t DEV_TIMEOUT = 1u;
+
+// A bounded wait gives up after this long (nanoseconds of %globaltimer).
+constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;  // 1 s
+// After giving up, drains of in-flight copies / MMAs wait at most this long.
+constexpr uint64_t DRAIN_LIMIT_NS = 100000000ull;  // 0.1 s
+
+constexpr float LOG2E = 1.4426950408889634f;
+
+// -------------------------------------------------------------------------
+// Work plan of the LM-head kernels.
+//
+// The N compacted rows are cut into m-tiles of BM rows and the vocabulary
+// into v-tiles of BN entries. m-tiles are taken in bands of at most GM; in a
+// band of gm m-tiles the vocabulary is split into gv = min(G / gm, n_vt)
+// contiguous parts, and CTA c (c < gm * gv) takes m-tile m0 + c % gm over
+// part c / gm. CTAs of one part walk the same v-tiles at the same time, so a
+// weight tile is fetched from HBM about once per band and re-read from L2 by
+// the gm CTAs that share it. Each (row, part) leaves one partial
+// (max, sum of exponentials, argmax) in slot `part` of the partial arrays;
+// the merge kernel combines the gv slots of a row. N is only known on the
+// device, so kernels recompute the plan from it.
+// -------------------------------------------------------------------------
+struct BandPlan {
+  int BM;    // rows per m-tile
+  int BN;    // vocabulary entries per v-tile
+  int GM;    // m-tiles per band (at most)
+  int G;     // CTAs of the LM-head grid
+  int n_vt;  // ceil(V / BN)
+};
+
+struct Band {
+  int m0;     // first m-tile of the band
+  int gm;     // m-tiles in the band
+  int gv;     // vocabulary parts per m-tile
+  int units;  // gm * gv CTAs busy in this band
+};
+
+__host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+__host__ __device__ __forceinline__ Band band_of(const BandPlan& p, int n_mt, int b) {
+  Band r;
+  r.m0 = b * p.GM;
+  r.gm = n_mt - r.m0 < p.GM ? n_mt - r.m0 : p.GM;
+  int gv = p.G / r.gm;
+  r.gv = gv < p.n_vt ? gv : p.n_vt;
+  if (r.gv < 1) r.gv = 1;
+  r.units = r.gm * r.gv;
+  return r;
+}
+
+// Number of partial slots of compacted row `row`.
+__host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int row) {
+  int n_mt = cdiv(n_rows, p.BM);
+  int b = (row / p.BM) / p.GM;
+  return band_of(p, n_mt, b).gv;
+}
+
+// Iterates the (m-tile, v-tile) sequence of this CTA (blockIdx.x) under the band plan.
+struct TileIter {
+  BandPlan p;
+  int n_mt, n_bands;
+  int b;       // current band
+  int m_tile;  // current m-tile
+  int part;    // vocabulary part of the current unit
+  int vt, vt_end;
+
+  __device__ void init(const BandPlan& plan, int n_rows) {
+    p = plan;
+    n_mt = cdiv(n_rows, p.BM);
+    n_bands = cdiv(n_mt, p.GM);
+    b = -1;
+    vt = vt_end = 0;
+  }
+  // Advances to the next unit; false when the CTA has no more work.
+  __device__ bool next_unit() {
+    for (++b; b < n_bands; ++b) {
+      Band bd = band_of(p, n_mt, b);
+      const int c = blockIdx.x;
+      if (c >= bd.units) continue;
+      m_tile = bd.m0 + c % bd.gm;
+      part = c / bd.gm;
+      vt = static_cast<int>(static_cast<int64_t>(part) * p.n_vt / bd.gv);
+      vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * p.n_vt / bd.gv);
+      return true;
+    }
+    return false;
+  }
+};
+
+
+// -------------------------------------------------------------------------
+// Online softmax state: running max m (natural units), sum s of exp(l - m),
+// lowest index a attaining m. Combine is commutative and keeps the lowest
+// index on equal maxima.
+// -------------------------------------------------------------------------
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void softmax_combine(float& m, float& s, int& a, float m2, float s2, int a2) {
+  if (m2 > m) {
+    s = s2 + (m == -INFINITY ? 0.f : s * ex2_approx((m - m2) * LOG2E));
+    m = m2;
+    a = a2;
+  } else if (m2 == m) {
+    if (m2 != -INFINITY) s += s2;
+    a = a2 < a ? a2 : a;
+  } else if (m2 != -INFINITY) {
+    s += s2 * ex2_approx((m2 - m) * LOG2E);
+  }
+}
+
+// -------------------------------------------------------------------------
+// PTX wrappers
+// -------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ uint32_t mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok;
+}
+
+// Single-thread bounded wait for the phase of parity `parity` to complete.
+// Returns false (and raises the CTA's abort flag) after WAIT_LIMIT_NS, or as
+// soon as another role of the CTA has raised the abort flag.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* status) {
+  if (mbar_try_wait(bar, parity)) return true;
+  uint64_t t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((it & 31u) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer_ns() - t0 > WAIT_LIMIT_NS) {
+        *abort_flag = 1;
+        atomicOr(status, DEV_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+
+// Whole-warp bounded wait with a warp-uniform outcome.
+__device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                               uint32_t* status) {
+  const uint32_t lane = threadIdx.x & 31u;
+  uint64_t t0 = 0;
+  for (uint32_t it = 0;; ++it) {
+    uint32_t ok = mbar_try_wait(bar, parity);
+    if (__all_sync(0xffffffffu, ok)) return true;
+    if ((it & 31u) == 31u) {
+      int stop = 0;
+      if (lane == 0) {
+        uint64_t now = globaltimer_ns();
+        if (t0 == 0) t0 = now;
+        if (*abort_flag) {
+          stop = 1;
+        } else if (now - t0 > WAIT_LIMIT_NS) {
+          *abort_flag = 1;
+          atomicOr(status, DEV_TIMEOUT);
+          stop = 1;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, stop, 0)) return false;
+    }
+  }
+}
+
+// Bounded wait that ignores the abort flag (used only to drain work in flight
+// before the CTA exits).
+__device__ __forceinline__ bool mbar_drain(uint32_t bar, uint32_t parity) {
+  uint64_t t0 = globaltimer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (globaltimer_ns() - t0 > DRAIN_LIMIT_NS) return false;
+  }
+  return true;
+}
+
+// ---- TMA ----------------------------------------------------------------
+__device__ __forceinline__ void prefetch_tmap(const void* tmap) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+}
+
+__device__ __forceinline__ uint64_t policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+__device__ __forceinline__ uint64_t policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+
+// 2-D tiled load global -> shared; completes `bytes` of transaction count on `bar`.
+// x is the innermost (contiguous) coordinate in elements, y the row.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const void* tmap, uint32_t bar, int x, int y,
+                                            uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(bar), "l"(policy)
+      : "memory");
+}
+
+// ---- tcgen05 ------------------------------------------------------------
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile stored with the
+// 128-byte swizzle (rows of 64 bf16 = 128 B, 8-row swizzle atoms of 1 KB):
+// start address >> 4 in bits 0-13, leading byte offset >> 4 in bits 16-29
+// (unused for swizzled K-major layouts), stride byte offset >> 4 (1 KB
+// between 8-row groups) in bits 32-45, descriptor version 1 in bits 46-47,
+// base offset 0 (tiles are 1 KB aligned), swizzle mode 2 (128 B) in bits 61-63.
+__device__ __forceinline__ uint64_t sw128_kmajor_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4);
+  d |= static_cast<uint64_t>(16u >> 4) << 16;
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;
+  d |= static_cast<uint64_t>(1u) << 46;
+  d |= static_cast<uint64_t>(2u) << 61;
+  return d;
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16 with bf16 A and B, fp32
+// accumulator, both operands K-major: D format F32 (bits 4-5 = 1), A format
+// BF16 (bits 7-9 = 1), B format BF16 (bits 10-12 = 1), N >> 3 in bits 17-22,
+// M >> 4 in bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(N >> 3) << 17) |
+         (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+// D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on `bar` when every tcgen05.mma issued so far by this thread has completed.
+__device__ __forceinline__ void umma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// Load 32 consecutive fp32 columns of this thread's TMEM lane (32x32b shape,
+// x32 repeat) and wait for the load to complete.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];\n\t"
+      "tcgen05.wait::ld.sync.aligned;"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+        "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+        "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+        "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr)
+      : "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+}  // namespace bd

@@ -1,0 +1,135 @@
+// Merge of the per-part softmax partials and the threshold commit with the
+// per-block top-1 fallback, for every tau of the grid in one pass.
+//
+// One CTA (4 warps) per block of the window. Warps split the partial slots
+// of each masked position, warp 0 finishes the merge and then applies, for
+// every tau_k, the rule
+//   commit(p, k) = masked(p) && active(block) && conf(p) >= tau_k           (Sec. 3.1, App. B.1)
+//                  || the block is fallback-eligible, holds a masked position,
+//                     no position cleared tau_k, and p is the masked position of
+//                     highest confidence (lowest position on ties)         (App. B.2)
+// with one warp ballot per tau (two for blocks longer than 32).
+#include "kernels.h"
+
+namespace bd {
+
+namespace {
+constexpr int THREADS = 128;
+constexpr int WARPS = THREADS / 32;
+constexpr int MAX_L = 64;
+}  // namespace
+
+__global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
+  __shared__ float sm_m[WARPS][MAX_L], sm_s[WARPS][MAX_L];
+  __shared__ int sm_a[WARPS][MAX_L];
+  const int blk = blockIdx.x;
+  const int L = a.block_len;
+  const int64_t base = static_cast<int64_t>(blk) * L;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_rows = *a.n_rows;
+
+  // ---- a3: merge of the partial slots (slots split across the 4 warps)
+  for (int jj = lane; jj < L; jj += 32) {
+    const int r = a.rowpos[base + jj];
+    float m = -INFINITY, s = 0.f;
+    int arg = 0x7fffffff;
+    if (r >= 0) {
+      const int ns = slots_of_row(a.plan, n_rows, r);
+      for (int slot = warp; slot < ns; slot += WARPS) {
+        const int64_t o = static_cast<int64_t>(slot) * a.P + r;
+        softmax_combine(m, s, arg, a.part_m[o], a.part_s[o], a.part_a[o]);
+      }
+    }
+    sm_m[warp][jj] = m;
+    sm_s[warp][jj] = s;
+    sm_a[warp][jj] = arg;
+  }
+  __syncthreads();
+  if (warp != 0) return;
+
+  const uint32_t flags = a.block_flags[blk];
+  const bool eligible = (flags & 2u) != 0;
+  bool live[2];
+  float conf[2];
+  int tok[2];
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int jj = lane + 32 * h;
+    live[h] = jj < L && a.rowpos[base + jj] >= 0;
+    conf[h] = 0.f;
+    tok[h] = -1;
+    if (live[h]) {
+      float m = sm_m[0][jj], s = sm_s[0][jj];
+      int arg = sm_a[0][jj];
+#pragma unroll
+      for (int w = 1; w < WARPS; ++w) softmax_combine(m, s, arg, sm_m[w][jj], sm_s[w][jj], sm_a[w][jj]);
+      conf[h] = 1.f / s;  // s >= 1: the maximum contributes exp(0)
+      tok[h] = arg;
+    }
+  }
+
+  // fallback candidate: highest confidence among masked positions, lowest position on ties
+  float best_c = -1.f;
+  int best_j = 0x7fffffff;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int jj = lane + 32 * h;
+    if (live[h] && (conf[h] > best_c || (conf[h] == best_c && jj < best_j))) {
+      best_c = conf[h];
+      best_j = jj;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float c2 = __shfl_xor_sync(0xffffffffu, best_c, o);
+    const int j2 = __shfl_xor_sync(0xffffffffu, best_j, o);
+    if (c2 > best_c || (c2 == best_c && j2 < best_j)) {
+      best_c = c2;
+      best_j = j2;
+    }
+  }
+  const bool any_live = __any_sync(0xffffffffu, live[0] || live[1]);
+  const bool take_fallback = eligible && any_live;
+
+  const int seq = blk / a.n_slots;
+  uint32_t bits[2] = {0u, 0u};
+  for (int k = 0; k < a.taus.T; ++k) {
+    const float tau = a.taus.tau[k];
+    bool c0 = live[0] && conf[0] >= tau;
+    bool c1 = live[1] && conf[1] >= tau;
+    uint32_t b0 = __ballot_sync(0xffffffffu, c0);
+    uint32_t b1 = __ballot_sync(0xffffffffu, c1);
+    if ((b0 | b1) == 0u && take_fallback) {
+      if (best_j < 32) {
+        b0 = 1u << best_j;
+        c0 = (lane == best_j);
+      } else {
+        b1 = 1u << (best_j - 32);
+        c1 = (lane == best_j - 32);
+      }
+    }
+    bits[0] |= static_cast<uint32_t>(c0) << k;
+    bits[1] |= static_cast<uint32_t>(c1) << k;
+    if (a.out_counts != nullptr && lane == 0) {
+      const int cnt = __popc(b0) + __popc(b1);
+      if (cnt) atomicAdd(a.out_counts + static_cast<int64_t>(seq) * a.taus.T + k, cnt);
+    }
+  }
+
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int jj = lane + 32 * h;
+    if (jj < L) {
+      a.out_tokens[base + jj] = tok[h];
+      a.out_conf[base + jj] = conf[h];
+      a.out_commit[base + jj] = bits[h];
+    }
+  }
+}
+
+cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st) {
+  merge_commit_kernel<<<a.n_blocks, THREADS, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace bd

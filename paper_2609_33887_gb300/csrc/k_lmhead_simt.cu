@@ -1,0 +1,141 @@
+// LM-head projection + mask-suppressed softmax statistics with fp32 FMA on
+// the CUDA cores. This is the exact-fp32 path (fp32 hidden states and head),
+// and it accepts bf16 / e4m3 heads too. Same band plan and partial layout as
+// the tensor-core kernel, with 32-row m-tiles and 256-entry v-tiles.
+#include <cuda_fp16.h>
+
+#include "../../include/bdcommit.h"
+#include "kernels.h"
+
+namespace bd {
+
+namespace {
+
+constexpr int KC = 32;      // hidden columns staged per step
+constexpr int THREADS = 256;
+static_assert(SIMT_BN == THREADS, "one vocabulary column per thread");
+static_assert(SIMT_BM == 32, "one row per lane in the reductions");
+
+__device__ __forceinline__ float load_h(const void* p, int64_t i, int dt) {
+  if (dt == BD_F32) return static_cast<const float*>(p)[i];
+  return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
+}
+
+__device__ __forceinline__ float e4m3_to_float(uint8_t c) {
+  uint32_t h2;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(static_cast<uint16_t>(c)));
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(h2 & 0xffffu)));
+}
+
+__device__ __forceinline__ float load_w(const void* p, int64_t i, int dt) {
+  if (dt == BD_F32) return static_cast<const float*>(p)[i];
+  if (dt == BD_BF16) return __bfloat162float(static_cast<const __nv_bfloat16*>(p)[i]);
+  return e4m3_to_float(static_cast<const uint8_t*>(p)[i]);
+}
+
+struct SimtSmem {
+  float hs[SIMT_BM][KC + 1];
+  union {
+    float ws[SIMT_BN][KC + 1];         // head tile during the K loop
+    float lg[SIMT_BM][SIMT_BN + 1];    // logits of the tile after it
+  } u;
+  float rm[SIMT_BM], rs[SIMT_BM];
+  int ra[SIMT_BM];
+};
+
+}  // namespace
+
+__global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
+  __shared__ SimtSmem sm;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int n_rows = *a.n_rows;
+
+  TileIter it;
+  it.init(a.plan, n_rows);
+  while (it.next_unit()) {
+    const int r0 = it.m_tile * SIMT_BM;
+    if (tid < SIMT_BM) {
+      sm.rm[tid] = -INFINITY;
+      sm.rs[tid] = 0.f;
+      sm.ra[tid] = 0x7fffffff;
+    }
+    for (int vt = it.vt; vt < it.vt_end; ++vt) {
+      const int v = vt * SIMT_BN + tid;
+      float acc[SIMT_BM];
+#pragma unroll
+      for (int r = 0; r < SIMT_BM; ++r) acc[r] = 0.f;
+      for (int k0 = 0; k0 < a.d; k0 += KC) {
+        // stage 32 hidden rows x KC columns (rows gathered through idx)
+        for (int e = tid; e < SIMT_BM * KC; e += THREADS) {
+          const int r = e / KC, kk = e % KC;
+          float x = 0.f;
+          if (r0 + r < n_rows && k0 + kk < a.d)
+            x = load_h(a.hidden, static_cast<int64_t>(a.idx[r0 + r]) * a.ldh + k0 + kk, a.hdtype);
+          sm.hs[r][kk] = x;
+        }
+        // stage 256 head rows x KC columns
+        for (int e = tid; e < SIMT_BN * KC; e += THREADS) {
+          const int vr = e / KC, kk = e % KC;
+          const int vv = vt * SIMT_BN + vr;
+          float x = 0.f;
+          if (vv < a.V && k0 + kk < a.d) x = load_w(a.w, static_cast<int64_t>(vv) * a.ldw + k0 + kk, a.wdtype);
+          sm.u.ws[vr][kk] = x;
+        }
+        __syncthreads();
+#pragma unroll 4
+        for (int kk = 0; kk < KC; ++kk) {
+          const float wv = sm.u.ws[tid][kk];
+#pragma unroll
+          for (int r = 0; r < SIMT_BM; ++r) acc[r] = fmaf(sm.hs[r][kk], wv, acc[r]);
+        }
+        __syncthreads();
+      }
+      const bool dead = (v >= a.V) || (v == a.mask_id);
+      const float sc = (a.wscale != nullptr && v < a.V) ? a.wscale[v] : 1.f;
+#pragma unroll
+      for (int r = 0; r < SIMT_BM; ++r) sm.u.lg[r][tid] = dead ? -INFINITY : acc[r] * sc;
+      __syncthreads();
+      // warp w reduces rows 4w..4w+3; lane l scans columns 8l..8l+7 in order
+      for (int rr = 0; rr < SIMT_BM / 8; ++rr) {
+        const int r = warp * (SIMT_BM / 8) + rr;
+        float m = -INFINITY, s = 0.f;
+        int arg = 0x7fffffff;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const float x = sm.u.lg[r][lane * 8 + j];
+          if (x != -INFINITY) softmax_combine(m, s, arg, x, 1.f, vt * SIMT_BN + lane * 8 + j);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+          const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+          const int a2 = __shfl_xor_sync(0xffffffffu, arg, o);
+          softmax_combine(m, s, arg, m2, s2, a2);
+        }
+        if (lane == 0) {
+          float M = sm.rm[r], S = sm.rs[r];
+          int A = sm.ra[r];
+          softmax_combine(M, S, A, m, s, arg);
+          sm.rm[r] = M;
+          sm.rs[r] = S;
+          sm.ra[r] = A;
+        }
+      }
+      __syncthreads();
+    }
+    if (tid < SIMT_BM && r0 + tid < n_rows) {
+      const int64_t o = static_cast<int64_t>(it.part) * a.P + r0 + tid;
+      a.part_m[o] = sm.rm[tid];
+      a.part_s[o] = sm.rs[tid];
+      a.part_a[o] = sm.ra[tid];
+    }
+    __syncthreads();
+  }
+}
+
+cudaError_t launch_lmhead_simt(const SimtArgs& a, cudaStream_t st) {
+  lmhead_simt_kernel<<<a.plan.G, THREADS, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace bd

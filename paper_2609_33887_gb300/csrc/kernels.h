@@ -1,0 +1,95 @@
+// Host-side launchers of the kernels of libbdcommit (internal interface
+// between api.cu and the kernel translation units).
+#pragma once
+
+#include <cstddef>
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+
+namespace bd {
+
+struct TauParams {
+  float tau[32];
+  int T;
+};
+
+// a0: compaction of the masked positions of active blocks (Sec. 2.1 / App. F
+// slot states). Writes idx[r] = position of compacted row r (ascending
+// positions), rowpos[p] = r or -1, and *n_rows = N.
+cudaError_t launch_compact(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
+                           int* idx, int* rowpos, int* n_rows, cudaStream_t st);
+
+// Packs the hidden rows of the compacted positions: hc[r] = hidden[idx[r]], bf16.
+cudaError_t launch_pack_rows_bf16(const void* hidden, int64_t ld, int d, const int* idx, const int* n_rows,
+                                  int P, void* hc, int64_t ldc, int sm_count, cudaStream_t st);
+
+// Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
+cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
+                                int sm_count, cudaStream_t st);
+
+// a1+a2 on the tensor cores: tcgen05 LM-head GEMM with the online softmax
+// epilogue. tmA describes hc [P, d] bf16, tmB the head [V, d] bf16.
+struct TcArgs {
+  const int* n_rows;
+  const float* wscale;  // [V] or nullptr
+  int V, d, P, mask_id;
+  BandPlan plan;
+  float* part_m;
+  float* part_s;
+  int* part_a;
+  uint32_t* status;
+};
+constexpr int TC_BM = 128;
+constexpr int TC_BN = 256;
+constexpr int TC_BK = 64;
+constexpr int TC_THREADS = 192;
+size_t tc_smem_bytes(int stages);
+cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const TcArgs& a, int stages,
+                             cudaStream_t st);
+
+// a1+a2 with fp32 FMA on the CUDA cores (exact fp32 path; any dtype combo).
+struct SimtArgs {
+  const void* hidden;
+  int64_t ldh;
+  int hdtype;  // BD_F32 / BD_BF16
+  const void* w;
+  int64_t ldw;
+  int wdtype;  // BD_F32 / BD_BF16 / BD_E4M3
+  const float* wscale;
+  const int* idx;
+  const int* n_rows;
+  int V, d, P, mask_id;
+  BandPlan plan;
+  float* part_m;
+  float* part_s;
+  int* part_a;
+};
+constexpr int SIMT_BM = 32;
+constexpr int SIMT_BN = 256;
+cudaError_t launch_lmhead_simt(const SimtArgs& a, cudaStream_t st);
+
+// a3+a4: merge of the partials per row, then the threshold commit with the
+// per-block top-1 fallback for every tau of the grid.
+struct CommitArgs {
+  const uint8_t* pos_masked;
+  const uint8_t* block_flags;
+  const int* rowpos;
+  const int* n_rows;
+  BandPlan plan;
+  int P;
+  const float* part_m;
+  const float* part_s;
+  const int* part_a;
+  int n_blocks, n_slots, block_len;
+  TauParams taus;
+  int32_t* out_tokens;
+  float* out_conf;
+  uint32_t* out_commit;
+  int32_t* out_counts;
+};
+cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st);
+
+}  // namespace bd

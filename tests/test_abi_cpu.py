@@ -1,0 +1,132 @@
+"""The C-ABI library without a GPU: it builds, loads, exports every symbol
+include/bdcommit.h declares (and nothing else), and its argument checks
+reject bad calls before any CUDA call."""
+
+import ctypes
+import math
+import os
+import re
+import shutil
+import subprocess
+
+import pytest
+
+from paper_2609_33887_gb300 import bdcommit as B
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "bdcommit.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("no CUDA toolkit")
+    import __graft_entry__
+
+    __graft_entry__.build()
+    return B.load_library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:int|size_t|const char\*)\s+(bd_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_abi():
+    assert declared_functions() == sorted([
+        "bd_commit_step", "bd_commit_step_ex", "bd_get_device_status", "bd_shutdown", "bd_status_string",
+        "bd_version", "bd_workspace_size"])
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+
+
+def test_library_exports_nothing_else(lib):
+    nm = shutil.which("nm")
+    if nm is None:
+        pytest.skip("no nm")
+    out = subprocess.run([nm, "-D", "--defined-only", B.LIB_PATH], capture_output=True, text=True).stdout
+    names = sorted(l.split()[-1] for l in out.splitlines() if " T " in l)
+    assert names == declared_functions()
+
+
+def test_status_strings_and_version(lib):
+    for code in range(-10, 1):
+        s = B.bd_status_string(code)
+        assert s and s != "unknown status"
+    assert B.bd_status_string(-99) == "unknown status"
+    assert B.bd_version() == 100
+
+
+# ----------------------------------------------------- argument checks --
+FAKE = 1 << 20  # a non-null, 256-byte aligned address that is never dereferenced
+
+
+def _args(**kw):
+    p = dict(n_seq=2, n_slots=2, L=32, d=128, V=1000, hdt=B.BD_BF16, wdt=B.BD_BF16, mask=-1,
+             taus=[0.5, 0.9], hptr=FAKE, wptr=FAKE, scale=None, rows=None, hld=None, wld=None)
+    p.update(kw)
+    P = p["n_seq"] * p["n_slots"] * p["L"]
+    h = B.bd_hidden(p["hptr"], p["hdt"], P if p["rows"] is None else p["rows"], p["d"],
+                    p["d"] if p["hld"] is None else p["hld"])
+    w = B.bd_weight(p["wptr"], p["wdt"], p["V"], p["d"], p["d"] if p["wld"] is None else p["wld"], p["scale"])
+    ms = B.bd_mask_state(p["n_seq"], p["n_slots"], p["L"], p["mask"], FAKE, FAKE)
+    arr = (ctypes.c_float * max(1, len(p["taus"])))(*p["taus"])
+    tg = B.bd_tau_grid(ctypes.cast(arr, ctypes.POINTER(ctypes.c_float)), len(p["taus"]))
+    return h, w, ms, tg, arr
+
+
+def _call(lib, variant=0, flags=0, outs=(FAKE, FAKE, FAKE), **kw):
+    h, w, ms, tg, _keep = _args(**kw)
+    ex = B.bd_exec()
+    ex.variant = variant
+    ex.flags = flags
+    return lib.bd_commit_step_ex(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+                                 outs[0], outs[1], outs[2], ctypes.byref(ex))
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(taus=[]), B.BD_ERR_TAU),
+    (dict(taus=[0.1] * 33), B.BD_ERR_TAU),
+    (dict(taus=[0.5, math.nan]), B.BD_ERR_TAU),
+    (dict(L=65), B.BD_ERR_SHAPE),
+    (dict(L=0), B.BD_ERR_SHAPE),
+    (dict(rows=100), B.BD_ERR_SHAPE),
+    (dict(hld=64), B.BD_ERR_SHAPE),
+    (dict(V=0), B.BD_ERR_SHAPE),
+    (dict(hdt=B.BD_F32), B.BD_ERR_DTYPE),
+    (dict(hdt=B.BD_BF16, wdt=B.BD_F32), B.BD_ERR_DTYPE),
+    (dict(hdt=7), B.BD_ERR_DTYPE),
+    (dict(wdt=B.BD_E4M3), B.BD_ERR_NULL),
+    (dict(mask=1000), B.BD_ERR_ARG),
+    (dict(mask=-2), B.BD_ERR_ARG),
+    (dict(hptr=FAKE + 2), B.BD_ERR_ALIGN),
+    (dict(wptr=FAKE + 8), B.BD_ERR_ALIGN),
+    (dict(d=100, hld=100, wld=100), B.BD_ERR_ALIGN),
+    (dict(hptr=None), B.BD_ERR_NULL),
+])
+def test_argument_checks(lib, kw, code):
+    assert _call(lib, **kw) == code
+
+
+def test_variant_flags_and_outputs_checked(lib):
+    assert _call(lib, variant=3) == B.BD_ERR_ARG
+    assert _call(lib, flags=1) == B.BD_ERR_ARG
+    assert _call(lib, variant=2, hdt=B.BD_F32, wdt=B.BD_F32) == B.BD_ERR_DTYPE
+    assert _call(lib, outs=(None, FAKE, FAKE)) == B.BD_ERR_NULL
+    assert _call(lib, outs=(FAKE + 1, FAKE, FAKE)) == B.BD_ERR_ALIGN
+
+
+def test_null_structs_rejected(lib):
+    h, w, ms, tg, _keep = _args()
+    assert lib.bd_commit_step(None, ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg), FAKE, FAKE, FAKE) == \
+        B.BD_ERR_NULL
+    assert lib.bd_workspace_size(ctypes.byref(h), None, ctypes.byref(ms), ctypes.byref(tg)) == 0
+
+
+def test_empty_window_is_a_no_op(lib):
+    # zero sequences: nothing to compute, nothing queued, no CUDA call
+    assert _call(lib, n_seq=0, hptr=None, wptr=None, outs=(None, None, None)) == B.BD_OK

@@ -1,0 +1,203 @@
+"""Parity of the CUDA commit step (through the C ABI) with the float64 oracle.
+
+Small cases run the oracle on every position: several m-tiles and v-tiles,
+ragged last tiles in rows, vocabulary and width, and the degenerate cases of
+the rule. Full-size workloads compare every position of the 8x2x32 workload
+and seeded samples of whole blocks of the larger ones, in the launch
+configuration bench.py times.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+from tests.helpers import oracle_on_workload
+from tests.parity import compare
+from workloads import CONFIGS, generate, scaled
+
+pytestmark = pytest.mark.gpu
+
+bdc = pytest.importorskip("paper_2609_33887_gb300")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    yield
+
+
+def run_gpu(wl, variant=0, workspace=None, stream=None):
+    cfg = wl.cfg
+    g = wl.to("cuda")
+    tokens, conf, commit, counts = bdc.commit_step(
+        g.hidden, g.weight, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, wl.tau,
+        weight_scale=g.weight_scale, mask_token_id=wl.mask_token_id, counts=True, variant=variant,
+        workspace=workspace, stream=stream)
+    torch.cuda.synchronize()
+    st = bdc.bd_get_device_status()
+    assert st == 0, bdc.bd_status_string(st)
+    return {
+        "tokens": tokens.cpu().numpy(),
+        "conf": conf.cpu().numpy(),
+        "commit": commit.cpu().numpy().view(np.uint32),
+        "counts": counts.cpu().numpy(),
+    }
+
+
+def check(wl, variant=0, blocks=None, ref=None):
+    out = run_gpu(wl, variant)
+    ref = oracle_on_workload(wl, blocks=blocks) if ref is None else ref
+    rep = compare(out, ref, wl.tau, wl.cfg.weight_dtype, wl.cfg.block_len, wl.cfg.n_slots)
+    assert rep.ok(), rep.failures
+    return out, ref, rep
+
+
+# ------------------------------------------------------------- small cases --
+
+SMALL = {
+    # one m-tile, four v-tiles with a ragged last one
+    "bf16_1mt": scaled(CONFIGS[1], n_seq=2, n_slots=2, d=256, V=1000),
+    # five m-tiles (ragged), ragged width (K tail of 8), twelve v-tiles
+    "bf16_5mt_ktail": scaled(CONFIGS[1], n_seq=8, n_slots=4, d=200, V=3000),
+    # sixteen m-tiles: two bands of the plan
+    "bf16_2bands": scaled(CONFIGS[2], n_seq=32, n_slots=4, d=128, V=2148),
+    # block_len 64, 16 thresholds
+    "bf16_L64": scaled(CONFIGS[3], n_seq=4, n_slots=4, d=192, V=4000),
+    # FP8 head with per-row scales
+    "e4m3": scaled(CONFIGS[4], n_seq=4, n_slots=4, d=512, V=5000),
+    "e4m3_ktail": scaled(CONFIGS[4], n_seq=3, n_slots=2, d=80, V=700),
+}
+
+
+def test_tiny_f32_full():
+    wl = generate(CONFIGS[0])
+    _, _, rep = check(wl)
+    assert rep.n_live == 32
+    assert rep.max_dconf < 1e-4  # exact fp32 path
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+def test_small_tensor_core(name):
+    wl = generate(SMALL[name])
+    _, _, rep = check(wl)
+    assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "e4m3"])
+def test_small_simt_variant(name):
+    wl = generate(SMALL[name])
+    check(wl, variant=1)
+
+
+def test_tc_and_simt_agree_on_argmax():
+    wl = generate(SMALL["bf16_5mt_ktail"])
+    a = run_gpu(wl, variant=2)
+    b = run_gpu(wl, variant=1)
+    assert np.array_equal(a["tokens"] < 0, b["tokens"] < 0)
+    assert np.abs(a["conf"] - b["conf"]).max() < 1e-3
+
+
+# -------------------------------------------------------------- edge cases --
+
+def test_nothing_masked():
+    wl = generate(scaled(SMALL["bf16_1mt"], mask_frac=0.0))
+    out, ref, rep = check(wl)
+    assert rep.n_live == 0
+    assert np.all(out["tokens"] == -1) and np.all(out["commit"] == 0) and np.all(out["conf"] == 0)
+    assert np.all(out["counts"] == 0)
+
+
+def test_everything_masked_and_every_block_eligible():
+    check(generate(scaled(SMALL["bf16_5mt_ktail"], mask_frac=1.0, fallback="all")))
+
+
+def test_no_block_eligible_and_half_inactive():
+    check(generate(scaled(SMALL["bf16_5mt_ktail"], fallback="none", active="first_half")))
+
+
+def test_some_blocks_without_masked_positions():
+    wl = generate(SMALL["bf16_5mt_ktail"])
+    pm = wl.pos_masked.clone().view(-1, wl.cfg.block_len)
+    pm[::3] = 0
+    wl.pos_masked = pm.reshape(-1).contiguous()
+    check(wl)
+
+
+@pytest.mark.parametrize("mask_id", [0, 2999, 2900])
+def test_mask_token_suppressed(mask_id):
+    # 2999: last entry, inside the ragged last v-tile; 0: first entry
+    cfg = scaled(SMALL["bf16_5mt_ktail"], mask_token_id=mask_id)
+    wl = generate(cfg)
+    # make the mask token the largest logit of the first 40 positions: with the
+    # suppression it must never be the token
+    w = wl.weight[mask_id].float()
+    h = wl.hidden.float()
+    h[:40] += 20.0 * w / (w * w).sum()
+    wl.hidden = h.to(wl.hidden.dtype)
+    out, ref, _ = check(wl)
+    assert not np.any(out["tokens"] == mask_id)
+
+
+def test_hidden_zero_gives_uniform_confidence():
+    wl = generate(scaled(SMALL["bf16_1mt"], mask_token_id=0))
+    wl.hidden = torch.zeros_like(wl.hidden)
+    out, ref, _ = check(wl)
+    live = ref["tokens"] >= 0
+    assert np.all(out["tokens"][live] == 1)
+    np.testing.assert_allclose(out["conf"][live], 1.0 / 999, rtol=1e-5)
+
+
+def test_identical_rows_give_identical_outputs():
+    wl = generate(SMALL["bf16_5mt_ktail"])
+    h = wl.hidden.clone()
+    h[:] = h[5]
+    wl.hidden = h
+    out, _, _ = check(wl)
+    live = out["tokens"] >= 0
+    assert len(set(out["tokens"][live].tolist())) == 1
+    assert len(set(out["conf"][live].tolist())) == 1
+
+
+@pytest.mark.parametrize("T", [1, 32])
+def test_grid_sizes(T):
+    taus = tuple(float(x) for x in np.linspace(0.05, 1.1, T)) if T > 1 else (0.5,)
+    check(generate(scaled(SMALL["bf16_5mt_ktail"], tau=taus)))
+
+
+def test_tau_zero_and_above_one():
+    wl = generate(scaled(SMALL["bf16_5mt_ktail"], tau=(0.0, 1.5)))
+    out, ref, _ = check(wl)
+    live = ref["tokens"] >= 0
+    assert np.array_equal((out["commit"] & 1) != 0, live)
+
+
+def test_odd_block_length():
+    check(generate(scaled(SMALL["bf16_1mt"], block_len=7, n_seq=5, n_slots=3)))
+
+
+# -------------------------------------------------------- full-size cases --
+
+def _sample_blocks(cfg, n, seed=99):
+    rng = np.random.default_rng(seed)
+    return sorted(rng.choice(cfg.n_blocks, size=min(n, cfg.n_blocks), replace=False).tolist())
+
+
+def test_full_size_b8_all_positions():
+    wl = generate(CONFIGS[1])
+    _, _, rep = check(wl)
+    assert rep.n_live > 250
+
+
+@pytest.mark.parametrize("i,n_blocks", [(2, 8), (3, 4), (4, 3)])
+def test_full_size_sampled_blocks(i, n_blocks):
+    wl = generate(CONFIGS[i])
+    blocks = _sample_blocks(CONFIGS[i], n_blocks)
+    _, _, rep = check(wl, blocks=blocks)
+    assert rep.n_live > 0

@@ -75,7 +75,11 @@ def block_flags_for(cfg: WorkloadConfig) -> torch.Tensor:
 
 
 def _realised_rows(weight_stored: torch.Tensor, scale: Optional[torch.Tensor], rows: torch.Tensor) -> torch.Tensor:
-    w = weight_stored[rows].float()
+    if weight_stored.dtype == torch.float8_e4m3fn:
+        # index through the byte view: some torch builds cannot index float8 tensors on the CPU
+        w = weight_stored.view(torch.uint8)[rows].view(torch.float8_e4m3fn).float()
+    else:
+        w = weight_stored[rows].float()
     if scale is not None:
         w = w * scale[rows, None]
     return w
