@@ -184,6 +184,38 @@ const char* bd_status_string(int status);
  * No call may be in flight. */
 int bd_shutdown(void);
 
+/* Size of the device scratch array that bd_commit_step_static works in. */
+#define BD_STATIC_SCRATCH_BYTES (32u * 1024u * 1024u)
+
+/* The commit step without any allocation. The paper has no counterpart: this
+ * is a service for callers that must not allocate device memory, such as code
+ * running inside an allocator or memory-pool callback (cudaMalloc there would
+ * re-enter the allocator), a process whose device memory is fully reserved by
+ * a framework's caching allocator, or a latency-critical serving loop that
+ * cannot afford cudaMalloc's implicit device-wide synchronisation.
+ *
+ * Same arguments and outputs as bd_commit_step, plus `stream` (a cudaStream_t,
+ * NULL = legacy default stream). Instead of a workspace, the call works in one
+ * file-scope device array of BD_STATIC_SCRATCH_BYTES (32 MiB) that every GPU
+ * which loads the library holds until the process exits. It calls no
+ * cudaMalloc, cudaFree or other allocating routine.
+ *   - Size limit: a call whose workspace (bd_workspace_size) would exceed
+ *     BD_STATIC_SCRATCH_BYTES returns BD_ERR_WORKSPACE before queuing anything
+ *     (the 8 x 2 x 32, d = 2048, V = 151936 bf16 window needs about 3 MiB).
+ *   - First call on a device: it looks up the array's device address with
+ *     cudaGetSymbolAddress (the device must be current) and caches it; make
+ *     that first call before any stream capture.
+ *   - Sharing: every call on a device uses the same array, which keeps the
+ *     previous call's contents (the call clears the one word that must start
+ *     at zero). Calls that can overlap on the GPU (different streams, or
+ *     different host threads) race on the array: serialise them.
+ *   - A bounded device-side wait that gives up is recorded in the array, not
+ *     in the word bd_get_device_status reads. */
+int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
+                          const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
+                          int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+                          void* stream);
+
 /* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
 int bd_version(void);
 

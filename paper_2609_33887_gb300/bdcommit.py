@@ -94,6 +94,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
                                       POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, POINTER(bd_exec)]),
         "bd_workspace_size": (c_size_t, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
                                          POINTER(bd_tau_grid)]),
+        "bd_commit_step_static": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                          POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, c_void_p]),
         "bd_get_device_status": (c_int, [c_void_p]),
         "bd_status_string": (ctypes.c_char_p, [c_int]),
         "bd_shutdown": (c_int, []),
@@ -215,6 +217,22 @@ def bd_commit_step(hidden, weight, weight_scale, pos_masked, block_flags, n_seq,
     return int(load_library().bd_commit_step(
         ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
         _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit)))
+
+
+def bd_commit_step_static(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                          mask_token_id, tau, out_tokens, out_conf, out_commit, *, stream=None) -> int:
+    """bd_commit_step_static: the commit step without any device allocation, for
+    callers that must not allocate (inside an allocator callback, under a
+    framework that owns all device memory, or on a serving path that cannot
+    take cudaMalloc's implicit synchronisation). It works in the library's
+    fixed 32 MiB device array; see include/bdcommit.h for its limits."""
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    return int(load_library().bd_commit_step_static(
+        ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+        _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit), _stream_handle(stream)))
 
 
 def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_len, tau, *,

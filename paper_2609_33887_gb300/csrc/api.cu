@@ -417,3 +417,174 @@ int bd_shutdown(void) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// bd_commit_step_static: the commit step for callers that cannot allocate.
+// Its workspace is the file-scope device array below; nothing here calls
+// cudaMalloc, cudaFree or any allocating routine.
+// ---------------------------------------------------------------------------
+namespace {
+
+static __device__ __align__(256) uint8_t g_static_scratch[BD_STATIC_SCRATCH_BYTES];
+
+// Offset, inside the workspace header, of the word the LM-head kernel reports
+// a timed-out wait in (the compacted row count sits at offset 0).
+constexpr size_t STATIC_STATUS_OFFSET = 128;
+
+struct StaticCtx {
+  bool ready = false;
+  int sm_count = 0;
+  uint8_t* scratch = nullptr;  // device address of g_static_scratch on this device
+};
+StaticCtx g_static[MAX_DEVICES];
+
+// Once per device, with that device current: checks the device, fetches the
+// tensor-map encoder and resolves the device address of g_static_scratch.
+// (In host code the array's name is only a host-side stand-in, so kernels
+// must be given the resolved address.)
+int static_ctx(StaticCtx** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return BD_ERR_CUDA;
+  if (dev < 0 || dev >= MAX_DEVICES) return BD_ERR_DEVICE;
+  std::lock_guard<std::mutex> lk(g_mu);
+  StaticCtx& s = g_static[dev];
+  if (!s.ready) {
+    int maj = 0, mnr = 0, sms = 0;
+    if (cudaDeviceGetAttribute(&maj, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&mnr, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+      return BD_ERR_CUDA;
+    if (maj != 10 || mnr != 3) return BD_ERR_DEVICE;
+    if (g_encode == nullptr) {
+      cudaDriverEntryPointQueryResult q;
+      void* fn = nullptr;
+      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+              cudaSuccess ||
+          q != cudaDriverEntryPointSuccess || fn == nullptr)
+        return BD_ERR_CUDA;
+      g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    void* p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
+    if (e != cudaSuccess || p == nullptr) return e == cudaSuccess ? BD_ERR_CUDA : cuda_status(e);
+    s.scratch = static_cast<uint8_t*>(p);
+    s.sm_count = sms;
+    s.ready = true;
+  }
+  *out = &s;
+  return BD_OK;
+}
+
+}  // namespace
+
+extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
+                                     const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
+                                     int32_t* out_tokens, float* out_conf, uint32_t* out_commit, void* stream) {
+  Call c;
+  int rc = check_args(hidden, weight, mask_state, tau_grid, 0, &c);
+  if (rc != BD_OK) return rc;
+  if (c.P == 0) return BD_OK;
+  if (!out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
+  if (!aligned(out_tokens, 4) || !aligned(out_conf, 4) || !aligned(out_commit, 4)) return BD_ERR_ALIGN;
+
+  StaticCtx* sctx = nullptr;
+  rc = static_ctx(&sctx);
+  if (rc != BD_OK) return rc;
+  const BandPlan plan = make_plan(c, sctx->sm_count);
+  const Layout lay = make_layout(c, plan);
+  if (lay.total > BD_STATIC_SCRATCH_BYTES) return BD_ERR_WORKSPACE;
+
+  uint8_t* ws = sctx->scratch;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
+  uint32_t* status = reinterpret_cast<uint32_t*>(ws + lay.hdr + STATIC_STATUS_OFFSET);
+  int* idx = reinterpret_cast<int*>(ws + lay.idx);
+  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
+  float* pm = reinterpret_cast<float*>(ws + lay.pm);
+  float* ps = reinterpret_cast<float*>(ws + lay.ps);
+  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+  const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+
+  // The array keeps the previous call's contents; only the timeout word must
+  // start at zero (everything else is written before it is read).
+  if (cudaMemsetAsync(status, 0, sizeof(uint32_t), st) != cudaSuccess) return BD_ERR_CUDA;
+
+  rc = cuda_status(bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows,
+                                      st));
+  if (rc != BD_OK) return rc;
+  CUtensorMap tmA, tmB;
+  if (c.tc) {
+    void* hc = ws + lay.hc;
+    rc = cuda_status(
+        bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, sctx->sm_count, st));
+    if (rc != BD_OK) return rc;
+    const void* wsrc = weight->data;
+    int64_t wld = c.ldw;
+    if (c.wdt == BD_E4M3) {
+      void* wq = ws + lay.wq;
+      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
+                                               sctx->sm_count, st));
+      if (rc != BD_OK) return rc;
+      wsrc = wq;
+      wld = c.ldq;
+    }
+    if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
+    if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
+    bd::TcArgs a;
+    a.n_rows = n_rows;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    a.status = status;
+    rc = cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
+  } else {
+    bd::SimtArgs a;
+    a.hidden = hidden->data;
+    a.ldh = c.ldh;
+    a.hdtype = c.hdt;
+    a.w = weight->data;
+    a.ldw = c.ldw;
+    a.wdtype = c.wdt;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.idx = idx;
+    a.n_rows = n_rows;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    rc = cuda_status(bd::launch_lmhead_simt(a, st));
+  }
+  if (rc != BD_OK) return rc;
+
+  bd::CommitArgs ca;
+  ca.pos_masked = mask_state->pos_masked;
+  ca.block_flags = mask_state->block_flags;
+  ca.rowpos = rowpos;
+  ca.n_rows = n_rows;
+  ca.plan = plan;
+  ca.P = P;
+  ca.part_m = pm;
+  ca.part_s = ps;
+  ca.part_a = pa;
+  ca.n_blocks = c.n_blocks;
+  ca.n_slots = c.n_slots;
+  ca.block_len = c.L;
+  std::memset(&ca.taus, 0, sizeof(ca.taus));
+  for (int k = 0; k < c.T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
+  ca.taus.T = c.T;
+  ca.out_tokens = out_tokens;
+  ca.out_conf = out_conf;
+  ca.out_commit = out_commit;
+  ca.out_counts = nullptr;
+  return cuda_status(bd::launch_merge_commit(ca, st));
+}

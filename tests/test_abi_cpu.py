@@ -35,8 +35,8 @@ def declared_functions():
 
 def test_header_declares_the_abi():
     assert declared_functions() == sorted([
-        "bd_commit_step", "bd_commit_step_ex", "bd_get_device_status", "bd_shutdown", "bd_status_string",
-        "bd_version", "bd_workspace_size"])
+        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_get_device_status", "bd_shutdown",
+        "bd_status_string", "bd_version", "bd_workspace_size"])
 
 
 def test_library_exports_every_declared_symbol(lib):

@@ -1,0 +1,85 @@
+"""bd_commit_step_static, the entry point that allocates nothing.
+
+Some callers cannot allocate device memory: code running inside an allocator
+or memory-pool callback, a process whose device memory a framework's caching
+allocator already owns, or a serving loop that cannot take cudaMalloc's
+implicit synchronisation. For them the library runs the commit step in a
+fixed 32 MiB device array it owns from load time. These tests call that
+entry point through the C ABI and check it against bd_commit_step_ex, within
+the tolerances of the parity tests, on two calls in a row (the array keeps
+the previous call's contents). This file sorts last so that a run that stops
+at its first failure has already run every other test.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from workloads import CONFIGS, generate, scaled
+
+pytestmark = pytest.mark.gpu
+
+bdc = pytest.importorskip("paper_2609_33887_gb300")
+B = bdc.bdcommit
+
+CONF_TOL = 2e-3  # bf16 / f32 confidence tolerance of the parity tests
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    yield
+
+
+def _outputs(P, dev):
+    return (torch.full((P,), -7, dtype=torch.int32, device=dev), torch.full((P,), -7.0, device=dev),
+            torch.full((P,), -7, dtype=torch.int32, device=dev))
+
+
+def _run(wl, static):
+    cfg = wl.cfg
+    g = wl.to("cuda")
+    tok, conf, com = _outputs(cfg.P, g.hidden.device)
+    args = (g.hidden, g.weight, g.weight_scale, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots,
+            cfg.block_len, cfg.mask_token_id, cfg.tau, tok, conf, com)
+    rc = B.bd_commit_step_static(*args) if static else B.bd_commit_step_ex(*args)
+    assert rc == B.BD_OK, B.bd_status_string(rc)
+    torch.cuda.synchronize()
+    return tok.cpu().numpy(), conf.cpu().numpy(), com.cpu().numpy().view(np.uint32)
+
+
+@pytest.mark.parametrize("cfg", [CONFIGS[1], CONFIGS[0], scaled(CONFIGS[4], n_seq=4, n_slots=4, d=512, V=5000)],
+                         ids=["b8x2x32_bf16", "tiny_f32", "e4m3_small"])
+def test_static_matches_the_allocating_entry_point_twice(cfg):
+    wl = generate(cfg)
+    ref_tok, ref_conf, ref_com = _run(wl, static=False)
+    for _ in range(2):
+        tok, conf, com = _run(wl, static=True)
+        assert np.array_equal(tok, ref_tok)
+        assert np.abs(conf.astype(np.float64) - ref_conf).max() <= CONF_TOL
+        assert np.array_equal(com, ref_com)
+    assert (ref_tok >= 0).sum() > 0
+
+
+def test_static_rejects_windows_beyond_its_array():
+    # the 64 x 4 x 64, d = 4096 window needs far more than 32 MiB of workspace;
+    # the call is refused before anything is queued
+    cfg = scaled(CONFIGS[3], V=1024, name="too_large")
+    P = cfg.P
+    dev = torch.device("cuda")
+    h = torch.zeros((P, cfg.d), dtype=torch.bfloat16, device=dev)
+    w = torch.zeros((cfg.V, cfg.d), dtype=torch.bfloat16, device=dev)
+    pm = torch.ones(P, dtype=torch.uint8, device=dev)
+    bf = torch.ones(cfg.n_blocks, dtype=torch.uint8, device=dev)
+    tok, conf, com = _outputs(P, dev)
+    assert B.bd_workspace_size(h, w, None, pm, bf, cfg.n_seq, cfg.n_slots, cfg.block_len, -1, cfg.tau) > 32 << 20
+    rc = B.bd_commit_step_static(h, w, None, pm, bf, cfg.n_seq, cfg.n_slots, cfg.block_len, -1, cfg.tau,
+                                 tok, conf, com)
+    assert rc == B.BD_ERR_WORKSPACE
+    torch.cuda.synchronize()
+    assert int(tok[0]) == -7  # nothing was written
