@@ -64,6 +64,18 @@ def timing_events(n, stream):
     return evs
 
 
+def aggregate_over_ranks(elapsed_ms, n_masked, dist=None, device="cpu"):
+    """Weak-scaling aggregation: the slowest rank's time and every rank's
+    masked positions (each rank serves its own independent window)."""
+    if dist is None:
+        return float(elapsed_ms), float(n_masked)
+    t = torch.tensor([float(elapsed_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    n = torch.tensor([float(n_masked)], dtype=torch.float64, device=device)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), float(n.item())
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -331,15 +343,7 @@ def run_ours(args):
     st = B.bd_get_device_status(stream)
     if st != 0:
         raise B.BdError(st, "timed region")
-    if pg:
-        t = torch.tensor([elapsed_ms], device=dev)
-        pg.all_reduce(t, op=pg.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
-        nm = torch.tensor([float(n_masked)], device=dev)
-        pg.all_reduce(nm, op=pg.ReduceOp.SUM)
-        total_masked = float(nm.item())
-    else:
-        total_masked = float(n_masked)
+    elapsed_ms, total_masked = aggregate_over_ranks(elapsed_ms, n_masked, pg, dev)
     ms_per_step = elapsed_ms / K
     value = total_masked * K / (elapsed_ms / 1e3)
 
@@ -373,11 +377,7 @@ def run_ours(args):
             e2e_step()
         e1.record(stream)
         torch.cuda.synchronize()
-        e_ms = e0.elapsed_time(e1)
-        if pg:
-            t = torch.tensor([e_ms], device=dev)
-            pg.all_reduce(t, op=pg.ReduceOp.MAX)
-            e_ms = float(t.item())
+        e_ms, _ = aggregate_over_ranks(e0.elapsed_time(e1), 0, pg, dev)
         h2d = h_host.numel() * h_host.element_size() + pm_host.numel() + bf_host.numel()
         d2h = sum(o.numel() * o.element_size() for o in out_host)
         e2e = {"value": total_masked * K / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
