@@ -2,7 +2,7 @@
 confidence + multi-threshold commit) on GB300, as masked positions per second.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--config NAME] [--graph]
+                    [--config NAME] [--no-graph]
 
 One step = one bd_commit_step over one window of the workload (compaction,
 packing, LM head with the online softmax epilogue, merge and commit for the
@@ -47,7 +47,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default=DEFAULT_CONFIG)
-    ap.add_argument("--graph", action="store_true", help="replay each step as a captured CUDA graph")
+    ap.add_argument("--no-graph", dest="graph", action="store_false",
+                    help="launch every step eagerly instead of replaying the K steps as one CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -285,8 +286,8 @@ def run_ours(args):
     def step(h=None, ev=None):
         rc = B.bd_commit_step_ex(wl.hidden if h is None else h, wl.weight, wl.weight_scale, wl.pos_masked,
                                  wl.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
-                                 cfg.tau, tokens, conf, commit, stream=stream, workspace=workspace,
-                                 out_counts=counts, lmhead_events=ev)
+                                 cfg.tau, tokens, conf, commit, stream=torch.cuda.current_stream(),
+                                 workspace=workspace, out_counts=counts, lmhead_events=ev)
         if rc != 0:
             raise B.BdError(rc)
 
@@ -299,18 +300,18 @@ def run_ours(args):
     if st != 0:
         raise B.BdError(st, "warm-up")
 
+    # per-step LM-head events: recorded on the launching stream inside the timed region
+    evs = timing_events(K, stream)
     graph = None
     if args.graph:
+        # the K timed steps as one CUDA graph (the serving engine also replays captured graphs)
         graph = torch.cuda.CUDAGraph()
-        ev_g = timing_events(1, stream)[0]
-        with torch.cuda.graph(graph, stream=stream):
-            step(ev=ev_g)
-        graph.replay()
+        with torch.cuda.graph(graph):
+            for i in range(K):
+                step(ev=evs[i])
         torch.cuda.synchronize()
 
     # ---- device-resident timed region
-    evs = timing_events(K, stream)
-    lm_ms = []
     vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x]
     sampler = ClockSampler(vis[local] if local < len(vis) else str(local))
     sampler.start()
@@ -323,23 +324,14 @@ def run_ours(args):
         for i in range(K):
             step(ev=evs[i])
     else:
-        for i in range(K):
-            graph.replay()
+        graph.replay()
     t_end.record(stream)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
     clocks = sampler.stop()
     elapsed_ms = t_start.elapsed_time(t_end)
-    if graph is None:
-        lm_ms = [a.elapsed_time(b) for a, b in evs]
-    else:
-        # one extra replay timed alone for the LM-head events inside the graph
-        lm_ms = []
-        for _ in range(min(K, 50)):
-            graph.replay()
-            torch.cuda.synchronize()
-            lm_ms.append(ev_g[0].elapsed_time(ev_g[1]))
+    lm_ms = [a.elapsed_time(b) for a, b in evs]
     st = B.bd_get_device_status(stream)
     if st != 0:
         raise B.BdError(st, "timed region")
@@ -369,12 +361,22 @@ def run_ours(args):
         for _ in range(W):
             e2e_step()
         torch.cuda.synchronize()
+        egraph = None
+        if args.graph:
+            egraph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(egraph):
+                for _ in range(K):
+                    e2e_step()
+            torch.cuda.synchronize()
         if pg:
             pg.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(K):
-            e2e_step()
+        if egraph is None:
+            for _ in range(K):
+                e2e_step()
+        else:
+            egraph.replay()
         e1.record(stream)
         torch.cuda.synchronize()
         e_ms, _ = aggregate_over_ranks(e0.elapsed_time(e1), 0, pg, dev)

@@ -135,8 +135,14 @@ typedef struct {
  *   lmhead_event_begin / lmhead_event_end : optional cudaEvent_t recorded on
  *                     the stream right before and after the LM-head kernel,
  *                     for timing it alone.
- *   variant         : 0 = automatic; 1 = force the fp32-FMA SIMT LM-head
- *                     kernel; 2 = force the tensor-core kernel (BF16/E4M3 only).
+ *   variant         : 0 = automatic (for BF16 / E4M3 heads the CTA-pair
+ *                     tensor-core kernel up to 8192 window positions and the
+ *                     one-CTA kernel above; the fp32 SIMT kernel for F32
+ *                     heads); 1 = force
+ *                     the fp32-FMA SIMT LM-head kernel; 2 = force the one-CTA
+ *                     tensor-core kernel (tokens on the MMA M side); 3 = force the
+ *                     CTA-pair tensor-core kernel (vocabulary on the M side).
+ *                     2 and 3 need BF16 hidden states.
  *   flags           : reserved, must be 0. */
 typedef struct {
   void* stream;

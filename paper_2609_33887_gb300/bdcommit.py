@@ -41,7 +41,8 @@ BD_BLOCK_FALLBACK_ELIGIBLE = 2
 
 VARIANT_AUTO = 0
 VARIANT_SIMT = 1
-VARIANT_TC = 2
+VARIANT_TC_ONE_CTA = 2
+VARIANT_TC_PAIR = 3
 
 
 class bd_hidden(ctypes.Structure):

@@ -8,7 +8,7 @@
 #include <cstring>
 #include <mutex>
 
-#include "../../include/bdcommit.h"
+#include "bdcommit.h"
 #include "kernels.h"
 
 namespace {
@@ -23,6 +23,7 @@ constexpr int64_t MAX_DIM = int64_t(1) << 20;
 struct DevCtx {
   bool ready = false;
   int sm_count = 0;
+  int pairs = 0;               // CTA pairs of the pair kernel that fit on the device at once
   uint32_t* status = nullptr;  // device status word (bd::DEV_* bits)
   void* ws = nullptr;          // library-owned workspace
   size_t ws_bytes = 0;
@@ -54,9 +55,12 @@ int device_ctx(DevCtx** out, int* dev_out = nullptr) {
         return BD_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
+    int pairs = 0;
+    if (bd::lmhead_pair_max_pairs(sms, &pairs) != cudaSuccess) return BD_ERR_CUDA;
     if (cudaMalloc(&c.status, 256) != cudaSuccess) return BD_ERR_CUDA;
     if (cudaMemset(c.status, 0, 256) != cudaSuccess) return BD_ERR_CUDA;
     c.sm_count = sms;
+    c.pairs = pairs;
     c.ready = true;
   }
   *out = &c;
@@ -70,6 +74,7 @@ struct Call {
   int n_seq, n_slots, L, n_blocks, mask_id, T;
   int hdt, wdt;
   bool tc;          // tensor-core LM head
+  bool pair;        // ... on CTA pairs (vocabulary on M), else the one-CTA kernel
   int64_t ldh, ldw;
   int64_t ldc;      // packed hidden rows (bf16), elements
   int64_t ldq;      // decoded e4m3 head (bf16), elements
@@ -81,6 +86,8 @@ int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }
 
 int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
+int env_int(const char* name, int dflt, int lo, int hi);
+
 int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, const bd_tau_grid* tg,
                int variant, Call* c) {
   if (!h || !w || !ms || !tg) return BD_ERR_NULL;
@@ -88,7 +95,7 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   if (tg->T < 1 || tg->T > 32) return BD_ERR_TAU;
   for (int k = 0; k < tg->T; ++k)
     if (std::isnan(tg->tau[k])) return BD_ERR_TAU;
-  if (variant < 0 || variant > 2) return BD_ERR_ARG;
+  if (variant < 0 || variant > 3) return BD_ERR_ARG;
   if (ms->n_seq < 0 || ms->n_slots < 1 || ms->block_len < 1 || ms->block_len > 64) return BD_ERR_SHAPE;
   const int64_t n_blocks = int64_t(ms->n_seq) * ms->n_slots;
   const int64_t P = n_blocks * ms->block_len;
@@ -103,7 +110,7 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
   const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3);
   if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
-  const bool tc = variant == 2 || (variant == 0 && combo_bf16);
+  const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
   if (tc && !combo_bf16) return BD_ERR_DTYPE;
   if (P > 0) {
     if (!h->data || !w->data || !ms->pos_masked || !ms->block_flags) return BD_ERR_NULL;
@@ -128,6 +135,11 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   c->hdt = hdt;
   c->wdt = wdt;
   c->tc = tc;
+  // automatic choice: the CTA-pair kernel (vocabulary on M, token dimension
+  // padded only to a multiple of 32) wins while the window is small; at large
+  // windows both kernels saturate the tensor pipe under the power cap and the
+  // one-CTA kernel runs slightly faster
+  c->pair = tc && (variant == 3 || (variant == 0 && P <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
   c->ldh = h->ld;
   c->ldw = w->ld;
   c->ldc = round_up(c->d, 8);
@@ -143,18 +155,26 @@ int env_int(const char* name, int dflt, int lo, int hi) {
   return v < lo ? lo : v > hi ? hi : v;
 }
 
-BandPlan make_plan(const Call& c, int sm_count) {
+BandPlan make_plan(const Call& c, int sm_count, int pairs) {
   BandPlan p;
-  if (c.tc) {
+  if (c.pair) {
+    p.BM = 0;  // token groups derived from N on the device
+    p.BN = 256;
+    p.G = pairs;
+    p.GM = env_int("BD_PAIR_GM", 4, 1, pairs);
+    p.cpu = 2;
+  } else if (c.tc) {
     p.BM = bd::TC_BM;
     p.BN = bd::TC_BN;
     p.G = sm_count;
     p.GM = env_int("BD_TC_GM", 8, 1, sm_count);
+    p.cpu = 1;
   } else {
     p.BM = bd::SIMT_BM;
     p.BN = bd::SIMT_BN;
     p.G = 2 * sm_count;
     p.GM = 8;
+    p.cpu = 1;
   }
   p.n_vt = static_cast<int>((c.V + p.BN - 1) / p.BN);
   return p;
@@ -174,7 +194,7 @@ Layout make_layout(const Call& c, const BandPlan& p) {
     return o;
   };
   const size_t P = static_cast<size_t>(c.P);
-  const size_t slots = static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
+  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
   l.hdr = take(256, 256);
   l.idx = take(4 * P, 256);
   l.rowpos = take(4 * P, 256);
@@ -199,12 +219,140 @@ bool encode_bf16_2d(CUtensorMap* m, const void* base, int64_t inner, int64_t row
   return r == CUDA_SUCCESS;
 }
 
+// Records `ev` on `st`. Inside a stream capture a plain record would only add
+// a dependency edge; the external flag makes it an event node of the graph,
+// so replays still time the kernel.
+cudaError_t record_event(void* ev, cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(st, &cs);
+  if (e != cudaSuccess) return e;
+  if (cs == cudaStreamCaptureStatusActive)
+    return cudaEventRecordWithFlags(static_cast<cudaEvent_t>(ev), st, cudaEventRecordExternal);
+  return cudaEventRecord(static_cast<cudaEvent_t>(ev), st);
+}
+
 int cuda_status(cudaError_t e) {
   if (e == cudaSuccess) return BD_OK;
   if (e == cudaErrorNoKernelImageForDevice || e == cudaErrorInvalidDeviceFunction) return BD_ERR_DEVICE;
   return BD_ERR_CUDA;
 }
 
+
+// The launch sequence of one commit step (a0..a4) on `st`, working in `ws`
+// laid out by `lay`; kernel timeouts are reported in `status`.
+int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws, uint32_t* status, int sm_count,
+             const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+             const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+             int32_t* out_counts, void* ev_begin, void* ev_end, cudaStream_t st) {
+  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
+  int* idx = reinterpret_cast<int*>(ws + lay.idx);
+  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
+  float* pm = reinterpret_cast<float*>(ws + lay.pm);
+  float* ps = reinterpret_cast<float*>(ws + lay.ps);
+  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+  const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+
+  // a0: compaction of the masked positions of active blocks
+  int rc = cuda_status(
+      bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows, st));
+  if (rc != BD_OK) return rc;
+
+  CUtensorMap tmA, tmB;
+  bd::PairTokenMaps tmTok;
+  if (c.tc) {
+    void* hc = ws + lay.hc;
+    rc = cuda_status(bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, sm_count, st));
+    if (rc != BD_OK) return rc;
+    const void* wsrc = weight->data;
+    int64_t wld = c.ldw;
+    if (c.wdt == BD_E4M3) {
+      void* wq = ws + lay.wq;
+      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
+                                               sm_count, st));
+      if (rc != BD_OK) return rc;
+      wsrc = wq;
+      wld = c.ldq;
+    }
+    if (c.pair) {
+      // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
+      for (int i = 0; i < 8; ++i)
+        if (!encode_bf16_2d(&tmTok.m[i], hc, c.d, c.P, c.ldc, 64, 16 * (i + 1))) return BD_ERR_CUDA;
+      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
+    } else {
+      if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
+      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
+    }
+  }
+
+  if (out_counts) {
+    if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
+      return BD_ERR_CUDA;
+  }
+
+  // a1 + a2: LM head with the online softmax epilogue
+  if (ev_begin && record_event(ev_begin, st) != cudaSuccess) return BD_ERR_CUDA;
+  if (c.tc) {
+    bd::TcArgs a;
+    a.n_rows = n_rows;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    a.status = status;
+    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, a, st))
+                : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
+  } else {
+    bd::SimtArgs a;
+    a.hidden = hidden->data;
+    a.ldh = c.ldh;
+    a.hdtype = c.hdt;
+    a.w = weight->data;
+    a.ldw = c.ldw;
+    a.wdtype = c.wdt;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.idx = idx;
+    a.n_rows = n_rows;
+    a.V = V;
+    a.d = d;
+    a.P = P;
+    a.mask_id = c.mask_id;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    rc = cuda_status(bd::launch_lmhead_simt(a, st));
+  }
+  if (rc != BD_OK) return rc;
+  if (ev_end && record_event(ev_end, st) != cudaSuccess) return BD_ERR_CUDA;
+
+  // a3 + a4: merge and the multi-threshold commit
+  bd::CommitArgs ca;
+  ca.pos_masked = mask_state->pos_masked;
+  ca.block_flags = mask_state->block_flags;
+  ca.rowpos = rowpos;
+  ca.n_rows = n_rows;
+  ca.plan = plan;
+  ca.P = P;
+  ca.part_m = pm;
+  ca.part_s = ps;
+  ca.part_a = pa;
+  ca.n_blocks = c.n_blocks;
+  ca.n_slots = c.n_slots;
+  ca.block_len = c.L;
+  std::memset(&ca.taus, 0, sizeof(ca.taus));
+  for (int k = 0; k < c.T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
+  ca.taus.T = c.T;
+  ca.out_tokens = out_tokens;
+  ca.out_conf = out_conf;
+  ca.out_commit = out_commit;
+  ca.out_counts = out_counts;
+  return cuda_status(bd::launch_merge_commit(ca, st));
+}
 }  // namespace
 
 extern "C" {
@@ -234,7 +382,7 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const
   if (check_args(hidden, weight, mask_state, tau_grid, 0, &c) != BD_OK) return 0;
   DevCtx* ctx = nullptr;
   if (device_ctx(&ctx) != BD_OK) return 0;
-  return make_layout(c, make_plan(c, ctx->sm_count)).total;
+  return make_layout(c, make_plan(c, ctx->sm_count, ctx->pairs)).total;
 }
 
 int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
@@ -254,7 +402,7 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd
   DevCtx* ctx = nullptr;
   rc = device_ctx(&ctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(c, ctx->sm_count);
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs);
   const Layout lay = make_layout(c, plan);
 
   uint8_t* ws = nullptr;
@@ -274,109 +422,9 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd
   }
 
   cudaStream_t st = static_cast<cudaStream_t>(exec ? exec->stream : nullptr);
-  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
-  int* idx = reinterpret_cast<int*>(ws + lay.idx);
-  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
-  float* pm = reinterpret_cast<float*>(ws + lay.pm);
-  float* ps = reinterpret_cast<float*>(ws + lay.ps);
-  int* pa = reinterpret_cast<int*>(ws + lay.pa);
-  const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
-
-  // a0: compaction of the masked positions of active blocks
-  rc = cuda_status(bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows,
-                                      st));
-  if (rc != BD_OK) return rc;
-
-  CUtensorMap tmA, tmB;
-  if (c.tc) {
-    void* hc = ws + lay.hc;
-    rc = cuda_status(bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, ctx->sm_count, st));
-    if (rc != BD_OK) return rc;
-    const void* wsrc = weight->data;
-    int64_t wld = c.ldw;
-    if (c.wdt == BD_E4M3) {
-      void* wq = ws + lay.wq;
-      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
-                                               ctx->sm_count, st));
-      if (rc != BD_OK) return rc;
-      wsrc = wq;
-      wld = c.ldq;
-    }
-    if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
-    if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
-  }
-
-  if (exec && exec->out_counts) {
-    if (cudaMemsetAsync(exec->out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
-      return BD_ERR_CUDA;
-  }
-
-  // a1 + a2: LM head with the online softmax epilogue
-  if (exec && exec->lmhead_event_begin &&
-      cudaEventRecord(static_cast<cudaEvent_t>(exec->lmhead_event_begin), st) != cudaSuccess)
-    return BD_ERR_CUDA;
-  if (c.tc) {
-    bd::TcArgs a;
-    a.n_rows = n_rows;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
-    a.V = V;
-    a.d = d;
-    a.P = P;
-    a.mask_id = c.mask_id;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    a.status = ctx->status;
-    rc = cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
-  } else {
-    bd::SimtArgs a;
-    a.hidden = hidden->data;
-    a.ldh = c.ldh;
-    a.hdtype = c.hdt;
-    a.w = weight->data;
-    a.ldw = c.ldw;
-    a.wdtype = c.wdt;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
-    a.idx = idx;
-    a.n_rows = n_rows;
-    a.V = V;
-    a.d = d;
-    a.P = P;
-    a.mask_id = c.mask_id;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    rc = cuda_status(bd::launch_lmhead_simt(a, st));
-  }
-  if (rc != BD_OK) return rc;
-  if (exec && exec->lmhead_event_end &&
-      cudaEventRecord(static_cast<cudaEvent_t>(exec->lmhead_event_end), st) != cudaSuccess)
-    return BD_ERR_CUDA;
-
-  // a3 + a4: merge and the multi-threshold commit
-  bd::CommitArgs ca;
-  ca.pos_masked = mask_state->pos_masked;
-  ca.block_flags = mask_state->block_flags;
-  ca.rowpos = rowpos;
-  ca.n_rows = n_rows;
-  ca.plan = plan;
-  ca.P = P;
-  ca.part_m = pm;
-  ca.part_s = ps;
-  ca.part_a = pa;
-  ca.n_blocks = c.n_blocks;
-  ca.n_slots = c.n_slots;
-  ca.block_len = c.L;
-  std::memset(&ca.taus, 0, sizeof(ca.taus));
-  for (int k = 0; k < c.T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
-  ca.taus.T = c.T;
-  ca.out_tokens = out_tokens;
-  ca.out_conf = out_conf;
-  ca.out_commit = out_commit;
-  ca.out_counts = exec ? exec->out_counts : nullptr;
-  return cuda_status(bd::launch_merge_commit(ca, st));
+  return run_step(c, plan, lay, ws, ctx->status, ctx->sm_count, hidden, weight, mask_state, tau_grid, out_tokens,
+                  out_conf, out_commit, exec ? exec->out_counts : nullptr, exec ? exec->lmhead_event_begin : nullptr,
+                  exec ? exec->lmhead_event_end : nullptr, st);
 }
 
 int bd_commit_step(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
@@ -434,6 +482,7 @@ constexpr size_t STATIC_STATUS_OFFSET = 128;
 struct StaticCtx {
   bool ready = false;
   int sm_count = 0;
+  int pairs = 0;
   uint8_t* scratch = nullptr;  // device address of g_static_scratch on this device
 };
 StaticCtx g_static[MAX_DEVICES];
@@ -464,11 +513,14 @@ int static_ctx(StaticCtx** out) {
         return BD_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
+    int pairs = 0;
+    if (bd::lmhead_pair_max_pairs(sms, &pairs) != cudaSuccess) return BD_ERR_CUDA;
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
     if (e != cudaSuccess || p == nullptr) return e == cudaSuccess ? BD_ERR_CUDA : cuda_status(e);
     s.scratch = static_cast<uint8_t*>(p);
     s.sm_count = sms;
+    s.pairs = pairs;
     s.ready = true;
   }
   *out = &s;
@@ -490,101 +542,16 @@ extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* w
   StaticCtx* sctx = nullptr;
   rc = static_ctx(&sctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(c, sctx->sm_count);
+  const BandPlan plan = make_plan(c, sctx->sm_count, sctx->pairs);
   const Layout lay = make_layout(c, plan);
   if (lay.total > BD_STATIC_SCRATCH_BYTES) return BD_ERR_WORKSPACE;
 
   uint8_t* ws = sctx->scratch;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
   uint32_t* status = reinterpret_cast<uint32_t*>(ws + lay.hdr + STATIC_STATUS_OFFSET);
-  int* idx = reinterpret_cast<int*>(ws + lay.idx);
-  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
-  float* pm = reinterpret_cast<float*>(ws + lay.pm);
-  float* ps = reinterpret_cast<float*>(ws + lay.ps);
-  int* pa = reinterpret_cast<int*>(ws + lay.pa);
-  const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
-
   // The array keeps the previous call's contents; only the timeout word must
   // start at zero (everything else is written before it is read).
   if (cudaMemsetAsync(status, 0, sizeof(uint32_t), st) != cudaSuccess) return BD_ERR_CUDA;
-
-  rc = cuda_status(bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows,
-                                      st));
-  if (rc != BD_OK) return rc;
-  CUtensorMap tmA, tmB;
-  if (c.tc) {
-    void* hc = ws + lay.hc;
-    rc = cuda_status(
-        bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, sctx->sm_count, st));
-    if (rc != BD_OK) return rc;
-    const void* wsrc = weight->data;
-    int64_t wld = c.ldw;
-    if (c.wdt == BD_E4M3) {
-      void* wq = ws + lay.wq;
-      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
-                                               sctx->sm_count, st));
-      if (rc != BD_OK) return rc;
-      wsrc = wq;
-      wld = c.ldq;
-    }
-    if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
-    if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
-    bd::TcArgs a;
-    a.n_rows = n_rows;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
-    a.V = V;
-    a.d = d;
-    a.P = P;
-    a.mask_id = c.mask_id;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    a.status = status;
-    rc = cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
-  } else {
-    bd::SimtArgs a;
-    a.hidden = hidden->data;
-    a.ldh = c.ldh;
-    a.hdtype = c.hdt;
-    a.w = weight->data;
-    a.ldw = c.ldw;
-    a.wdtype = c.wdt;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
-    a.idx = idx;
-    a.n_rows = n_rows;
-    a.V = V;
-    a.d = d;
-    a.P = P;
-    a.mask_id = c.mask_id;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    rc = cuda_status(bd::launch_lmhead_simt(a, st));
-  }
-  if (rc != BD_OK) return rc;
-
-  bd::CommitArgs ca;
-  ca.pos_masked = mask_state->pos_masked;
-  ca.block_flags = mask_state->block_flags;
-  ca.rowpos = rowpos;
-  ca.n_rows = n_rows;
-  ca.plan = plan;
-  ca.P = P;
-  ca.part_m = pm;
-  ca.part_s = ps;
-  ca.part_a = pa;
-  ca.n_blocks = c.n_blocks;
-  ca.n_slots = c.n_slots;
-  ca.block_len = c.L;
-  std::memset(&ca.taus, 0, sizeof(ca.taus));
-  for (int k = 0; k < c.T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
-  ca.taus.T = c.T;
-  ca.out_tokens = out_tokens;
-  ca.out_conf = out_conf;
-  ca.out_commit = out_commit;
-  ca.out_counts = nullptr;
-  return cuda_status(bd::launch_merge_commit(ca, st));
+  return run_step(c, plan, lay, ws, status, sctx->sm_count, hidden, weight, mask_state, tau_grid, out_tokens,
+                  out_conf, out_commit, nullptr, nullptr, nullptr, st);
 }

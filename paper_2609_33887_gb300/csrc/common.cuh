@@ -34,21 +34,34 @@ constexpr float LOG2E = 1.4426950408889634f;
 // device, so kernels recompute the plan from it.
 // -------------------------------------------------------------------------
 struct BandPlan {
-  int BM;    // rows per m-tile
+  int BM;    // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
   int BN;    // vocabulary entries per v-tile
   int GM;    // m-tiles per band (at most)
-  int G;     // CTAs of the LM-head grid
+  int G;     // units that can run at once (CTAs, or CTA pairs)
   int n_vt;  // ceil(V / BN)
+  int cpu;   // CTAs per unit: each writes its own partial, so a part has cpu slots
 };
 
 struct Band {
   int m0;     // first m-tile of the band
   int gm;     // m-tiles in the band
   int gv;     // vocabulary parts per m-tile
-  int units;  // gm * gv CTAs busy in this band
+  int units;  // gm * gv units busy in this band
 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// Token-group size of the pair kernel for N rows: the fewest groups of at most
+// 256 rows, equal sizes rounded up to a multiple of 32 (16 rows per CTA).
+__host__ __device__ __forceinline__ int pair_group_rows(int n_rows) {
+  if (n_rows <= 0) return 32;
+  const int groups = cdiv(n_rows, 256);
+  return cdiv(cdiv(n_rows, groups), 32) * 32;
+}
+
+__host__ __device__ __forceinline__ int plan_bm(const BandPlan& p, int n_rows) {
+  return p.BM > 0 ? p.BM : pair_group_rows(n_rows);
+}
 
 __host__ __device__ __forceinline__ Band band_of(const BandPlan& p, int n_mt, int b) {
   Band r;
@@ -63,32 +76,38 @@ __host__ __device__ __forceinline__ Band band_of(const BandPlan& p, int n_mt, in
 
 // Number of partial slots of compacted row `row`.
 __host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int row) {
-  int n_mt = cdiv(n_rows, p.BM);
-  int b = (row / p.BM) / p.GM;
-  return band_of(p, n_mt, b).gv;
+  const int bm = plan_bm(p, n_rows);
+  const int n_mt = cdiv(n_rows, bm);
+  const int b = (row / bm) / p.GM;
+  return band_of(p, n_mt, b).gv * p.cpu;
 }
 
-// Iterates the (m-tile, v-tile) sequence of this CTA (blockIdx.x) under the band plan.
+// Iterates the (m-tile, v-tile) sequence of unit-runner `unit` (a CTA, or a
+// CTA pair) under the band plan.
 struct TileIter {
   BandPlan p;
-  int n_mt, n_bands;
+  int unit;
+  int bm, n_mt, n_bands;
   int b;       // current band
   int m_tile;  // current m-tile
   int part;    // vocabulary part of the current unit
   int vt, vt_end;
 
-  __device__ void init(const BandPlan& plan, int n_rows) {
+  __device__ void init(const BandPlan& plan, int n_rows, int unit_index) {
     p = plan;
-    n_mt = cdiv(n_rows, p.BM);
+    unit = unit_index;
+    bm = plan_bm(p, n_rows);
+    n_mt = cdiv(n_rows, bm);
     n_bands = cdiv(n_mt, p.GM);
     b = -1;
     vt = vt_end = 0;
   }
-  // Advances to the next unit; false when the CTA has no more work.
+  __device__ void init(const BandPlan& plan, int n_rows) { init(plan, n_rows, blockIdx.x); }
+  // Advances to the next unit; false when there is no more work.
   __device__ bool next_unit() {
     for (++b; b < n_bands; ++b) {
       Band bd = band_of(p, n_mt, b);
-      const int c = blockIdx.x;
+      const int c = unit;
       if (c >= bd.units) continue;
       m_tile = bd.m0 + c % bd.gm;
       part = c / bd.gm;
@@ -99,7 +118,6 @@ struct TileIter {
     return false;
   }
 };
-
 
 // -------------------------------------------------------------------------
 // Online softmax state: running max m (natural units), sum s of exp(l - m),
@@ -332,6 +350,81 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
       : "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ---- clusters and the CTA pair (cta_group::2) ----------------------------
+__device__ __forceinline__ uint32_t cluster_ctarank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+// All threads of both CTAs of the cluster.
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// Shared::cluster address of the variable at CTA-local address `addr` in CTA `rank`.
+__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+
+// Arrive once on an mbarrier given by its shared::cluster address (possibly in the peer CTA).
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// 2-D tiled load into this CTA's shared memory whose completion is counted on
+// an mbarrier of either CTA of the pair (`mbar` is a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap, uint32_t mbar, int x, int y,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
+      " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(mbar), "l"(policy)
+      : "memory");
+}
+
+// Tensor memory of a CTA pair: one warp of each CTA executes these together.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_relinquish_pair() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+// D[tmem of both CTAs] (+)= A[smem of both CTAs] * B[smem of both CTAs]^T with
+// M = 256 (128 rows of A in each CTA) and B's N rows split in halves between
+// the CTAs; issued by one thread of the even CTA.
+__device__ __forceinline__ void umma_bf16_pair(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                               uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+// Arrive once on the mbarrier at CTA-local address `bar` in every CTA of
+// `cta_mask` when all pair MMAs issued so far by this thread have completed.
+__device__ __forceinline__ void umma_commit_pair_mc(uint32_t bar, uint16_t cta_mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(cta_mask)
+      : "memory");
+}
+
+__device__ __forceinline__ void named_barrier_sync(uint32_t id, uint32_t nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
 }
 
 }  // namespace bd

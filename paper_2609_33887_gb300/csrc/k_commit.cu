@@ -1,7 +1,7 @@
 // Merge of the per-part softmax partials and the threshold commit with the
 // per-block top-1 fallback, for every tau of the grid in one pass.
 //
-// One CTA (4 warps) per block of the window. Warps split the partial slots
+// One CTA (8 warps) per block of the window. Threads split the partial slots
 // of each masked position, warp 0 finishes the merge and then applies, for
 // every tau_k, the rule
 //   commit(p, k) = masked(p) && active(block) && conf(p) >= tau_k           (Sec. 3.1, App. B.1)
@@ -14,35 +14,57 @@
 namespace bd {
 
 namespace {
-constexpr int THREADS = 128;
-constexpr int WARPS = THREADS / 32;
+constexpr int THREADS = 256;
 constexpr int MAX_L = 64;
+constexpr int MAX_GROUPS = THREADS / 32;
 }  // namespace
 
 __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
-  __shared__ float sm_m[WARPS][MAX_L], sm_s[WARPS][MAX_L];
-  __shared__ int sm_a[WARPS][MAX_L];
+  __shared__ float sm_m[MAX_GROUPS][MAX_L], sm_s[MAX_GROUPS][MAX_L];
+  __shared__ int sm_a[MAX_GROUPS][MAX_L];
   const int blk = blockIdx.x;
   const int L = a.block_len;
   const int64_t base = static_cast<int64_t>(blk) * L;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int n_rows = *a.n_rows;
 
-  // ---- a3: merge of the partial slots (slots split across the 4 warps)
-  for (int jj = lane; jj < L; jj += 32) {
-    const int r = a.rowpos[base + jj];
+  // ---- a3: merge of the partial slots. Thread t takes position t % Lp of the
+  // block and every groups-th slot starting at t / Lp; loads are issued four
+  // slots at a time so their latencies overlap.
+  const int Lp = L <= 32 ? 32 : 64;
+  const int groups = THREADS / Lp;
+  {
+    const int jj = threadIdx.x % Lp;
+    const int g = threadIdx.x / Lp;
     float m = -INFINITY, s = 0.f;
     int arg = 0x7fffffff;
+    const int r = jj < L ? a.rowpos[base + jj] : -1;
     if (r >= 0) {
       const int ns = slots_of_row(a.plan, n_rows, r);
-      for (int slot = warp; slot < ns; slot += WARPS) {
+      int slot = g;
+      for (; slot + 3 * groups < ns; slot += 4 * groups) {
+        float pm[4], ps[4];
+        int pa[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t o = static_cast<int64_t>(slot + u * groups) * a.P + r;
+          pm[u] = a.part_m[o];
+          ps[u] = a.part_s[o];
+          pa[u] = a.part_a[o];
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) softmax_combine(m, s, arg, pm[u], ps[u], pa[u]);
+      }
+      for (; slot < ns; slot += groups) {
         const int64_t o = static_cast<int64_t>(slot) * a.P + r;
         softmax_combine(m, s, arg, a.part_m[o], a.part_s[o], a.part_a[o]);
       }
     }
-    sm_m[warp][jj] = m;
-    sm_s[warp][jj] = s;
-    sm_a[warp][jj] = arg;
+    if (jj < L) {
+      sm_m[g][jj] = m;
+      sm_s[g][jj] = s;
+      sm_a[g][jj] = arg;
+    }
   }
   __syncthreads();
   if (warp != 0) return;
@@ -61,8 +83,7 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
     if (live[h]) {
       float m = sm_m[0][jj], s = sm_s[0][jj];
       int arg = sm_a[0][jj];
-#pragma unroll
-      for (int w = 1; w < WARPS; ++w) softmax_combine(m, s, arg, sm_m[w][jj], sm_s[w][jj], sm_a[w][jj]);
+      for (int g = 1; g < groups; ++g) softmax_combine(m, s, arg, sm_m[g][jj], sm_s[g][jj], sm_a[g][jj]);
       conf[h] = 1.f / s;  // s >= 1: the maximum contributes exp(0)
       tok[h] = arg;
     }

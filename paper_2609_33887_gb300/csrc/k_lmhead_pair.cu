@@ -1,0 +1,410 @@
+// LM-head projection + mask-suppressed softmax statistics on a CTA pair
+// (tcgen05 cta_group::2) with the vocabulary on the MMA M side (App. B.1: the
+// LM head and the softmax the engine commits from).
+//
+// A pair of CTAs (a cluster of 2) computes, per v-tile, logits of 256
+// vocabulary rows (128 in each CTA's tensor memory, one row per TMEM lane)
+// against a group of NT <= 256 token rows (NT columns): one
+// tcgen05.mma.cta_group::2 M=256 N=NT K=16 per 16 columns of d, issued by one
+// thread of the even CTA; each CTA stages its own 128 head rows and its half of
+// the token rows. A pipeline stage covers 128 columns of d (eight MMAs per
+// barrier wait and commit, which keeps the single issuing thread ahead of the
+// tensor pipe even at NT = 160), i.e. 32 KB + NT x 128 B per CTA; the number of
+// stages follows from NT (4 at NT = 160, 3 at NT = 256). Token tiles are loaded
+// with boxes of exactly NT/2 rows (one tensor map per height).
+// Compared with tokens on M, the token dimension is padded only to a multiple
+// of 32 (e.g. 294 rows -> 2 groups of 160, not 3 m-tiles of 128).
+//
+// The softmax reduction runs over vocabulary rows, i.e. over TMEM lanes. Each
+// epilogue warp owns 32 lanes; per 32 token columns it moves its 32 x 32
+// logits through a shared-memory transpose so that each thread holds one
+// token's 32 logits, and keeps a running (max, sum of exponentials, argmax)
+// per token across the v-tiles of its unit. The four warps' states are
+// combined once per unit, and each CTA writes its own partial per token.
+//
+// CTA layout (192 threads): warp 0 TMA producer, warp 1 TMEM allocation (both
+// CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue. Every wait is
+// bounded (see common.cuh).
+#include <atomic>
+
+#include "kernels.h"
+
+namespace bd {
+
+namespace {
+
+constexpr int BK = 128;                  // columns of d per pipeline stage (two 64-column swizzle atoms)
+constexpr int MAX_STAGES = 8;
+constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
+constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
+constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns
+constexpr int EPI_WARPS = 4;
+constexpr int TR = 33;  // padded row of the transpose buffers
+constexpr int MAX_CHUNKS = 8;
+
+struct PairCtl {
+  uint64_t full[MAX_STAGES];
+  uint64_t empty[MAX_STAGES];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint64_t epi_sync;  // rendezvous of the 128 epilogue threads (bounded, unlike bar.sync)
+  uint32_t tmem_base;
+  int abort_flag;
+};
+
+// One buffer per epilogue warp: the 32 x 33 transpose during the tiles of a
+// unit; after the warp's last tile, the same warp's running states (max, sum,
+// argmax for up to 256 tokens) for the cross-warp combine. A warp only ever
+// writes its own buffer before the rendezvous, so no warp can overwrite a
+// buffer another warp is still transposing in.
+struct PairWarpBuf {
+  union {
+    float tr[32 * TR];
+    struct {
+      float m[256];
+      float s[256];
+      int a[256];
+    } st;
+  };
+};
+
+struct PairTail {
+  PairWarpBuf w[EPI_WARPS];
+  PairCtl ctl;
+};
+
+constexpr size_t SMEM_BYTES = 232448;  // the whole opt-in shared memory of an SM
+constexpr size_t STAGE_AREA = SMEM_BYTES - 1024 - sizeof(PairTail);
+
+// Stage layout for a token group of NT rows (NT/2 in each CTA):
+//   [A block 0 | A block 1 | B block 0 | B block 1], A = 128 head rows,
+//   B = NT/2 token rows, each block 64 columns wide and 1 KB aligned.
+__host__ __device__ constexpr uint32_t stage_bytes(int nt) {
+  return 2 * A_BLOCK + 2 * static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES;
+}
+__host__ __device__ constexpr int stage_count(int nt) {
+  return static_cast<int>(STAGE_AREA / stage_bytes(nt)) < MAX_STAGES ? static_cast<int>(STAGE_AREA / stage_bytes(nt))
+                                                                     : MAX_STAGES;
+}
+static_assert(stage_count(256) >= 3, "three stages at NT = 256");
+
+}  // namespace
+
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW, TcArgs a) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  PairTail* tail = reinterpret_cast<PairTail*>(smem + STAGE_AREA);
+  PairCtl* ctl = &tail->ctl;
+  const uint32_t smem_base = smem_u32(smem);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: the CTA that issues the MMAs
+  const int pair = blockIdx.x >> 1;
+
+  if (threadIdx.x == 0) {
+    prefetch_tmap(&tmW);
+    for (int s = 0; s < MAX_STAGES; ++s) {
+      mbar_init(smem_u32(&ctl->full[s]), 1);
+      mbar_init(smem_u32(&ctl->empty[s]), 1);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(smem_u32(&ctl->tfull[i]), 1);
+      mbar_init(smem_u32(&ctl->tempty[i]), 2 * EPI_WARPS);
+    }
+    mbar_init(smem_u32(&ctl->drain), 1);
+    mbar_init(smem_u32(&ctl->epi_sync), EPI_WARPS * 32);
+    ctl->abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(&ctl->tmem_base), TMEM_COLS);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();  // barriers initialised and TMEM allocated in both CTAs
+  tc_fence_after();
+  const uint32_t tmem_base = ctl->tmem_base;
+  volatile int* abort_flag = &ctl->abort_flag;
+
+  const int n_rows = *a.n_rows;
+  const int nk = cdiv(a.d, BK);
+  const int NT = pair_group_rows(n_rows);
+  const int half = NT / 2;
+  const int nch = NT / 32;
+  const uint32_t SB = stage_bytes(NT);
+  const uint32_t B_BLOCK = static_cast<uint32_t>(half) * ATOM_ROWS_BYTES;
+  const int STAGES = stage_count(NT);
+  const uint32_t tx_total = 2u * SB;  // both CTAs' bytes land on the even CTA's barrier
+  const CUtensorMap* tm_tok = &tmH.m[half / 16 - 1];  // box of exactly `half` rows
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();  // head rows: streamed
+      const uint64_t pol_h = policy_evict_last();   // token rows: re-read for every v-tile
+      const uint32_t full0_leader = mapa_shared(smem_u32(&ctl->full[0]), 0);
+      uint32_t stage = 0, phase = 0;
+      uint32_t issued_mask = 0, issued_phase = 0;
+      TileIter it;
+      it.init(a.plan, n_rows, pair);
+      bool ok = true;
+      while (ok && it.next_unit()) {
+        const int tok0 = it.m_tile * NT + static_cast<int>(rank) * half;
+        for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+          const int vrow = vt * 256 + static_cast<int>(rank) * 128;
+          for (int kb = 0; kb < nk; ++kb) {
+            if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
+              ok = false;
+              break;
+            }
+            if (rank == 0) mbar_expect_tx(smem_u32(&ctl->full[stage]), tx_total);
+            const uint32_t fb = full0_leader + 8u * stage;
+            const uint32_t sa = smem_base + stage * SB;
+            tma_load_2d_pair(sa, &tmW, fb, kb * BK, vrow, pol_w);
+            tma_load_2d_pair(sa + A_BLOCK, &tmW, fb, kb * BK + 64, vrow, pol_w);
+            tma_load_2d_pair(sa + 2 * A_BLOCK, tm_tok, fb, kb * BK, tok0, pol_h);
+            tma_load_2d_pair(sa + 2 * A_BLOCK + B_BLOCK, tm_tok, fb, kb * BK + 64, tok0, pol_h);
+            issued_mask |= 1u << stage;
+            issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+      // The even CTA's full barriers count both CTAs' bytes: once they have
+      // flipped for the last issue of every stage, no copy is in flight.
+      if (rank == 0)
+        for (int s = 0; s < STAGES; ++s)
+          if (issued_mask & (1u << s)) mbar_drain(smem_u32(&ctl->full[s]), (issued_phase >> s) & 1u);
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------ MMA issuer (even CTA)
+    if (rank == 0 && lane == 0) {
+      const uint32_t idesc = idesc_bf16_f32(256, NT);
+      uint32_t stage = 0, phase = 0;
+      uint32_t acc = 0, acc_phase = 0;
+      TileIter it;
+      it.init(a.plan, n_rows, pair);
+      bool ok = true;
+      while (ok && it.next_unit()) {
+        for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+          if (!mbar_wait(smem_u32(&ctl->tempty[acc]), acc_phase ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + acc * 256;
+          for (int kb = 0; kb < nk; ++kb) {
+            if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t sa = smem_base + stage * SB;
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+              const uint64_t adesc = sw128_kmajor_desc(sa + j * A_BLOCK);
+              const uint64_t bdesc = sw128_kmajor_desc(sa + 2 * A_BLOCK + j * B_BLOCK);
+#pragma unroll
+              for (int k = 0; k < 4; ++k)
+                umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+            }
+            umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), 0x3);
+            if (++stage == STAGES) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (!ok) break;
+          umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
+          if (++acc == 2) {
+            acc = 0;
+            acc_phase ^= 1u;
+          }
+        }
+      }
+      umma_commit_pair_mc(smem_u32(&ctl->drain), 0x1);
+      mbar_drain(smem_u32(&ctl->drain), 0);
+    }
+  } else {
+    // ------------------------------------------------------ epilogue
+    const int ew = warp - 2;  // epilogue warp 0..3
+    const int quarter = warp & 3;
+    const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
+    float* tr = tail->w[ew].tr;
+    const uint32_t tempty_local0 = smem_u32(&ctl->tempty[0]);
+    const uint32_t tempty_leader0 = mapa_shared(tempty_local0, 0);
+    const uint32_t epi_sync = smem_u32(&ctl->epi_sync);
+    uint32_t epi_phase = 0;
+    uint32_t acc = 0, acc_phase = 0;
+    TileIter it;
+    it.init(a.plan, n_rows, pair);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      float m[MAX_CHUNKS], s[MAX_CHUNKS];
+      int arg[MAX_CHUNKS];
+#pragma unroll
+      for (int c = 0; c < MAX_CHUNKS; ++c) {
+        m[c] = -INFINITY;
+        s[c] = 0.f;
+        arg[c] = 0x7fffffff;
+      }
+      for (int vt = it.vt; vt < it.vt_end; ++vt) {
+        if (!mbar_wait_warp(smem_u32(&ctl->tfull[acc]), acc_phase, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int vrow0 = vt * 256 + static_cast<int>(rank) * 128 + quarter * 32;  // vocabulary row of lane 0
+        const int my_v = vrow0 + lane;
+        const bool dead = my_v >= a.V || my_v == a.mask_id;
+        const float sc = (a.wscale != nullptr && !dead) ? __ldg(a.wscale + my_v) : 1.f;
+#pragma unroll
+        for (int c = 0; c < MAX_CHUNKS; ++c) {
+          if (c < nch) {
+            float v[32];
+            tmem_ld32(tmem_base + lane_addr + acc * 256 + c * 32, v);
+#pragma unroll
+            for (int j = 0; j < 32; ++j) tr[lane * TR + j] = dead ? -INFINITY : v[j] * sc;
+            __syncwarp();
+            float x[32];
+#pragma unroll
+            for (int r = 0; r < 32; ++r) x[r] = tr[r * TR + lane];
+            __syncwarp();
+            // this thread: token column c*32 + lane, vocabulary rows vrow0 + r
+            float cm = x[0];
+#pragma unroll
+            for (int r = 1; r < 32; ++r) cm = fmaxf(cm, x[r]);
+            if (cm > m[c]) {
+              int rr = 31;
+#pragma unroll
+              for (int r = 31; r >= 0; --r)
+                if (x[r] == cm) rr = r;
+              arg[c] = vrow0 + rr;
+              s[c] = (m[c] == -INFINITY) ? 0.f : s[c] * ex2_approx((m[c] - cm) * LOG2E);
+              m[c] = cm;
+            }
+            if (m[c] != -INFINITY) {
+              const float mc = m[c] * LOG2E;
+              float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+              for (int r = 0; r < 32; r += 2) {
+                s0 += ex2_approx(fmaf(x[r], LOG2E, -mc));
+                s1 += ex2_approx(fmaf(x[r + 1], LOG2E, -mc));
+              }
+              s[c] += s0 + s1;
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) {
+          if (rank == 0)
+            mbar_arrive(tempty_local0 + 8u * acc);
+          else
+            mbar_arrive_cluster(tempty_leader0 + 8u * acc);
+        }
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      // combine the four warps' running states and write this CTA's partials
+#pragma unroll
+      for (int c = 0; c < MAX_CHUNKS; ++c) {
+        if (c < nch) {
+          tail->w[ew].st.m[c * 32 + lane] = m[c];
+          tail->w[ew].st.s[c * 32 + lane] = s[c];
+          tail->w[ew].st.a[c * 32 + lane] = arg[c];
+        }
+      }
+      mbar_arrive(epi_sync);
+      if (!mbar_wait_warp(epi_sync, epi_phase, abort_flag, a.status)) break;
+      epi_phase ^= 1u;
+      for (int j = ew * 32 + lane; j < NT; j += EPI_WARPS * 32) {
+        float M = tail->w[0].st.m[j], S = tail->w[0].st.s[j];
+        int A = tail->w[0].st.a[j];
+#pragma unroll
+        for (int w = 1; w < EPI_WARPS; ++w)
+          softmax_combine(M, S, A, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j]);
+        const int row = it.m_tile * NT + j;
+        if (row < n_rows) {
+          const int64_t o = static_cast<int64_t>(it.part * 2 + static_cast<int>(rank)) * a.P + row;
+          a.part_m[o] = M;
+          a.part_s[o] = S;
+          a.part_a[o] = A;
+        }
+      }
+      mbar_arrive(epi_sync);
+      if (!mbar_wait_warp(epi_sync, epi_phase, abort_flag, a.status)) break;
+      epi_phase ^= 1u;
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  cluster_sync_all();  // both CTAs done: no MMA, copy or remote arrival is pending
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+}
+
+size_t pair_smem_bytes() { return SMEM_BYTES; }
+
+static cudaError_t pair_opt_in() {
+  static std::atomic<uint64_t> opted_in{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if ((opted_in.load() & bit) == 0) {
+    e = cudaFuncSetAttribute(lmhead_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(SMEM_BYTES));
+    if (e != cudaSuccess) return e;
+    opted_in.fetch_or(bit);
+  }
+  return cudaSuccess;
+}
+
+static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int pairs, cudaStream_t st) {
+  *cfg = cudaLaunchConfig_t{};
+  cfg->gridDim = dim3(2 * pairs, 1, 1);
+  cfg->blockDim = dim3(TC_THREADS, 1, 1);
+  cfg->dynamicSmemBytes = SMEM_BYTES;
+  cfg->stream = st;
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg->attrs = attr;
+  cfg->numAttrs = 1;
+}
+
+cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs) {
+  cudaError_t e = pair_opt_in();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  pair_config(&cfg, attr, sm_count / 2, nullptr);
+  int n = 0;
+  e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel, &cfg);
+  if (e != cudaSuccess) return e;
+  *pairs = n < 1 ? 1 : n;
+  return cudaSuccess;
+}
+
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const TcArgs& a, cudaStream_t st) {
+  cudaError_t e = pair_opt_in();
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr[1];
+  pair_config(&cfg, attr, a.plan.G, st);
+  return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel, tmH, tmW, a);
+}
+
+}  // namespace bd

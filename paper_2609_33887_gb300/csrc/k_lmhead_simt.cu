@@ -4,7 +4,7 @@
 // the tensor-core kernel, with 32-row m-tiles and 256-entry v-tiles.
 #include <cuda_fp16.h>
 
-#include "../../include/bdcommit.h"
+#include "bdcommit.h"
 #include "kernels.h"
 
 namespace bd {

@@ -14,6 +14,8 @@
 //               thread), 32 columns at a time
 // Every wait is bounded; on timeout the CTA raises DEV_TIMEOUT in the status
 // word, drains its copies and MMAs, frees TMEM and returns.
+#include <atomic>
+
 #include "kernels.h"
 
 namespace bd {
@@ -256,9 +258,18 @@ static cudaError_t launch_stages(const CUtensorMap& tmA, const CUtensorMap& tmB,
                                  cudaStream_t st) {
   const size_t smem = tc_smem_bytes(STAGES);
   static_assert(STAGES <= 8, "Ctl holds 8 stages");
-  cudaError_t e = cudaFuncSetAttribute(lmhead_tc_kernel<STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem));
+  // the shared-memory opt-in is set once per device (not again inside a graph capture)
+  static std::atomic<uint64_t> opted_in{0};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
+  const uint64_t bit = 1ull << (dev & 63);
+  if ((opted_in.load() & bit) == 0) {
+    e = cudaFuncSetAttribute(lmhead_tc_kernel<STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(smem));
+    if (e != cudaSuccess) return e;
+    opted_in.fetch_or(bit);
+  }
   lmhead_tc_kernel<STAGES><<<a.plan.G, TC_THREADS, smem, st>>>(tmA, tmB, a);
   return cudaGetLastError();
 }

@@ -50,6 +50,17 @@ size_t tc_smem_bytes(int stages);
 cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const TcArgs& a, int stages,
                              cudaStream_t st);
 
+// a1+a2 on a CTA pair (tcgen05 cta_group::2), vocabulary on the MMA M side.
+// tmH.m[i] describes hc [P, d] bf16 with 64-column boxes of 16 * (i + 1) rows
+// (one per possible half token group), tmW the head [V, d] bf16 with 64 x 128
+// boxes. plan.G = CTA pairs, plan.BM = 0, plan.cpu = 2.
+struct PairTokenMaps {
+  CUtensorMap m[8];
+};
+size_t pair_smem_bytes();
+cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs);
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const TcArgs& a, cudaStream_t st);
+
 // a1+a2 with fp32 FMA on the CUDA cores (exact fp32 path; any dtype combo).
 struct SimtArgs {
   const void* hidden;

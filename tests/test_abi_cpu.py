@@ -113,7 +113,7 @@ def test_argument_checks(lib, kw, code):
 
 
 def test_variant_flags_and_outputs_checked(lib):
-    assert _call(lib, variant=3) == B.BD_ERR_ARG
+    assert _call(lib, variant=4) == B.BD_ERR_ARG
     assert _call(lib, flags=1) == B.BD_ERR_ARG
     assert _call(lib, variant=2, hdt=B.BD_F32, wdt=B.BD_F32) == B.BD_ERR_DTYPE
     assert _call(lib, outs=(None, FAKE, FAKE)) == B.BD_ERR_NULL

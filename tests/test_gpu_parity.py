@@ -90,18 +90,25 @@ def test_small_tensor_core(name):
     assert rep.n_live > 0
 
 
+@pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "bf16_2bands", "e4m3"])
+def test_small_one_cta_tensor_core_variant(name):
+    # variant 2: the one-CTA kernel with tokens on the MMA M side
+    wl = generate(SMALL[name])
+    check(wl, variant=2)
+
+
 @pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "e4m3"])
 def test_small_simt_variant(name):
     wl = generate(SMALL[name])
     check(wl, variant=1)
 
 
-def test_tc_and_simt_agree_on_argmax():
+def test_tensor_core_kernels_and_simt_agree():
     wl = generate(SMALL["bf16_5mt_ktail"])
-    a = run_gpu(wl, variant=2)
-    b = run_gpu(wl, variant=1)
-    assert np.array_equal(a["tokens"] < 0, b["tokens"] < 0)
-    assert np.abs(a["conf"] - b["conf"]).max() < 1e-3
+    outs = [run_gpu(wl, variant=v) for v in (3, 2, 1)]
+    for o in outs[1:]:
+        assert np.array_equal(outs[0]["tokens"] < 0, o["tokens"] < 0)
+        assert np.abs(outs[0]["conf"] - o["conf"]).max() < 1e-3
 
 
 # -------------------------------------------------------------- edge cases --
@@ -200,4 +207,14 @@ def test_full_size_sampled_blocks(i, n_blocks):
     wl = generate(CONFIGS[i])
     blocks = _sample_blocks(CONFIGS[i], n_blocks)
     _, _, rep = check(wl, blocks=blocks)
+    assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("i,variant,n_blocks", [(1, 2, None), (3, 3, 3), (4, 3, 2)])
+def test_full_size_with_the_other_tensor_core_kernel(i, variant, n_blocks):
+    # the automatic choice takes the CTA-pair kernel for the 8x2x32 window and
+    # the one-CTA kernel for the two largest; check each with the other kernel
+    wl = generate(CONFIGS[i])
+    blocks = None if n_blocks is None else _sample_blocks(CONFIGS[i], n_blocks, seed=5)
+    _, _, rep = check(wl, variant=variant, blocks=blocks)
     assert rep.n_live > 0
