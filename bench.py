@@ -300,8 +300,16 @@ def run_ours(args):
     if st != 0:
         raise B.BdError(st, "warm-up")
 
-    # per-step LM-head events: recorded on the launching stream inside the timed region
-    evs = timing_events(K, stream)
+    # LM-head events on every EVENT_STRIDE-th step of the timed region (on the
+    # launching stream): an event node between two kernels turns their
+    # programmatic (overlapped) launch back into full serialisation, so timing
+    # every step would slow every step down
+    EVENT_STRIDE = 10
+    ev_steps = list(range(0, K, EVENT_STRIDE))
+    evs_list = timing_events(len(ev_steps), stream)
+    evs = [None] * K
+    for j, i in enumerate(ev_steps):
+        evs[i] = evs_list[j]
     graph = None
     if args.graph:
         # the K timed steps as one CUDA graph (the serving engine also replays captured graphs)
@@ -331,7 +339,7 @@ def run_ours(args):
         pg.barrier()
     clocks = sampler.stop()
     elapsed_ms = t_start.elapsed_time(t_end)
-    lm_ms = [a.elapsed_time(b) for a, b in evs]
+    lm_ms = [a.elapsed_time(b) for a, b in evs_list]
     st = B.bd_get_device_status(stream)
     if st != 0:
         raise B.BdError(st, "timed region")
@@ -385,7 +393,8 @@ def run_ours(args):
         e2e = {"value": total_masked * K / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h),
                "note": "pinned host hidden states + mask state in, tokens/conf/commit/counts out, per step; "
-                       "LM-head weights stay resident in HBM"}
+                       "LM-head weights stay resident in HBM"
+                       + ("; the K steps replayed as one CUDA graph" if args.graph else "")}
 
     # ---- roofline of the dominant kernel (LM head)
     hbm_gbs, tc_tflops, tc_sus, peak_src = peaks()
@@ -405,6 +414,7 @@ def run_ours(args):
         roof = {"bound": "hbm", "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
                 "frac": achieved / hbm_gbs, "traffic": traffic, "peak_source": f"hbm_gbs of {peak_src}"}
     roof["lmhead_ms_avg"] = lmhead_ms = statistics.mean(lm_ms)
+    roof["lmhead_launches_timed"] = len(lm_ms)
     roof["hbm_view"] = {"algorithmic_bytes": abytes, "achieved_gbs": abytes / lm_avg_s / 1e9,
                         "frac": abytes / lm_avg_s / 1e9 / hbm_gbs}
     roof["algorithmic_flops"] = flops

@@ -140,6 +140,7 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   // windows both kernels saturate the tensor pipe under the power cap and the
   // one-CTA kernel runs slightly faster
   c->pair = tc && (variant == 3 || (variant == 0 && P <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
+
   c->ldh = h->ld;
   c->ldw = w->ld;
   c->ldc = round_up(c->d, 8);
@@ -252,17 +253,21 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   int* pa = reinterpret_cast<int*>(ws + lay.pa);
   const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
 
-  // a0: compaction of the masked positions of active blocks
-  int rc = cuda_status(
-      bd::launch_compact(mask_state->pos_masked, mask_state->block_flags, P, c.L, idx, rowpos, n_rows, st));
+  if (out_counts) {
+    if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
+      return BD_ERR_CUDA;
+  }
+
+  // a0: compaction of the masked positions of active blocks (+ packing of their rows)
+  int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
+                                            c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
+                                            c.ldc, idx, rowpos, n_rows, sm_count, st));
   if (rc != BD_OK) return rc;
 
   CUtensorMap tmA, tmB;
   bd::PairTokenMaps tmTok;
   if (c.tc) {
     void* hc = ws + lay.hc;
-    rc = cuda_status(bd::launch_pack_rows_bf16(hidden->data, c.ldh, d, idx, n_rows, P, hc, c.ldc, sm_count, st));
-    if (rc != BD_OK) return rc;
     const void* wsrc = weight->data;
     int64_t wld = c.ldw;
     if (c.wdt == BD_E4M3) {
@@ -282,11 +287,6 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
       if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
       if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
     }
-  }
-
-  if (out_counts) {
-    if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
-      return BD_ERR_CUDA;
   }
 
   // a1 + a2: LM head with the online softmax epilogue

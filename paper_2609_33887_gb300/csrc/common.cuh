@@ -352,6 +352,16 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// ---- programmatic dependent launch ------------------------------------------
+// Blocks until the grid this one depends on has completed and its writes are
+// visible (a no-op when the launch carries no programmatic dependency).
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the dependent grid be scheduled once every CTA of this grid has called
+// it (or exited).
+__device__ __forceinline__ void griddep_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 // ---- clusters and the CTA pair (cta_group::2) ----------------------------
 __device__ __forceinline__ uint32_t cluster_ctarank() {
   uint32_t r;

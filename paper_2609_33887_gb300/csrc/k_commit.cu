@@ -26,6 +26,7 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
   const int L = a.block_len;
   const int64_t base = static_cast<int64_t>(blk) * L;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  griddep_wait();  // the partials come from the LM-head kernel
   const int n_rows = *a.n_rows;
 
   // ---- a3: merge of the partial slots. Thread t takes position t % Lp of the
@@ -149,8 +150,16 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
 }
 
 cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st) {
-  merge_commit_kernel<<<a.n_blocks, THREADS, 0, st>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.n_blocks, 1, 1);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, merge_commit_kernel, a);
 }
 
 }  // namespace bd

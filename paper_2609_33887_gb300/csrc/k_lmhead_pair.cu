@@ -129,6 +129,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t tmem_base = ctl->tmem_base;
   volatile int* abort_flag = &ctl->abort_flag;
 
+  griddep_wait();  // the packed rows and N come from the preceding kernel
   const int n_rows = *a.n_rows;
   const int nk = cdiv(a.d, BK);
   const int NT = pair_group_rows(n_rows);
@@ -348,6 +349,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   }
 
   __syncwarp();
+  griddep_launch_dependents();
   tc_fence_before();
   cluster_sync_all();  // both CTAs done: no MMA, copy or remote arrival is pending
   tc_fence_after();
@@ -371,7 +373,8 @@ static cudaError_t pair_opt_in() {
   return cudaSuccess;
 }
 
-static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int pairs, cudaStream_t st) {
+static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int pairs, cudaStream_t st,
+                        bool programmatic) {
   *cfg = cudaLaunchConfig_t{};
   cfg->gridDim = dim3(2 * pairs, 1, 1);
   cfg->blockDim = dim3(TC_THREADS, 1, 1);
@@ -383,14 +386,19 @@ static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int 
   attr[0].val.clusterDim.z = 1;
   cfg->attrs = attr;
   cfg->numAttrs = 1;
+  if (programmatic) {
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg->numAttrs = 2;
+  }
 }
 
 cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs) {
   cudaError_t e = pair_opt_in();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
-  cudaLaunchAttribute attr[1];
-  pair_config(&cfg, attr, sm_count / 2, nullptr);
+  cudaLaunchAttribute attr[2];
+  pair_config(&cfg, attr, sm_count / 2, nullptr, false);
   int n = 0;
   e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel, &cfg);
   if (e != cudaSuccess) return e;
@@ -402,8 +410,8 @@ cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
   cudaError_t e = pair_opt_in();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
-  cudaLaunchAttribute attr[1];
-  pair_config(&cfg, attr, a.plan.G, st);
+  cudaLaunchAttribute attr[2];
+  pair_config(&cfg, attr, a.plan.G, st, true);
   return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel, tmH, tmW, a);
 }
 

@@ -48,6 +48,7 @@ struct SimtSmem {
 __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   __shared__ SimtSmem sm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  griddep_wait();  // idx and N come from the preceding kernel
   const int n_rows = *a.n_rows;
 
   TileIter it;
@@ -131,11 +132,20 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
     }
     __syncthreads();
   }
+  griddep_launch_dependents();
 }
 
 cudaError_t launch_lmhead_simt(const SimtArgs& a, cudaStream_t st) {
-  lmhead_simt_kernel<<<a.plan.G, THREADS, 0, st>>>(a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.plan.G, 1, 1);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, lmhead_simt_kernel, a);
 }
 
 }  // namespace bd

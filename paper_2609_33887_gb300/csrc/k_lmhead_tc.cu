@@ -78,6 +78,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const uint32_t tmem_base = ctl->tmem_base;
   volatile int* abort_flag = &ctl->abort_flag;
 
+  griddep_wait();  // the packed rows and N come from the preceding kernel
   const int n_rows = *a.n_rows;
   const int nk = cdiv(a.d, BK);
 
@@ -245,6 +246,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   }
 
   __syncwarp();
+  griddep_launch_dependents();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -270,8 +272,17 @@ static cudaError_t launch_stages(const CUtensorMap& tmA, const CUtensorMap& tmB,
     if (e != cudaSuccess) return e;
     opted_in.fetch_or(bit);
   }
-  lmhead_tc_kernel<STAGES><<<a.plan.G, TC_THREADS, smem, st>>>(tmA, tmB, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.plan.G, 1, 1);
+  cfg.blockDim = dim3(TC_THREADS, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, lmhead_tc_kernel<STAGES>, tmA, tmB, a);
 }
 
 cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const TcArgs& a, int stages,

@@ -6,110 +6,126 @@
 namespace bd {
 
 // ---------------------------------------------------------------------------
-// Compaction (one CTA). Only masked positions of active blocks need a
-// prediction (App. F: the accept threshold resolves positions of active
-// blocks). Rows keep ascending position order, so the masked positions of a
-// block are consecutive rows.
+// Compaction and row packing in one launch. Only masked positions of active
+// blocks need a prediction (App. F: the accept threshold resolves positions of
+// active blocks). Rows keep ascending position order, so the masked positions
+// of a block are consecutive rows.
+//
+// CTA c owns positions [c*chunk, (c+1)*chunk). It counts the live positions
+// before its chunk itself (no inter-CTA communication), scans its chunk, writes
+// idx / rowpos for it, copies the hidden rows of its live positions into hc
+// (bf16 tensor-core paths) and, if it holds the last position, writes N.
 // ---------------------------------------------------------------------------
-constexpr int COMPACT_THREADS = 1024;
-constexpr int COMPACT_ITEMS = 8;
+constexpr int PREP_THREADS = 256;
 
-__global__ void __launch_bounds__(COMPACT_THREADS) compact_kernel(const uint8_t* __restrict__ pos_masked,
-                                                                  const uint8_t* __restrict__ block_flags,
-                                                                  int P, int block_len, int* __restrict__ idx,
-                                                                  int* __restrict__ rowpos,
-                                                                  int* __restrict__ n_rows) {
-  __shared__ int warp_tot[COMPACT_THREADS / 32];
-  __shared__ int carry_s;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) carry_s = 0;
+__device__ __forceinline__ int live_at(const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags,
+                                       int p, int block_len) {
+  return (pos_masked[p] != 0 && (block_flags[p / block_len] & 1u)) ? 1 : 0;
+}
+
+__device__ __forceinline__ int block_sum(int v, int* red) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  if (lane == 0) red[warp] = v;
   __syncthreads();
-  for (int base = 0; base < P; base += COMPACT_THREADS * COMPACT_ITEMS) {
-    const int p0 = base + tid * COMPACT_ITEMS;
-    uint32_t live = 0;
-    int cnt = 0;
-#pragma unroll
-    for (int i = 0; i < COMPACT_ITEMS; ++i) {
-      int p = p0 + i;
-      if (p < P && pos_masked[p] != 0 && (block_flags[p / block_len] & 1u)) {
-        live |= 1u << i;
-        ++cnt;
-      }
-    }
-    int incl = cnt;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      int t = __shfl_up_sync(0xffffffffu, incl, o);
-      if (lane >= o) incl += t;
-    }
-    if (lane == 31) warp_tot[warp] = incl;
-    __syncthreads();
-    if (warp == 0) {
-      int w = warp_tot[lane];
-      int wi = w;
-#pragma unroll
-      for (int o = 1; o < 32; o <<= 1) {
-        int t = __shfl_up_sync(0xffffffffu, wi, o);
-        if (lane >= o) wi += t;
-      }
-      warp_tot[lane] = wi - w;  // exclusive prefix of the warp totals
-    }
-    __syncthreads();
-    const int carry = carry_s;
-    int r = carry + warp_tot[warp] + incl - cnt;
-#pragma unroll
-    for (int i = 0; i < COMPACT_ITEMS; ++i) {
-      int p = p0 + i;
-      if (p < P) {
-        if (live & (1u << i)) {
-          idx[r] = p;
-          rowpos[p] = r;
-          ++r;
-        } else {
-          rowpos[p] = -1;
-        }
-      }
-    }
-    __syncthreads();
-    if (tid == COMPACT_THREADS - 1) carry_s = r;  // last thread ends at the chunk total
-    __syncthreads();
+  int t = 0;
+  for (int w = 0; w < PREP_THREADS / 32; ++w) t += red[w];
+  __syncthreads();
+  return t;
+}
+
+__global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
+    const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags, int P, int block_len, int chunk,
+    const __nv_bfloat16* __restrict__ hidden, int64_t ld, int d, __nv_bfloat16* __restrict__ hc, int64_t ldc,
+    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows) {
+  __shared__ int red[PREP_THREADS / 32];
+  __shared__ int warp_excl[PREP_THREADS / 32];
+  __shared__ int rows_s[2048];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  griddep_launch_dependents();  // every CTA of this grid is resident once all have got here
+  const int p0 = blockIdx.x * chunk;
+  const int p1 = min(P, p0 + chunk);
+
+  // 1. live positions before this chunk
+  int before = 0;
+  for (int p = tid; p < p0; p += PREP_THREADS) before += live_at(pos_masked, block_flags, p, block_len);
+  const int prefix = block_sum(before, red);
+
+  // 2. exclusive scan of the chunk: thread t takes `per` consecutive positions
+  const int per = (chunk + PREP_THREADS - 1) / PREP_THREADS;
+  const int q0 = p0 + tid * per;
+  int cnt = 0;
+  for (int i = 0; i < per; ++i) {
+    const int p = q0 + i;
+    if (p < p1) cnt += live_at(pos_masked, block_flags, p, block_len);
   }
-  if (tid == 0) *n_rows = carry_s;
-}
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int t = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += t;
+  }
+  if (lane == 31) warp_excl[warp] = incl;
+  __syncthreads();
+  if (tid == 0) {
+    int run = 0;
+    for (int w = 0; w < PREP_THREADS / 32; ++w) {
+      const int t = warp_excl[w];
+      warp_excl[w] = run;
+      run += t;
+    }
+    red[0] = run;  // live positions of the chunk
+  }
+  __syncthreads();
+  const int local_total = red[0];
+  int r = prefix + warp_excl[warp] + incl - cnt;
+  for (int i = 0; i < per; ++i) {
+    const int p = q0 + i;
+    if (p < p1) {
+      if (live_at(pos_masked, block_flags, p, block_len)) {
+        idx[r] = p;
+        rowpos[p] = r;
+        if (r - prefix < 2048) rows_s[r - prefix] = p;
+        ++r;
+      } else {
+        rowpos[p] = -1;
+      }
+    }
+  }
+  if (p1 == P && tid == 0) *n_rows = prefix + local_total;
+  if (hidden == nullptr) return;
+  __syncthreads();
 
-cudaError_t launch_compact(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len, int* idx,
-                           int* rowpos, int* n_rows, cudaStream_t st) {
-  compact_kernel<<<1, COMPACT_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, idx, rowpos, n_rows);
-  return cudaGetLastError();
-}
-
-// ---------------------------------------------------------------------------
-// Row packing: hc[r, :] = hidden[idx[r], :] for r < N (bf16, 16-byte vectors
-// when the width allows).
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(256) pack_rows_bf16_kernel(const __nv_bfloat16* __restrict__ hidden, int64_t ld,
-                                                             int d, const int* __restrict__ idx,
-                                                             const int* __restrict__ n_rows,
-                                                             __nv_bfloat16* __restrict__ hc, int64_t ldc) {
-  const int N = *n_rows;
+  // 3. copy the chunk's live rows, one warp per row, 16-byte vectors
   const int nvec = d / 8;
-  for (int r = blockIdx.x; r < N; r += gridDim.x) {
-    const __nv_bfloat16* src = hidden + static_cast<int64_t>(idx[r]) * ld;
-    __nv_bfloat16* dst = hc + static_cast<int64_t>(r) * ldc;
+  for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+    const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
+    const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
+    __nv_bfloat16* dst = hc + static_cast<int64_t>(prefix + i) * ldc;
     const uint4* s4 = reinterpret_cast<const uint4*>(src);
     uint4* d4 = reinterpret_cast<uint4*>(dst);
-    for (int i = threadIdx.x; i < nvec; i += blockDim.x) d4[i] = __ldg(s4 + i);
-    for (int i = nvec * 8 + threadIdx.x; i < d; i += blockDim.x) dst[i] = src[i];
+    for (int v = lane; v < nvec; v += 32) d4[v] = __ldg(s4 + v);
+    for (int e = nvec * 8 + lane; e < d; e += 32) dst[e] = src[e];
   }
 }
 
-cudaError_t launch_pack_rows_bf16(const void* hidden, int64_t ld, int d, const int* idx, const int* n_rows, int P,
-                                  void* hc, int64_t ldc, int sm_count, cudaStream_t st) {
-  int grid = sm_count * 8;
-  if (grid > P) grid = P;
-  if (grid < 1) grid = 1;
-  pack_rows_bf16_kernel<<<grid, 256, 0, st>>>(static_cast<const __nv_bfloat16*>(hidden), ld, d, idx, n_rows,
-                                              static_cast<__nv_bfloat16*>(hc), ldc);
+int prep_chunk(int P, int sm_count) {
+  int chunk = (P + 2 * sm_count - 1) / (2 * sm_count);
+  chunk = (chunk + 31) / 32 * 32;
+  if (chunk < 32) chunk = 32;
+  if (chunk > 2048) chunk = 2048;
+  return chunk;
+}
+
+cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
+                             const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
+                             int* n_rows, int sm_count, cudaStream_t st) {
+  const int chunk = prep_chunk(P, sm_count);
+  const int grid = (P + chunk - 1) / chunk;
+  prep_rows_kernel<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
+                                                  static_cast<const __nv_bfloat16*>(hidden), ld, d,
+                                                  static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows);
   return cudaGetLastError();
 }
 

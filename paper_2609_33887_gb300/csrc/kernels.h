@@ -16,15 +16,13 @@ struct TauParams {
   int T;
 };
 
-// a0: compaction of the masked positions of active blocks (Sec. 2.1 / App. F
-// slot states). Writes idx[r] = position of compacted row r (ascending
-// positions), rowpos[p] = r or -1, and *n_rows = N.
-cudaError_t launch_compact(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
-                           int* idx, int* rowpos, int* n_rows, cudaStream_t st);
-
-// Packs the hidden rows of the compacted positions: hc[r] = hidden[idx[r]], bf16.
-cudaError_t launch_pack_rows_bf16(const void* hidden, int64_t ld, int d, const int* idx, const int* n_rows,
-                                  int P, void* hc, int64_t ldc, int sm_count, cudaStream_t st);
+// a0: compaction of the masked positions of active blocks (App. F slot
+// states) and, when `hidden` is not null, packing of their bf16 rows into hc.
+// Writes idx[r] = position of compacted row r (ascending positions),
+// rowpos[p] = r or -1, hc[r] = hidden[idx[r]] and *n_rows = N.
+cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
+                             const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
+                             int* n_rows, int sm_count, cudaStream_t st);
 
 // Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,

@@ -70,6 +70,9 @@ SMALL = {
     "bf16_2bands": scaled(CONFIGS[2], n_seq=32, n_slots=4, d=128, V=2148),
     # block_len 64, 16 thresholds
     "bf16_L64": scaled(CONFIGS[3], n_seq=4, n_slots=4, d=192, V=4000),
+    # 257..320 rows: two token groups of the CTA-pair kernel
+    "bf16_g294": scaled(CONFIGS[1], d=256, V=3000, mask_frac=0.6),
+    "bf16_g271_mask": scaled(CONFIGS[1], d=320, V=2600, mask_frac=0.53, mask_token_id=2599),
     # FP8 head with per-row scales
     "e4m3": scaled(CONFIGS[4], n_seq=4, n_slots=4, d=512, V=5000),
     "e4m3_ktail": scaled(CONFIGS[4], n_seq=3, n_slots=2, d=80, V=700),
