@@ -36,8 +36,9 @@ from workloads import CONFIGS, by_name, generate  # noqa: E402
 DEFAULT_CONFIG = CONFIGS[1].name
 METRIC = "masked positions/s through fused LM-head+confidence+commit"
 UNIT = "positions/s"
-KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_tc.cu", "paper_2609_33887_gb300/csrc/common.cuh"]
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_tc_traffic.txt")
+# the LM-head kernel the automatic choice runs on the 8x2x32 window (the CTA-pair kernel)
+KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_pair.cu", "paper_2609_33887_gb300/csrc/common.cuh"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_pair_traffic.txt")
 
 
 def parse_args():
