@@ -1,4 +1,5 @@
-"""Float64 CPU oracle for the block-diffusion commit step.
+"""CPU oracles: float64 for the block-diffusion commit step, exact rationals
+for the Redline selection.
 
 TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and
 ``bench.py`` (its ``cpu_baseline`` leg and its ``--impl reference`` arm) may
@@ -9,9 +10,14 @@ Parity status: every function here is pinned by ``tests/test_oracle_pins.py``
 (closed forms, a 50-digit brute force, invariants, a logsumexp cross-check and
 hand-derived commit-rule cases). The only reading that no paper number can pin
 is which blocks may take the top-1 fallback: that is an input (the caller's
-``block_flags``), not a computation of the oracle.
+``block_flags``), not a computation of the oracle. ``redline_oracle`` is
+pinned by ``tests/test_redline_oracle.py`` (every p-value, valid mark and
+deployment of the paper's appendix grid tables, the calibration-size table,
+brute-force enumeration, closed-testing identities and an exact family-wise
+error).
 """
 
+from . import redline_oracle
 from .commit_oracle import (
     ACTIVE,
     FALLBACK_ELIGIBLE,
@@ -32,6 +38,7 @@ __all__ = [
     "decode_bf16",
     "decode_e4m3",
     "lm_head_logits",
+    "redline_oracle",
     "row_confidence",
     "weights_f64",
 ]
