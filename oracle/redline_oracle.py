@@ -101,6 +101,20 @@ def _scaled_terms(n: int, a: Fraction):
             t = t * (n - j) * num // ((j + 1) * q)
 
 
+def binom_cdf_sum(k: int, n: int, alpha) -> Fraction:
+    """The same sum as binom_cdf, accumulated over the exact integer terms of
+    _scaled_terms and normalised once (fast for large n and any alpha)."""
+    a = as_fraction(alpha)
+    if k < 0:
+        return Fraction(0)
+    acc = 0
+    for j, t in enumerate(_scaled_terms(n, a)):
+        if j > k:
+            break
+        acc += t
+    return Fraction(acc, a.denominator**n)
+
+
 def binom_cdf_table(n: int, alpha, k_max: int) -> List[Fraction]:
     """[Pr[Bin(n, alpha) <= k] for k = 0..k_max], accumulated once over the terms."""
     a = as_fraction(alpha)
@@ -118,7 +132,7 @@ def binom_cdf_table(n: int, alpha, k_max: int) -> List[Fraction]:
 
 def p_value(V: int, n: int, alpha) -> Fraction:
     """p = Pr_{Bin(n, alpha)}[S <= V] for H0: R > alpha (exact-binomial appendix)."""
-    return binom_cdf(V, n, alpha)
+    return binom_cdf_sum(V, n, alpha)
 
 
 def p_values(V: Sequence[int], n: int, alpha) -> List[Fraction]:
@@ -239,15 +253,7 @@ def power(n: int, R, alpha, level) -> Fraction:
     """Probability that a configuration of true risk R passes a test at `level`:
     Pr[Bin(n, R) <= critical_count(n, alpha, level)]."""
     c = critical_count(n, alpha, level)
-    if c < 0:
-        return Fraction(0)
-    r = as_fraction(R)
-    acc = 0
-    for j, t in enumerate(_scaled_terms(n, r)):
-        if j > c:
-            break
-        acc += t
-    return Fraction(acc, r.denominator**n)
+    return binom_cdf_sum(c, n, R) if c >= 0 else Fraction(0)
 
 
 # --------------------------------------------------------------------------

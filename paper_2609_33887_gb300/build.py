@@ -1,8 +1,9 @@
 """Build libbdcommit.so in-tree with nvcc for sm_103a.
 
-Each CUDA translation unit is compiled in parallel, then linked into one
-shared library (static CUDA runtime, no link-time dependency on libcuda: the
-tensor-map encoder is fetched through the runtime's driver entry point).
+Each translation unit (CUDA .cu, host-only C++ .cpp) is compiled in
+parallel, then linked into one shared library (static CUDA runtime, no
+link-time dependency on libcuda: the tensor-map encoder is fetched through the
+runtime's driver entry point).
 A stamp of the sources and flags skips the build when nothing changed.
 """
 
@@ -37,7 +38,7 @@ def _nvcc() -> str:
 
 
 def _sources():
-    return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith(".cu"))
+    return sorted(os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cu", ".cpp")))
 
 
 def _stamp(nvcc: str, extra) -> str:
@@ -45,7 +46,7 @@ def _stamp(nvcc: str, extra) -> str:
     h.update(" ".join([nvcc] + NVCC_FLAGS + list(extra)).encode())
     files = _sources() + sorted(
         os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))
-    ) + [os.path.join(INCLUDE, "bdcommit.h")]
+    ) + sorted(os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h"))
     for f in files:
         h.update(f.encode())
         with open(f, "rb") as fh:
@@ -54,7 +55,7 @@ def _stamp(nvcc: str, extra) -> str:
 
 
 def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
-    """Compile every CUDA source and link libbdcommit.so; returns its path."""
+    """Compile every source and link libbdcommit.so; returns its path."""
     nvcc = _nvcc()
     os.makedirs(BUILD, exist_ok=True)
     stamp_file = os.path.join(BUILD, "libbdcommit.stamp")
@@ -65,7 +66,7 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
                 return LIB
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+        obj = os.path.join(BUILD, os.path.splitext(os.path.basename(src))[0] + ".o")
         cmd = [nvcc] + NVCC_FLAGS + list(extra_flags) + ["-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:

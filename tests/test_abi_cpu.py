@@ -1,6 +1,6 @@
 """The C-ABI library without a GPU: it builds, loads, exports every symbol
-include/bdcommit.h declares (and nothing else), and its argument checks
-reject bad calls before any CUDA call."""
+the headers under include/ declare (and nothing else), and its argument
+checks reject bad calls before any CUDA call."""
 
 import ctypes
 import math
@@ -14,7 +14,8 @@ import pytest
 from paper_2609_33887_gb300 import bdcommit as B
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-HEADER = os.path.join(ROOT, "include", "bdcommit.h")
+INCLUDE = os.path.join(ROOT, "include")
+HEADERS = sorted(os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h"))
 
 
 @pytest.fixture(scope="module")
@@ -28,15 +29,20 @@ def lib():
 
 
 def declared_functions():
-    text = open(HEADER).read()
-    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:int|size_t|const char\*)\s+(bd_\w+)\s*\(", text, flags=re.M)))
+    names = set()
+    for h in HEADERS:
+        text = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"^\s*(?:int|size_t|const char\*)\s+(bd_\w+)\s*\(", text, flags=re.M))
+    return sorted(names)
 
 
 def test_header_declares_the_abi():
     assert declared_functions() == sorted([
         "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_get_device_status", "bd_shutdown",
-        "bd_status_string", "bd_version", "bd_workspace_size"])
+        "bd_status_string", "bd_version", "bd_workspace_size",
+        "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
+        "bd_redline_select", "bd_redline_sweep", "bd_redline_critical_count", "bd_redline_power",
+        "bd_redline_min_calibration", "bd_redline_tpf"])
 
 
 def test_library_exports_every_declared_symbol(lib):

@@ -26,6 +26,7 @@ import numpy as np
 import pytest
 
 from oracle import redline_oracle as R
+from tests.redline_helpers import exact_holm_fwer_nested
 from workloads.redline_inputs import losses_matrix, outcome_matrix
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "redline_grids.json")
@@ -243,9 +244,11 @@ def test_cdf_closed_forms():
         assert all(x > y for x, y in zip(ps, ps[1:]))
     # the reference row of every grid: V = 0 gives (1 - alpha)^n, printed 3e-23 at n = 1012, alpha = 0.05
     assert printed_match(R.p_value(0, 1012, F("0.05")), "3e-23")
-    # table and critical count agree with the direct sum
+    # table, integer-term sum and critical count agree with the direct sum
     tab = R.binom_cdf_table(300, F("0.07"), 320)
     assert tab == [R.binom_cdf(k, 300, F("0.07")) for k in range(321)]
+    for a in (F(0), F(1), F(0.3), F("0.07")):
+        assert all(R.binom_cdf_sum(k, 60, a) == R.binom_cdf(k, 60, a) for k in range(-1, 62))
     for lv in (F(1, 1000), F(1, 80), F(1, 10), F(1, 2)):
         c = R.critical_count(300, F("0.07"), lv)
         assert all((t <= lv) == (k <= c) for k, t in enumerate(tab))
@@ -355,39 +358,6 @@ def test_tpf_from_counts():
 # --------------------------------------------------------------------------
 # family-wise error (validity appendix, synthetic Monte Carlo)
 # --------------------------------------------------------------------------
-def exact_holm_fwer_nested(n, alpha, delta, risks):
-    """FWER of Holm when every configuration's losses come from one shared
-    uniform per prompt (risks sorted ascending, one per hypothesis of the
-    family). The counts are nested, V_0 <= V_1 <= ..., so the sorted p-values
-    follow the risk order, and Holm rejects a hypothesis with R > alpha only
-    if it rejects the first of them, at sorted position f: that needs
-    V_i <= c_i for every i <= f, with c_i the critical count at
-    delta / (m - i). The V_i are prefix sums of multinomial cell counts of the
-    uniform over [0, r_0), [r_0, r_1), ..., [r_{f-1}, r_f) and [r_f, 1)."""
-    m = len(risks)
-    assert list(risks) == sorted(risks)
-    tab = R.binom_cdf_table(n, alpha, n)
-    crit = [max([v for v in range(n + 1) if tab[v] <= delta / (m - i)], default=-1) for i in range(m)]
-    f = next(i for i, r in enumerate(risks) if r > alpha)
-    widths = [float(risks[0])] + [float(risks[i] - risks[i - 1]) for i in range(1, f + 1)]
-    rest = 1.0 - float(risks[f])
-    lg = math.lgamma
-    total = 0.0
-
-    def rec(i, used, logp):
-        nonlocal total
-        if i > f:
-            r = n - used
-            total += math.exp(lg(n + 1) + logp - lg(r + 1) + r * math.log(rest))
-            return
-        top = crit[i] - used if widths[i] > 0 else min(0, crit[i] - used)
-        for c in range(0, top + 1):
-            rec(i + 1, used + c, logp + (c * math.log(widths[i]) if c else 0.0) - lg(c + 1))
-
-    rec(0, 0, 0.0)
-    return total
-
-
 def test_montecarlo_fwer_paper_setting():
     """Five configurations of true risk {0.01, 0.02, 0.07, 0.07, 0.07}, alpha =
     0.05, n = 800, shared uniform: the exact FWER of Holm is far below delta
