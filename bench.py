@@ -249,6 +249,47 @@ def run_reference(args):
 
 
 # ---------------------------------------------------------------- our arm --
+def redline_timing(with_oracle: bool) -> dict:
+    """Host time of the Redline selection (libbdcommit, include/redline.h) on a
+    grid shaped like the paper's largest (m = 50 configurations, n = 1012
+    prompts, seeded synthetic outcomes): counting + p-values + Holm + deployment
+    at one budget, and a sweep over 30 budgets; beside it the exact oracle on
+    the same grid at one budget."""
+    from paper_2609_33887_gb300 import redline as N
+    from workloads.redline_inputs import random_grid
+
+    gr = random_grid(1012, 50, seed=3)
+    alphas = [i / 100 for i in range(1, 31)]
+
+    def best_us(fn, min_s=0.2):
+        reps, t0 = 0, time.perf_counter()
+        while True:
+            fn()
+            reps += 1
+            dt = time.perf_counter() - t0
+            if dt >= min_s and reps >= 5:
+                return dt / reps * 1e6
+
+    def select():
+        V = N.bd_redline_violations(gr.outcomes, gr.ref)
+        return N.bd_redline_select(V, gr.cost, 1012, 0.10, gr.ref)["deployed"]
+
+    V = N.bd_redline_violations(gr.outcomes, gr.ref)
+    out = {"grid": "m50 n1012 synthetic outcomes, delta 0.10, Holm",
+           "select_us": best_us(select),
+           "sweep30_us": best_us(lambda: N.bd_redline_sweep(V, gr.cost, 1012, alphas, gr.ref)),
+           "deployed": select()}
+    if with_oracle:
+        from oracle import redline_oracle as RO
+
+        t0 = time.perf_counter()
+        Vo = RO.joint_violations(gr.outcomes.tolist(), gr.ref)
+        dep = RO.redline(Vo, list(gr.cost), 1012, 0.10, 0.10, gr.ref)["deployed"]
+        out["oracle_select_ms"] = (time.perf_counter() - t0) * 1e3
+        out["oracle_agrees"] = dep == out["deployed"]
+    return out
+
+
 def run_ours(args):
     import paper_2609_33887_gb300 as bdc
     from paper_2609_33887_gb300 import bdcommit as B
@@ -292,7 +333,9 @@ def run_ours(args):
         if rc != 0:
             raise B.BdError(rc)
 
-    launches_per_step = 4 + (1 if cfg.weight_dtype == "e4m3" else 0)
+    # library kernels per step: compaction + row packing, LM head, merge + commit
+    # (+ the e4m3 decode); the counts reset is a runtime memset, not one of ours
+    launches_per_step = 3 + (1 if cfg.weight_dtype == "e4m3" else 0)
     K, W = args.steps, args.warmup
     for _ in range(W):
         step()
@@ -437,6 +480,8 @@ def run_ours(args):
                "sample": f"{passes} pass(es) over {len(blocks)} whole blocks of {cfg.name} ({tot_n} masked "
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
+    redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
+
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
@@ -453,6 +498,7 @@ def run_ours(args):
             "e2e": e2e,
             "gpu_launches": launches_per_step * K,
             "clocks": clocks,
+            "redline": redline,
         }
         print(json.dumps(line), flush=True)
     if pg:

@@ -1,11 +1,12 @@
-"""GB300-native (sm_103a) commit step of a multi-block diffusion LM engine.
+"""GB300-native (sm_103a) commit step of a multi-block diffusion LM engine,
+and the Redline selection of the configuration to deploy.
 
-The work happens in libbdcommit.so (include/bdcommit.h); this package holds
-its CUDA sources (csrc/), the in-tree build step (build.py) and the ctypes
-binding (bdcommit.py).
+The work happens in libbdcommit.so (include/bdcommit.h, include/redline.h);
+this package holds its sources (csrc/), the in-tree build step (build.py) and
+the ctypes bindings (bdcommit.py, redline.py).
 """
 
-from . import bdcommit
+from . import bdcommit, redline
 from .bdcommit import (
     BD_BLOCK_ACTIVE,
     BD_BLOCK_FALLBACK_ELIGIBLE,
@@ -37,4 +38,5 @@ __all__ = [
     "bdcommit",
     "commit_step",
     "load_library",
+    "redline",
 ]
