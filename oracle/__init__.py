@@ -1,5 +1,5 @@
 """CPU oracles: float64 for the block-diffusion commit step, exact rationals
-for the Redline selection.
+for the Redline selection, plain loops for the commit sweep.
 
 TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and
 ``bench.py`` (its ``cpu_baseline`` leg and its ``--impl reference`` arm) may
@@ -14,10 +14,12 @@ is which blocks may take the top-1 fallback: that is an input (the caller's
 pinned by ``tests/test_redline_oracle.py`` (every p-value, valid mark and
 deployment of the paper's appendix grid tables, the calibration-size table,
 brute-force enumeration, closed-testing identities and an exact family-wise
-error).
+error). ``sweep_oracle`` is pinned by ``tests/test_sweep_oracle.py``
+(hand-derived cases, an independent whole-array formulation, and the
+maximal-exact-commit invariant over simulated decodes).
 """
 
-from . import redline_oracle
+from . import redline_oracle, sweep_oracle
 from .commit_oracle import (
     ACTIVE,
     FALLBACK_ELIGIBLE,
@@ -39,6 +41,7 @@ __all__ = [
     "decode_e4m3",
     "lm_head_logits",
     "redline_oracle",
+    "sweep_oracle",
     "row_confidence",
     "weights_f64",
 ]
