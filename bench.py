@@ -440,6 +440,35 @@ def run_ours(args):
                        "LM-head weights stay resident in HBM"
                        + ("; the K steps replayed as one CUDA graph" if args.graph else "")}
 
+    # ---- the commit sweep that follows the step in a decode loop (on a copy of
+    # the window: it updates the window in place)
+    sweep = None
+    if rank == 0:
+        tok_w = torch.full((P,), -1, dtype=torch.int32, device=dev)
+        pm_w, fl_w = wl.pos_masked.clone(), wl.block_flags.clone()
+        cache_w = torch.empty(P, dtype=torch.int32, device=dev)
+        ncom_w = torch.empty(cfg.n_seq, dtype=torch.int32, device=dev)
+
+        def sweep_once():
+            rc = B.bd_commit_sweep(tok_w, pm_w, fl_w, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
+                                   tokens, commit, len(cfg.tau) - 1, B.BD_SWEEP_ADMIT | B.BD_SWEEP_ELIGIBLE_OLDEST,
+                                   cache_w, ncom_w, None, stream=stream)
+            if rc != 0:
+                raise B.BdError(rc, "bd_commit_sweep")
+
+        for _ in range(10):
+            sweep_once()
+        n_sw = 500
+        (e0, e1), = timing_events(1, stream)
+        e0.record(stream)
+        for _ in range(n_sw):
+            sweep_once()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        sweep = {"us_per_launch": e0.elapsed_time(e1) * 1e3 / n_sw, "launches_timed": n_sw,
+                 "window_positions": P, "ctas": cfg.n_seq, "bound": "latency (one CTA per sequence)",
+                 "note": "bd_commit_sweep on the bench window after the timed steps, back to back on one stream"}
+
     # ---- roofline of the dominant kernel (LM head)
     hbm_gbs, tc_tflops, tc_sus, peak_src = peaks()
     flops, abytes = algorithmic(cfg, n_masked)
@@ -499,6 +528,7 @@ def run_ours(args):
             "gpu_launches": launches_per_step * K,
             "clocks": clocks,
             "redline": redline,
+            "sweep": sweep,
         }
         print(json.dumps(line), flush=True)
     if pg:

@@ -222,6 +222,64 @@ int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
                           int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                           void* stream);
 
+/* ------------------------------------------------------- commit sweep --
+ * The block-buffer update that follows the commit step in every decode step
+ * (engine appendix: slot states; maximal-exact-commit appendix, proof part 1).
+ *
+ * The window's own state, updated in place, device memory:
+ *   tokens      [P] int32 : the token each position holds (its content at
+ *                           masked positions is irrelevant)
+ *   pos_masked  [P] uint8 : 1 = still masked (the commit step's pos_masked)
+ *   block_flags [n_seq * n_slots] : BD_BLOCK_* bits; BD_BLOCK_ACTIVE set =
+ *                           an admitted block, clear = a placeholder slot
+ *   n_seq, n_slots, block_len, mask_token_id as in bd_mask_state, with
+ *   n_slots <= 64 and n_slots * block_len <= 4096 (block_len <= 64). */
+typedef struct {
+  int32_t n_seq;
+  int32_t n_slots;
+  int32_t block_len;
+  int32_t mask_token_id;
+  int32_t* tokens;
+  uint8_t* pos_masked;
+  uint8_t* block_flags;
+} bd_window;
+
+#define BD_SWEEP_ADMIT 1u           /* vacated slots return as admitted, all-masked blocks (else placeholders) */
+#define BD_SWEEP_ELIGIBLE_OLDEST 2u /* afterwards only the oldest active block of a sequence is fallback-eligible */
+
+/* One decode step's state update at the deployed threshold tau_index, on
+ * `stream` (a cudaStream_t, NULL = legacy default), after the commit step on
+ * the same stream (it may start while that step finishes and waits for it):
+ *   1. every position that is masked, in an active block and has bit
+ *      tau_index set in step_commit takes step_tokens[p] and is unmasked
+ *      (other bits are ignored);
+ *   2. the sweep visits each sequence's slots left to right and commits a
+ *      block when it is active, has no masked position (complete, hence
+ *      commit-ready under the default commit semantics) and its predecessor
+ *      was committed (or it is the first slot), so chains commit at once;
+ *   3. the c committed blocks leave the window for the cache: their tokens go
+ *      to out_cache_tokens [P] at blocks (s * n_slots + j), j < c (the rest of
+ *      that array is left untouched); out_n_committed[s] = c;
+ *   4. the remaining slots shift left by c with their tokens, masks and flags;
+ *      the c vacated slots at the end are mask-filled (tokens = mask_token_id,
+ *      or -1 when it is -1) and get flags 0, or BD_BLOCK_ACTIVE with
+ *      BD_SWEEP_ADMIT; with BD_SWEEP_ELIGIBLE_OLDEST the fallback bit is then
+ *      moved to the first active slot of each sequence.
+ * out_n_resolved [n_seq] (optional, may be NULL) receives the positions step 1
+ * resolved. step_tokens / step_commit are the commit step's out_tokens /
+ * out_commit. Afterwards no window block is active, complete and preceded
+ * only by committed blocks (the paper's zero exact-committable but
+ * uncommitted blocks).
+ * With n_seq == 0 the call does nothing and every array may be NULL.
+ * Errors (nothing queued): BD_ERR_NULL for a missing pointer; BD_ERR_SHAPE for
+ * n_seq < 0, n_slots outside 1..64, block_len outside 1..64, n_slots * block_len > 4096,
+ * or more than 2^24 positions; BD_ERR_ARG for tau_index outside 0..31 or
+ * unknown option bits; BD_ERR_DEVICE off sm_103; BD_ERR_CUDA if the launch
+ * fails. No allocation; calls on one window must be serialised. */
+int bd_commit_sweep(const bd_window* window, const int32_t* step_tokens, const uint32_t* step_commit,
+                    int32_t tau_index, uint32_t options, int32_t* out_cache_tokens, int32_t* out_n_committed,
+                    int32_t* out_n_resolved, void* stream);
+
 /* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
 int bd_version(void);
 

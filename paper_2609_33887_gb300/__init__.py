@@ -11,15 +11,19 @@ from .bdcommit import (
     BD_BLOCK_ACTIVE,
     BD_BLOCK_FALLBACK_ELIGIBLE,
     BD_OK,
+    BD_SWEEP_ADMIT,
+    BD_SWEEP_ELIGIBLE_OLDEST,
     BdError,
     bd_commit_step,
     bd_commit_step_ex,
+    bd_commit_sweep,
     bd_get_device_status,
     bd_shutdown,
     bd_status_string,
     bd_version,
     bd_workspace_size,
     commit_step,
+    commit_sweep,
     load_library,
 )
 
@@ -27,9 +31,12 @@ __all__ = [
     "BD_BLOCK_ACTIVE",
     "BD_BLOCK_FALLBACK_ELIGIBLE",
     "BD_OK",
+    "BD_SWEEP_ADMIT",
+    "BD_SWEEP_ELIGIBLE_OLDEST",
     "BdError",
     "bd_commit_step",
     "bd_commit_step_ex",
+    "bd_commit_sweep",
     "bd_get_device_status",
     "bd_shutdown",
     "bd_status_string",
@@ -37,6 +44,7 @@ __all__ = [
     "bd_workspace_size",
     "bdcommit",
     "commit_step",
+    "commit_sweep",
     "load_library",
     "redline",
 ]

@@ -39,6 +39,9 @@ BD_E4M3 = 2
 BD_BLOCK_ACTIVE = 1
 BD_BLOCK_FALLBACK_ELIGIBLE = 2
 
+BD_SWEEP_ADMIT = 1
+BD_SWEEP_ELIGIBLE_OLDEST = 2
+
 VARIANT_AUTO = 0
 VARIANT_SIMT = 1
 VARIANT_TC_ONE_CTA = 2
@@ -69,6 +72,11 @@ class bd_exec(ctypes.Structure):
                 ("variant", c_int32), ("flags", c_int32)]
 
 
+class bd_window(ctypes.Structure):
+    _fields_ = [("n_seq", c_int32), ("n_slots", c_int32), ("block_len", c_int32), ("mask_token_id", c_int32),
+                ("tokens", c_void_p), ("pos_masked", c_void_p), ("block_flags", c_void_p)]
+
+
 class BdError(RuntimeError):
     def __init__(self, status: int, where: str = "bd_commit_step"):
         self.status = status
@@ -97,6 +105,8 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
                                          POINTER(bd_tau_grid)]),
         "bd_commit_step_static": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
                                           POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, c_void_p]),
+        "bd_commit_sweep": (c_int, [POINTER(bd_window), c_void_p, c_void_p, c_int32, ctypes.c_uint32, c_void_p,
+                                    c_void_p, c_void_p, c_void_p]),
         "bd_get_device_status": (c_int, [c_void_p]),
         "bd_status_string": (ctypes.c_char_p, [c_int]),
         "bd_shutdown": (c_int, []),
@@ -255,3 +265,35 @@ def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_l
     if rc != BD_OK:
         raise BdError(rc)
     return tokens, conf, commit, cnt
+
+
+def bd_commit_sweep(tokens, pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id, step_tokens,
+                    step_commit, tau_index, options, out_cache_tokens, out_n_committed, out_n_resolved=None,
+                    stream=None) -> int:
+    """The block-buffer update after a commit step (include/bdcommit.h); returns the status.
+    tokens int32 [P], pos_masked uint8 [P], block_flags uint8 [n_seq * n_slots] are updated in place."""
+    win = bd_window(n_seq, n_slots, block_len, mask_token_id, _ptr(tokens), _ptr(pos_masked), _ptr(block_flags))
+    return load_library().bd_commit_sweep(ctypes.byref(win), _ptr(step_tokens), _ptr(step_commit), int(tau_index),
+                                          int(options), _ptr(out_cache_tokens), _ptr(out_n_committed),
+                                          _ptr(out_n_resolved), _stream_handle(stream))
+
+
+def commit_sweep(tokens, pos_masked, block_flags, n_seq, n_slots, block_len, step_tokens, step_commit, tau_index,
+                 *, mask_token_id=-1, options=0, stream=None):
+    """Allocate the outputs on the window's device, queue the sweep, raise on error.
+
+    Returns (cache int32 [P]: committed blocks of sequence s at blocks s * n_slots + j, j < n_committed[s];
+    n_committed int32 [n_seq]; n_resolved int32 [n_seq])."""
+    for t, dt in ((tokens, torch.int32), (pos_masked, torch.uint8), (block_flags, torch.uint8),
+                  (step_tokens, torch.int32), (step_commit, torch.int32)):
+        if t.dtype != dt or not t.is_contiguous():
+            raise ValueError("window and step tensors must be contiguous int32 / uint8 tensors")
+    dev = tokens.device
+    cache = torch.full((tokens.numel(),), -1, dtype=torch.int32, device=dev)
+    n_committed = torch.empty(n_seq, dtype=torch.int32, device=dev)
+    n_resolved = torch.empty(n_seq, dtype=torch.int32, device=dev)
+    rc = bd_commit_sweep(tokens, pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id, step_tokens,
+                         step_commit, tau_index, options, cache, n_committed, n_resolved, stream=stream)
+    if rc != BD_OK:
+        raise BdError(rc, "bd_commit_sweep")
+    return cache, n_committed, n_resolved

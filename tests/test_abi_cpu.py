@@ -38,7 +38,8 @@ def declared_functions():
 
 def test_header_declares_the_abi():
     assert declared_functions() == sorted([
-        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_get_device_status", "bd_shutdown",
+        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status",
+        "bd_shutdown",
         "bd_status_string", "bd_version", "bd_workspace_size",
         "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
         "bd_redline_select", "bd_redline_sweep", "bd_redline_critical_count", "bd_redline_power",
@@ -136,3 +137,33 @@ def test_null_structs_rejected(lib):
 def test_empty_window_is_a_no_op(lib):
     # zero sequences: nothing to compute, nothing queued, no CUDA call
     assert _call(lib, n_seq=0, hptr=None, wptr=None, outs=(None, None, None)) == B.BD_OK
+
+
+# ------------------------------------------------ commit sweep argument checks --
+def _sweep(lib, n_seq=2, n_slots=4, L=32, tau_index=0, options=0, ptrs=(FAKE,) * 3, step=(FAKE, FAKE),
+           cache=FAKE, n_committed=FAKE):
+    win = B.bd_window(n_seq, n_slots, L, -1, *ptrs)
+    return lib.bd_commit_sweep(ctypes.byref(win), step[0], step[1], tau_index, options, cache, n_committed, None, 0)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(L=0), B.BD_ERR_SHAPE),
+    (dict(L=65), B.BD_ERR_SHAPE),
+    (dict(n_slots=0), B.BD_ERR_SHAPE),
+    (dict(n_slots=65, L=1), B.BD_ERR_SHAPE),
+    (dict(n_seq=-1), B.BD_ERR_SHAPE),
+    (dict(tau_index=32), B.BD_ERR_ARG),
+    (dict(tau_index=-1), B.BD_ERR_ARG),
+    (dict(options=4), B.BD_ERR_ARG),
+    (dict(ptrs=(None, FAKE, FAKE)), B.BD_ERR_NULL),
+    (dict(step=(FAKE, None)), B.BD_ERR_NULL),
+    (dict(cache=None), B.BD_ERR_NULL),
+    (dict(n_committed=None), B.BD_ERR_NULL),
+])
+def test_sweep_argument_checks(lib, kw, code):
+    assert _sweep(lib, **kw) == code
+
+
+def test_sweep_empty_window_is_a_no_op(lib):
+    assert _sweep(lib, n_seq=0, ptrs=(None, None, None), step=(None, None), cache=None, n_committed=None) == B.BD_OK
+    assert lib.bd_commit_sweep(None, FAKE, FAKE, 0, 0, FAKE, FAKE, None, 0) == B.BD_ERR_NULL
