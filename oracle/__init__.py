@@ -1,5 +1,6 @@
-"""CPU oracles: float64 for the block-diffusion commit step, exact rationals
-for the Redline selection, plain loops for the commit sweep.
+"""CPU oracles: float64 for the block-diffusion commit step and for
+speculative verification, exact rationals for the Redline selection, plain
+loops for the commit sweep.
 
 TEST INFRASTRUCTURE. Only ``tests/``, ``__graft_entry__.smoke()`` and
 ``bench.py`` (its ``cpu_baseline`` leg and its ``--impl reference`` arm) may
@@ -16,10 +17,13 @@ deployment of the paper's appendix grid tables, the calibration-size table,
 brute-force enumeration, closed-testing identities and an exact family-wise
 error). ``sweep_oracle`` is pinned by ``tests/test_sweep_oracle.py``
 (hand-derived cases, an independent whole-array formulation, and the
-maximal-exact-commit invariant over simulated decodes).
+maximal-exact-commit invariant over simulated decodes). ``verify_oracle`` is
+pinned by ``tests/test_verify_oracle.py`` (closed forms, a 50-digit brute
+force, a hand-derived case for both branches of the rule, the nesting in eps,
+and the paper's lossless tokens per forward from its draft agreement).
 """
 
-from . import redline_oracle, sweep_oracle
+from . import redline_oracle, sweep_oracle, verify_oracle
 from .commit_oracle import (
     ACTIVE,
     FALLBACK_ELIGIBLE,
@@ -42,6 +46,7 @@ __all__ = [
     "lm_head_logits",
     "redline_oracle",
     "sweep_oracle",
+    "verify_oracle",
     "row_confidence",
     "weights_f64",
 ]
