@@ -222,6 +222,63 @@ int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
                           int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                           void* stream);
 
+/* ---------------------------------------------- speculative verification --
+ * The same LM head and fused softmax serve the verification step of
+ * speculative decoding with the lossy typical-acceptance rule the paper tests
+ * (typical-acceptance appendix): a draft token x is accepted when the target's
+ * probability of it exceeds min(eps, sqrt(eps) * exp(-H)), H the entropy of the
+ * target's next-token distribution; the lossless reference accepts x only when
+ * it is the target's argmax (lossless-reference appendix). A request accepts
+ * the longest prefix of its drafts that pass.
+ *
+ * Draft tokens of a verification batch, device memory:
+ *   n_req    requests (>= 0)
+ *   n_draft  draft tokens per request, 1..32
+ *   draft    [n_req * n_draft] int32: draft token i of request q at
+ *            q * n_draft + i; an entry outside [0, vocab) has probability 0
+ * The hidden states then hold n_req * (n_draft + 1) rows: row
+ * q * (n_draft + 1) + i is the target state whose next-token distribution
+ * verifies draft token i (i < n_draft); the last row of a request gives the
+ * token the target adds after the accepted prefix when every draft passes. */
+typedef struct {
+  int32_t n_req;
+  int32_t n_draft;
+  const int32_t* draft;
+} bd_draft;
+
+/* Typical-acceptance settings: HOST array eps[0..E-1], 1 <= E <= 31, each in
+ * (0, 1] (a lower eps accepts more). Copied at call time. */
+typedef struct {
+  const float* eps;
+  int32_t E;
+} bd_eps_grid;
+
+#define BD_ACCEPT_LOSSLESS_BIT 31 /* bit of out_accept set when the draft is the target's argmax */
+
+/* One verification step, asynchronous on exec->stream (exec may be NULL).
+ * Outputs, device arrays, all fully written (R = n_req * (n_draft + 1)):
+ *   out_tokens   [R] int32  : the target's argmax (lowest index on ties)
+ *   out_p_draft  [R] float  : target probability of the row's draft token (0 on
+ *                             the last row of a request)
+ *   out_entropy  [R] float  : entropy of the target distribution, in nats
+ *   out_accept   [R] uint32 : bit k = accepted at eps[k]; bit 31 = lossless
+ *                             (0 on the last row of a request)
+ *   out_accepted [n_req * (E + 1)] int32 : accepted prefix length of request q
+ *                             at eps[k] at q * (E + 1) + k, the lossless rule at
+ *                             column E; accepted tokens for the target forward
+ *                             are that length + 1
+ * Same hidden / weight dtypes, alignment rules, variants and workspace rules
+ * as bd_commit_step_ex (size from bd_verify_workspace_size); exec->out_counts
+ * must be NULL. Errors: as bd_commit_step_ex, with BD_ERR_TAU for a bad eps
+ * grid and BD_ERR_SHAPE for n_draft outside 1..32 or hidden->rows != R. */
+int bd_verify_step(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft,
+                   const bd_eps_grid* eps, int32_t* out_tokens, float* out_p_draft, float* out_entropy,
+                   uint32_t* out_accept, int32_t* out_accepted, const bd_exec* exec);
+
+/* Bytes of device workspace bd_verify_step needs for these arguments (0 if invalid). */
+size_t bd_verify_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft,
+                                const bd_eps_grid* eps);
+
 /* ------------------------------------------------------- commit sweep --
  * The block-buffer update that follows the commit step in every decode step
  * (engine appendix: slot states; maximal-exact-commit appendix, proof part 1).

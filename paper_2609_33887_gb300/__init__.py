@@ -20,11 +20,14 @@ from .bdcommit import (
     bd_get_device_status,
     bd_shutdown,
     bd_status_string,
+    bd_verify_step,
+    bd_verify_workspace_size,
     bd_version,
     bd_workspace_size,
     commit_step,
     commit_sweep,
     load_library,
+    verify_step,
 )
 
 __all__ = [
@@ -40,6 +43,8 @@ __all__ = [
     "bd_get_device_status",
     "bd_shutdown",
     "bd_status_string",
+    "bd_verify_step",
+    "bd_verify_workspace_size",
     "bd_version",
     "bd_workspace_size",
     "bdcommit",
@@ -47,4 +52,5 @@ __all__ = [
     "commit_sweep",
     "load_library",
     "redline",
+    "verify_step",
 ]

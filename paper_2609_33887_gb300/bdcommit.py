@@ -72,6 +72,17 @@ class bd_exec(ctypes.Structure):
                 ("variant", c_int32), ("flags", c_int32)]
 
 
+class bd_draft(ctypes.Structure):
+    _fields_ = [("n_req", c_int32), ("n_draft", c_int32), ("draft", c_void_p)]
+
+
+class bd_eps_grid(ctypes.Structure):
+    _fields_ = [("eps", POINTER(c_float)), ("E", c_int32)]
+
+
+BD_ACCEPT_LOSSLESS_BIT = 31
+
+
 class bd_window(ctypes.Structure):
     _fields_ = [("n_seq", c_int32), ("n_slots", c_int32), ("block_len", c_int32), ("mask_token_id", c_int32),
                 ("tokens", c_void_p), ("pos_masked", c_void_p), ("block_flags", c_void_p)]
@@ -105,6 +116,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
                                          POINTER(bd_tau_grid)]),
         "bd_commit_step_static": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
                                           POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, c_void_p]),
+        "bd_verify_step": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_draft), POINTER(bd_eps_grid),
+                                   c_void_p, c_void_p, c_void_p, c_void_p, c_void_p, POINTER(bd_exec)]),
+        "bd_verify_workspace_size": (c_size_t, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_draft),
+                                                POINTER(bd_eps_grid)]),
         "bd_commit_sweep": (c_int, [POINTER(bd_window), c_void_p, c_void_p, c_int32, ctypes.c_uint32, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),
         "bd_get_device_status": (c_int, [c_void_p]),
@@ -297,3 +312,57 @@ def commit_sweep(tokens, pos_masked, block_flags, n_seq, n_slots, block_len, ste
     if rc != BD_OK:
         raise BdError(rc, "bd_commit_sweep")
     return cache, n_committed, n_resolved
+
+
+def make_eps_grid(eps: Sequence[float]):
+    arr = (c_float * max(1, len(eps)))(*[float(e) for e in eps])
+    return bd_eps_grid(ctypes.cast(arr, POINTER(c_float)), len(eps)), arr
+
+
+def bd_verify_workspace_size(hidden, weight, weight_scale, draft, n_req, n_draft, eps) -> int:
+    h, w = make_hidden(hidden), make_weight(weight, weight_scale)
+    dr = bd_draft(n_req, n_draft, _ptr(draft))
+    eg, _keep = make_eps_grid(eps)
+    return int(load_library().bd_verify_workspace_size(ctypes.byref(h), ctypes.byref(w), ctypes.byref(dr),
+                                                       ctypes.byref(eg)))
+
+
+def bd_verify_step(hidden, weight, weight_scale, draft, n_req, n_draft, eps, out_tokens, out_p_draft, out_entropy,
+                   out_accept, out_accepted, stream=None, workspace=None, lmhead_events=None, variant=0) -> int:
+    """Speculative-decoding verification (include/bdcommit.h); returns the status."""
+    h, w = make_hidden(hidden), make_weight(weight, weight_scale)
+    dr = bd_draft(n_req, n_draft, _ptr(draft))
+    eg, _keep = make_eps_grid(eps)
+    ex = bd_exec()
+    ex.stream = _stream_handle(stream)
+    if workspace is not None:
+        ex.workspace = workspace.data_ptr()
+        ex.workspace_bytes = workspace.numel() * workspace.element_size()
+    if lmhead_events is not None:
+        ex.lmhead_event_begin = lmhead_events[0].cuda_event
+        ex.lmhead_event_end = lmhead_events[1].cuda_event
+    ex.variant = variant
+    return load_library().bd_verify_step(ctypes.byref(h), ctypes.byref(w), ctypes.byref(dr), ctypes.byref(eg),
+                                         _ptr(out_tokens), _ptr(out_p_draft), _ptr(out_entropy), _ptr(out_accept),
+                                         _ptr(out_accepted), ctypes.byref(ex))
+
+
+def verify_step(hidden, weight, draft, n_req, n_draft, eps, *, weight_scale=None, stream=None, workspace=None,
+                variant=VARIANT_AUTO, lmhead_events=None):
+    """Allocate the outputs on the hidden states' device, queue the verification, raise on error.
+
+    Returns a dict of tensors: tokens int32 [R], p_draft float32 [R], entropy float32 [R],
+    accept int32 [R] (uint32 bit masks), accepted int32 [n_req, E + 1]."""
+    R = n_req * (n_draft + 1)
+    dev = hidden.device
+    out = {"tokens": torch.empty(R, dtype=torch.int32, device=dev),
+           "p_draft": torch.empty(R, dtype=torch.float32, device=dev),
+           "entropy": torch.empty(R, dtype=torch.float32, device=dev),
+           "accept": torch.empty(R, dtype=torch.int32, device=dev),
+           "accepted": torch.empty((n_req, len(eps) + 1), dtype=torch.int32, device=dev)}
+    rc = bd_verify_step(hidden, weight, weight_scale, draft, n_req, n_draft, eps, out["tokens"], out["p_draft"],
+                        out["entropy"], out["accept"], out["accepted"], stream=stream, workspace=workspace,
+                        lmhead_events=lmhead_events, variant=variant)
+    if rc != BD_OK:
+        raise BdError(rc, "bd_verify_step")
+    return out

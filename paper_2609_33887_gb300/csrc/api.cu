@@ -555,3 +555,267 @@ extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* w
   return run_step(c, plan, lay, ws, status, sctx->sm_count, hidden, weight, mask_state, tau_grid, out_tokens,
                   out_conf, out_commit, nullptr, nullptr, nullptr, st);
 }
+
+// ---------------------------------------------------------------------------
+// bd_verify_step: speculative-decoding verification on the same LM head
+// (typical-acceptance and lossless-reference appendices).
+// ---------------------------------------------------------------------------
+namespace {
+
+struct VerifyCall {
+  Call c;  // P = rows, T = E
+  int n_req, n_draft;
+};
+
+int check_verify(const bd_hidden* h, const bd_weight* w, const bd_draft* dr, const bd_eps_grid* eg, int variant,
+                 VerifyCall* vc) {
+  if (!h || !w || !dr || !eg) return BD_ERR_NULL;
+  if (!eg->eps || eg->E < 1 || eg->E > 31) return BD_ERR_TAU;
+  for (int k = 0; k < eg->E; ++k)
+    if (!(eg->eps[k] > 0.f && eg->eps[k] <= 1.f)) return BD_ERR_TAU;  // NaN fails too
+  if (variant < 0 || variant > 3) return BD_ERR_ARG;
+  if (dr->n_req < 0 || dr->n_draft < 1 || dr->n_draft > 32) return BD_ERR_SHAPE;
+  const int64_t R = int64_t(dr->n_req) * (dr->n_draft + 1);
+  if (R > MAX_POSITIONS || h->rows != R) return BD_ERR_SHAPE;
+  if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
+  if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
+  if (h->ld < h->cols || w->ld < w->dim) return BD_ERR_SHAPE;
+  const int hdt = h->dtype, wdt = w->dtype;
+  const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
+  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3);
+  if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
+  const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
+  if (tc && !combo_bf16) return BD_ERR_DTYPE;
+  if (R > 0) {
+    if (!h->data || !w->data || !dr->draft) return BD_ERR_NULL;
+    if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
+    if (!aligned(dr->draft, 4)) return BD_ERR_ALIGN;
+  }
+  if (tc) {
+    if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
+    if (!aligned(w->data, 16) || (w->ld * esize(wdt)) % 16 != 0) return BD_ERR_ALIGN;
+  } else {
+    if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
+  }
+  if (w->scale && wdt == BD_E4M3 && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  Call& c = vc->c;
+  c = Call{};
+  c.P = R;
+  c.d = w->dim;
+  c.V = w->vocab;
+  c.n_seq = dr->n_req;
+  c.n_slots = 1;
+  c.L = dr->n_draft + 1;
+  c.n_blocks = dr->n_req;
+  c.mask_id = -1;  // the target's full distribution
+  c.T = eg->E;
+  c.hdt = hdt;
+  c.wdt = wdt;
+  c.tc = tc;
+  c.pair = tc && (variant == 3 || (variant == 0 && R <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
+  c.ldh = h->ld;
+  c.ldw = w->ld;
+  c.ldc = h->ld;  // the rows are read in place
+  c.ldq = round_up(c.d, 8);
+  vc->n_req = dr->n_req;
+  vc->n_draft = dr->n_draft;
+  return BD_OK;
+}
+
+struct VerifyLayout {
+  size_t hdr, idx, draft_row, pm, ps, pa, pt, px, wq, total;
+};
+
+VerifyLayout make_verify_layout(const Call& c, const BandPlan& p) {
+  VerifyLayout l{};
+  size_t off = 0;
+  auto take = [&off](size_t bytes, size_t align) {
+    off = (off + align - 1) / align * align;
+    size_t o = off;
+    off += bytes;
+    return o;
+  };
+  const size_t R = static_cast<size_t>(c.P);
+  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
+  l.hdr = take(256, 256);
+  l.idx = take(4 * R, 256);
+  l.draft_row = take(4 * R, 256);
+  l.pm = take(4 * slots * R, 256);
+  l.ps = take(4 * slots * R, 256);
+  l.pa = take(4 * slots * R, 256);
+  l.pt = take(4 * slots * R, 256);
+  l.px = take(4 * slots * R, 256);
+  l.wq = (c.tc && c.wdt == BD_E4M3) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
+  l.total = (off + 255) / 256 * 256;
+  return l;
+}
+
+int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& lay, uint8_t* ws, uint32_t* status,
+               int sm_count, const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft,
+               const bd_eps_grid* eps, int32_t* out_tokens, float* out_p_draft, float* out_entropy,
+               uint32_t* out_accept, int32_t* out_accepted, void* ev_begin, void* ev_end, cudaStream_t st) {
+  const Call& c = vc.c;
+  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
+  int* idx = reinterpret_cast<int*>(ws + lay.idx);
+  int* draft_row = reinterpret_cast<int*>(ws + lay.draft_row);
+  float* pm = reinterpret_cast<float*>(ws + lay.pm);
+  float* ps = reinterpret_cast<float*>(ws + lay.ps);
+  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+  float* pt = reinterpret_cast<float*>(ws + lay.pt);
+  float* px = reinterpret_cast<float*>(ws + lay.px);
+  const int R = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+
+  int rc = cuda_status(bd::launch_prep_verify(draft->draft, vc.n_req, vc.n_draft, idx, draft_row, n_rows, st));
+  if (rc != BD_OK) return rc;
+
+  CUtensorMap tmA, tmB;
+  bd::PairTokenMaps tmTok;
+  if (c.tc) {
+    const void* wsrc = weight->data;
+    int64_t wld = c.ldw;
+    if (c.wdt == BD_E4M3) {
+      void* wq = ws + lay.wq;
+      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
+                                               sm_count, st));
+      if (rc != BD_OK) return rc;
+      wsrc = wq;
+      wld = c.ldq;
+    }
+    if (c.pair) {
+      for (int i = 0; i < 8; ++i)
+        if (!encode_bf16_2d(&tmTok.m[i], hidden->data, c.d, c.P, c.ldh, 64, 16 * (i + 1))) return BD_ERR_CUDA;
+      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
+    } else {
+      if (!encode_bf16_2d(&tmA, hidden->data, c.d, c.P, c.ldh, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
+      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
+    }
+  }
+
+  if (ev_begin && record_event(ev_begin, st) != cudaSuccess) return BD_ERR_CUDA;
+  if (c.tc) {
+    bd::TcArgs a;
+    a.n_rows = n_rows;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.V = V;
+    a.d = d;
+    a.P = R;
+    a.mask_id = -1;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    a.status = status;
+    a.draft_row = draft_row;
+    a.part_t = pt;
+    a.part_x = px;
+    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, a, st))
+                : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
+  } else {
+    bd::SimtArgs a;
+    a.hidden = hidden->data;
+    a.ldh = c.ldh;
+    a.hdtype = c.hdt;
+    a.w = weight->data;
+    a.ldw = c.ldw;
+    a.wdtype = c.wdt;
+    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.idx = idx;
+    a.n_rows = n_rows;
+    a.V = V;
+    a.d = d;
+    a.P = R;
+    a.mask_id = -1;
+    a.plan = plan;
+    a.part_m = pm;
+    a.part_s = ps;
+    a.part_a = pa;
+    a.draft_row = draft_row;
+    a.part_t = pt;
+    a.part_x = px;
+    rc = cuda_status(bd::launch_lmhead_simt(a, st));
+  }
+  if (rc != BD_OK) return rc;
+  if (ev_end && record_event(ev_end, st) != cudaSuccess) return BD_ERR_CUDA;
+
+  bd::VerifyArgs va;
+  va.draft_row = draft_row;
+  va.n_rows = n_rows;
+  va.plan = plan;
+  va.P = R;
+  va.part_m = pm;
+  va.part_s = ps;
+  va.part_a = pa;
+  va.part_t = pt;
+  va.part_x = px;
+  va.n_req = vc.n_req;
+  va.n_draft = vc.n_draft;
+  va.E = eps->E;
+  std::memset(va.eps, 0, sizeof(va.eps));
+  std::memset(va.sqrt_eps, 0, sizeof(va.sqrt_eps));
+  for (int k = 0; k < eps->E; ++k) {
+    va.eps[k] = eps->eps[k];
+    va.sqrt_eps[k] = static_cast<float>(std::sqrt(static_cast<double>(eps->eps[k])));
+  }
+  va.out_tokens = out_tokens;
+  va.out_p_draft = out_p_draft;
+  va.out_entropy = out_entropy;
+  va.out_accept = out_accept;
+  va.out_accepted = out_accepted;
+  return cuda_status(bd::launch_merge_verify(va, st));
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t bd_verify_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft,
+                                const bd_eps_grid* eps) {
+  VerifyCall vc;
+  if (check_verify(hidden, weight, draft, eps, 0, &vc) != BD_OK) return 0;
+  DevCtx* ctx = nullptr;
+  if (device_ctx(&ctx) != BD_OK) return 0;
+  return make_verify_layout(vc.c, make_plan(vc.c, ctx->sm_count, ctx->pairs)).total;
+}
+
+int bd_verify_step(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft, const bd_eps_grid* eps,
+                   int32_t* out_tokens, float* out_p_draft, float* out_entropy, uint32_t* out_accept,
+                   int32_t* out_accepted, const bd_exec* exec) {
+  const int variant = exec ? exec->variant : 0;
+  if (exec && (exec->flags != 0 || exec->out_counts != nullptr)) return BD_ERR_ARG;
+  VerifyCall vc;
+  int rc = check_verify(hidden, weight, draft, eps, variant, &vc);
+  if (rc != BD_OK) return rc;
+  if (vc.c.P == 0) return BD_OK;
+  if (!out_tokens || !out_p_draft || !out_entropy || !out_accept || !out_accepted) return BD_ERR_NULL;
+  if (!aligned(out_tokens, 4) || !aligned(out_p_draft, 4) || !aligned(out_entropy, 4) || !aligned(out_accept, 4) ||
+      !aligned(out_accepted, 4))
+    return BD_ERR_ALIGN;
+  if (exec && exec->workspace && !aligned(exec->workspace, 256)) return BD_ERR_ALIGN;
+
+  DevCtx* ctx = nullptr;
+  rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  const BandPlan plan = make_plan(vc.c, ctx->sm_count, ctx->pairs);
+  const VerifyLayout lay = make_verify_layout(vc.c, plan);
+  uint8_t* ws = nullptr;
+  if (exec && exec->workspace) {
+    if (exec->workspace_bytes < lay.total) return BD_ERR_WORKSPACE;
+    ws = static_cast<uint8_t*>(exec->workspace);
+  } else {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (ctx->ws_bytes < lay.total) {
+      if (ctx->ws) cudaFree(ctx->ws);  // synchronises the device: no call can still use it
+      ctx->ws = nullptr;
+      ctx->ws_bytes = 0;
+      if (cudaMalloc(&ctx->ws, lay.total) != cudaSuccess) return BD_ERR_CUDA;
+      ctx->ws_bytes = lay.total;
+    }
+    ws = static_cast<uint8_t*>(ctx->ws);
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(exec ? exec->stream : nullptr);
+  return run_verify(vc, plan, lay, ws, ctx->status, ctx->sm_count, hidden, weight, draft, eps, out_tokens,
+                    out_p_draft, out_entropy, out_accept, out_accepted, exec ? exec->lmhead_event_begin : nullptr,
+                    exec ? exec->lmhead_event_end : nullptr, st);
+}
+
+}  // extern "C"

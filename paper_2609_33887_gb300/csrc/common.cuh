@@ -143,6 +143,39 @@ __device__ __forceinline__ void softmax_combine(float& m, float& s, int& a, floa
   }
 }
 
+// The same combine carrying t = sum exp(l - m) * (l - m) * log2(e), the first
+// moment of the shifted logits in log2 units (the entropy accumulator of the
+// verification path: H = ln s - t / (s * log2(e))). Rescaling a state from max
+// m to M > m multiplies both sums by f = 2^((m - M) log2 e) and shifts every
+// (l - m) by (m - M): t -> f * (t + (m - M) log2(e) * s).
+__device__ __forceinline__ void softmax_combine_t(float& m, float& s, int& a, float& t, float m2, float s2, int a2,
+                                                  float t2) {
+  if (m2 > m) {
+    if (m == -INFINITY) {
+      t = t2;
+      s = s2;
+    } else {
+      const float dm = (m - m2) * LOG2E;
+      const float f = ex2_approx(dm);
+      t = t2 + f * fmaf(dm, s, t);
+      s = s2 + f * s;
+    }
+    m = m2;
+    a = a2;
+  } else if (m2 == m) {
+    if (m2 != -INFINITY) {
+      s += s2;
+      t += t2;
+    }
+    a = a2 < a ? a2 : a;
+  } else if (m2 != -INFINITY) {
+    const float dm = (m2 - m) * LOG2E;
+    const float f = ex2_approx(dm);
+    t += f * fmaf(dm, s2, t2);
+    s += f * s2;
+  }
+}
+
 // -------------------------------------------------------------------------
 // PTX wrappers
 // -------------------------------------------------------------------------

@@ -25,6 +25,11 @@
 // CTA layout (192 threads): warp 0 TMA producer, warp 1 TMEM allocation (both
 // CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue. Every wait is
 // bounded (see common.cuh).
+//
+// The verification instantiation (VERIFY = true, speculative decoding) also
+// carries, per token, the entropy accumulator sum exp(l - m) (l - m) log2(e)
+// and the logit of the token's draft entry (typical-acceptance appendix); its
+// larger combine buffers cost shared memory, so it may run one stage fewer.
 #include <atomic>
 
 #include "kernels.h"
@@ -55,9 +60,11 @@ struct PairCtl {
 
 // One buffer per epilogue warp: the 32 x 33 transpose during the tiles of a
 // unit; after the warp's last tile, the same warp's running states (max, sum,
-// argmax for up to 256 tokens) for the cross-warp combine. A warp only ever
-// writes its own buffer before the rendezvous, so no warp can overwrite a
-// buffer another warp is still transposing in.
+// argmax for up to 256 tokens; with VERIFY also the entropy accumulator and
+// the draft logit) for the cross-warp combine. A warp only ever writes its own
+// buffer before the rendezvous, so no warp can overwrite a buffer another warp
+// is still transposing in.
+template <bool VERIFY>
 struct PairWarpBuf {
   union {
     float tr[32 * TR];
@@ -65,17 +72,23 @@ struct PairWarpBuf {
       float m[256];
       float s[256];
       int a[256];
+      float t[VERIFY ? 256 : 1];
+      float x[VERIFY ? 256 : 1];
     } st;
   };
 };
 
+template <bool VERIFY>
 struct PairTail {
-  PairWarpBuf w[EPI_WARPS];
+  PairWarpBuf<VERIFY> w[EPI_WARPS];
   PairCtl ctl;
 };
 
 constexpr size_t SMEM_BYTES = 232448;  // the whole opt-in shared memory of an SM
-constexpr size_t STAGE_AREA = SMEM_BYTES - 1024 - sizeof(PairTail);
+template <bool VERIFY>
+__host__ __device__ constexpr size_t stage_area() {
+  return SMEM_BYTES - 1024 - sizeof(PairTail<VERIFY>);
+}
 
 // Stage layout for a token group of NT rows (NT/2 in each CTA):
 //   [A block 0 | A block 1 | B block 0 | B block 1], A = 128 head rows,
@@ -83,19 +96,23 @@ constexpr size_t STAGE_AREA = SMEM_BYTES - 1024 - sizeof(PairTail);
 __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
   return 2 * A_BLOCK + 2 * static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES;
 }
+template <bool VERIFY>
 __host__ __device__ constexpr int stage_count(int nt) {
-  return static_cast<int>(STAGE_AREA / stage_bytes(nt)) < MAX_STAGES ? static_cast<int>(STAGE_AREA / stage_bytes(nt))
-                                                                     : MAX_STAGES;
+  return static_cast<int>(stage_area<VERIFY>() / stage_bytes(nt)) < MAX_STAGES
+             ? static_cast<int>(stage_area<VERIFY>() / stage_bytes(nt))
+             : MAX_STAGES;
 }
-static_assert(stage_count(256) >= 3, "three stages at NT = 256");
+static_assert(stage_count<false>(256) >= 3 && stage_count<true>(256) >= 3, "three stages at NT = 256");
+static_assert(stage_count<false>(160) == 4, "four stages at NT = 160 on the commit path");
 
 }  // namespace
 
+template <bool VERIFY>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW, TcArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  PairTail* tail = reinterpret_cast<PairTail*>(smem + STAGE_AREA);
+  PairTail<VERIFY>* tail = reinterpret_cast<PairTail<VERIFY>*>(smem + stage_area<VERIFY>());
   PairCtl* ctl = &tail->ctl;
   const uint32_t smem_base = smem_u32(smem);
 
@@ -137,7 +154,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   const int nch = NT / 32;
   const uint32_t SB = stage_bytes(NT);
   const uint32_t B_BLOCK = static_cast<uint32_t>(half) * ATOM_ROWS_BYTES;
-  const int STAGES = stage_count(NT);
+  const int STAGES = stage_count<VERIFY>(NT);
   const uint32_t tx_total = 2u * SB;  // both CTAs' bytes land on the even CTA's barrier
   const CUtensorMap* tm_tok = &tmH.m[half / 16 - 1];  // box of exactly `half` rows
 
@@ -249,11 +266,20 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     while (ok && it.next_unit()) {
       float m[MAX_CHUNKS], s[MAX_CHUNKS];
       int arg[MAX_CHUNKS];
+      float t[MAX_CHUNKS], lx[MAX_CHUNKS];  // VERIFY only
+      int xd[MAX_CHUNKS];                   // VERIFY only: draft entry of this thread's token
 #pragma unroll
       for (int c = 0; c < MAX_CHUNKS; ++c) {
         m[c] = -INFINITY;
         s[c] = 0.f;
         arg[c] = 0x7fffffff;
+        t[c] = 0.f;
+        lx[c] = -INFINITY;
+        xd[c] = -1;
+        if constexpr (VERIFY) {
+          const int row = it.m_tile * NT + c * 32 + lane;
+          if (c < nch && row < n_rows) xd[c] = a.draft_row[row];
+        }
       }
       for (int vt = it.vt; vt < it.vt_end; ++vt) {
         if (!mbar_wait_warp(smem_u32(&ctl->tfull[acc]), acc_phase, abort_flag, a.status)) {
@@ -276,6 +302,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             float x[32];
 #pragma unroll
             for (int r = 0; r < 32; ++r) x[r] = tr[r * TR + lane];
+            if constexpr (VERIFY) {
+              const int rel = xd[c] - vrow0;
+              if (rel >= 0 && rel < 32) lx[c] = tr[rel * TR + lane];
+            }
             __syncwarp();
             // this thread: token column c*32 + lane, vocabulary rows vrow0 + r
             float cm = x[0];
@@ -287,18 +317,46 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               for (int r = 31; r >= 0; --r)
                 if (x[r] == cm) rr = r;
               arg[c] = vrow0 + rr;
-              s[c] = (m[c] == -INFINITY) ? 0.f : s[c] * ex2_approx((m[c] - cm) * LOG2E);
+              if constexpr (VERIFY) {
+                if (m[c] == -INFINITY) {
+                  s[c] = 0.f;
+                  t[c] = 0.f;
+                } else {
+                  const float dm = (m[c] - cm) * LOG2E;
+                  const float f = ex2_approx(dm);
+                  t[c] = f * fmaf(dm, s[c], t[c]);
+                  s[c] *= f;
+                }
+              } else {
+                s[c] = (m[c] == -INFINITY) ? 0.f : s[c] * ex2_approx((m[c] - cm) * LOG2E);
+              }
               m[c] = cm;
             }
             if (m[c] != -INFINITY) {
               const float mc = m[c] * LOG2E;
-              float s0 = 0.f, s1 = 0.f;
+              if constexpr (VERIFY) {
+                // -inf logits give u = -inf, e = 0; clamping u keeps e * u at 0
+                float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
-              for (int r = 0; r < 32; r += 2) {
-                s0 += ex2_approx(fmaf(x[r], LOG2E, -mc));
-                s1 += ex2_approx(fmaf(x[r + 1], LOG2E, -mc));
+                for (int r = 0; r < 32; r += 2) {
+                  const float u0 = fmaf(x[r], LOG2E, -mc), u1 = fmaf(x[r + 1], LOG2E, -mc);
+                  const float e0 = ex2_approx(u0), e1 = ex2_approx(u1);
+                  s0 += e0;
+                  s1 += e1;
+                  t0 = fmaf(e0, fmaxf(u0, -256.f), t0);
+                  t1 = fmaf(e1, fmaxf(u1, -256.f), t1);
+                }
+                s[c] += s0 + s1;
+                t[c] += t0 + t1;
+              } else {
+                float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+                for (int r = 0; r < 32; r += 2) {
+                  s0 += ex2_approx(fmaf(x[r], LOG2E, -mc));
+                  s1 += ex2_approx(fmaf(x[r + 1], LOG2E, -mc));
+                }
+                s[c] += s0 + s1;
               }
-              s[c] += s0 + s1;
             }
           }
         }
@@ -323,6 +381,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           tail->w[ew].st.m[c * 32 + lane] = m[c];
           tail->w[ew].st.s[c * 32 + lane] = s[c];
           tail->w[ew].st.a[c * 32 + lane] = arg[c];
+          if constexpr (VERIFY) {
+            tail->w[ew].st.t[c * 32 + lane] = t[c];
+            tail->w[ew].st.x[c * 32 + lane] = lx[c];
+          }
         }
       }
       mbar_arrive(epi_sync);
@@ -331,15 +393,31 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       for (int j = ew * 32 + lane; j < NT; j += EPI_WARPS * 32) {
         float M = tail->w[0].st.m[j], S = tail->w[0].st.s[j];
         int A = tail->w[0].st.a[j];
+        float T = 0.f, LX = -INFINITY;
+        if constexpr (VERIFY) {
+          T = tail->w[0].st.t[j];
+          LX = tail->w[0].st.x[j];
+        }
 #pragma unroll
-        for (int w = 1; w < EPI_WARPS; ++w)
-          softmax_combine(M, S, A, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j]);
+        for (int w = 1; w < EPI_WARPS; ++w) {
+          if constexpr (VERIFY) {
+            softmax_combine_t(M, S, A, T, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j],
+                              tail->w[w].st.t[j]);
+            LX = fmaxf(LX, tail->w[w].st.x[j]);
+          } else {
+            softmax_combine(M, S, A, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j]);
+          }
+        }
         const int row = it.m_tile * NT + j;
         if (row < n_rows) {
           const int64_t o = static_cast<int64_t>(it.part * 2 + static_cast<int>(rank)) * a.P + row;
           a.part_m[o] = M;
           a.part_s[o] = S;
           a.part_a[o] = A;
+          if constexpr (VERIFY) {
+            a.part_t[o] = T;
+            a.part_x[o] = LX;
+          }
         }
       }
       mbar_arrive(epi_sync);
@@ -358,6 +436,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
 size_t pair_smem_bytes() { return SMEM_BYTES; }
 
+template <bool VERIFY>
 static cudaError_t pair_opt_in() {
   static std::atomic<uint64_t> opted_in{0};
   int dev = 0;
@@ -365,7 +444,7 @@ static cudaError_t pair_opt_in() {
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if ((opted_in.load() & bit) == 0) {
-    e = cudaFuncSetAttribute(lmhead_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(lmhead_pair_kernel<VERIFY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(SMEM_BYTES));
     if (e != cudaSuccess) return e;
     opted_in.fetch_or(bit);
@@ -394,25 +473,27 @@ static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int 
 }
 
 cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs) {
-  cudaError_t e = pair_opt_in();
+  cudaError_t e = pair_opt_in<false>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
   pair_config(&cfg, attr, sm_count / 2, nullptr, false);
   int n = 0;
-  e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel<false>, &cfg);
   if (e != cudaSuccess) return e;
   *pairs = n < 1 ? 1 : n;
   return cudaSuccess;
 }
 
 cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const TcArgs& a, cudaStream_t st) {
-  cudaError_t e = pair_opt_in();
+  const bool verify = a.part_t != nullptr;
+  cudaError_t e = verify ? pair_opt_in<true>() : pair_opt_in<false>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
   pair_config(&cfg, attr, a.plan.G, st, true);
-  return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel, tmH, tmW, a);
+  return verify ? cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<true>, tmH, tmW, a)
+                : cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<false>, tmH, tmW, a);
 }
 
 }  // namespace bd

@@ -1,7 +1,9 @@
 // LM-head projection + mask-suppressed softmax statistics with fp32 FMA on
 // the CUDA cores. This is the exact-fp32 path (fp32 hidden states and head),
 // and it accepts bf16 / e4m3 heads too. Same band plan and partial layout as
-// the tensor-core kernel, with 32-row m-tiles and 256-entry v-tiles.
+// the tensor-core kernel, with 32-row m-tiles and 256-entry v-tiles. The
+// verification instantiation (VERIFY = true) also carries the entropy
+// accumulator and the logit of each row's draft entry.
 #include <cuda_fp16.h>
 
 #include "bdcommit.h"
@@ -41,10 +43,13 @@ struct SimtSmem {
   } u;
   float rm[SIMT_BM], rs[SIMT_BM];
   int ra[SIMT_BM];
+  float rt[SIMT_BM], rx[SIMT_BM];  // VERIFY only
+  int xd[SIMT_BM];
 };
 
 }  // namespace
 
+template <bool VERIFY>
 __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   __shared__ SimtSmem sm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -59,7 +64,13 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
       sm.rm[tid] = -INFINITY;
       sm.rs[tid] = 0.f;
       sm.ra[tid] = 0x7fffffff;
+      if constexpr (VERIFY) {
+        sm.rt[tid] = 0.f;
+        sm.rx[tid] = -INFINITY;
+        sm.xd[tid] = r0 + tid < n_rows ? a.draft_row[r0 + tid] : -1;
+      }
     }
+    __syncthreads();
     for (int vt = it.vt; vt < it.vt_end; ++vt) {
       const int v = vt * SIMT_BN + tid;
       float acc[SIMT_BM];
@@ -94,29 +105,52 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
       const bool dead = (v >= a.V) || (v == a.mask_id);
       const float sc = (a.wscale != nullptr && v < a.V) ? a.wscale[v] : 1.f;
 #pragma unroll
-      for (int r = 0; r < SIMT_BM; ++r) sm.u.lg[r][tid] = dead ? -INFINITY : acc[r] * sc;
+      for (int r = 0; r < SIMT_BM; ++r) {
+        const float l = dead ? -INFINITY : acc[r] * sc;
+        sm.u.lg[r][tid] = l;
+        if constexpr (VERIFY) {
+          if (v == sm.xd[r]) sm.rx[r] = l;  // one column per row holds the draft entry
+        }
+      }
       __syncthreads();
       // warp w reduces rows 4w..4w+3; lane l scans columns 8l..8l+7 in order
       for (int rr = 0; rr < SIMT_BM / 8; ++rr) {
         const int r = warp * (SIMT_BM / 8) + rr;
-        float m = -INFINITY, s = 0.f;
+        float m = -INFINITY, s = 0.f, t = 0.f;
         int arg = 0x7fffffff;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           const float x = sm.u.lg[r][lane * 8 + j];
-          if (x != -INFINITY) softmax_combine(m, s, arg, x, 1.f, vt * SIMT_BN + lane * 8 + j);
+          if (x != -INFINITY) {
+            // one logit is a state of max x, sum 1 and first moment 0
+            if constexpr (VERIFY)
+              softmax_combine_t(m, s, arg, t, x, 1.f, vt * SIMT_BN + lane * 8 + j, 0.f);
+            else
+              softmax_combine(m, s, arg, x, 1.f, vt * SIMT_BN + lane * 8 + j);
+          }
         }
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
           const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
           const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
           const int a2 = __shfl_xor_sync(0xffffffffu, arg, o);
-          softmax_combine(m, s, arg, m2, s2, a2);
+          if constexpr (VERIFY) {
+            const float t2 = __shfl_xor_sync(0xffffffffu, t, o);
+            softmax_combine_t(m, s, arg, t, m2, s2, a2, t2);
+          } else {
+            softmax_combine(m, s, arg, m2, s2, a2);
+          }
         }
         if (lane == 0) {
           float M = sm.rm[r], S = sm.rs[r];
           int A = sm.ra[r];
-          softmax_combine(M, S, A, m, s, arg);
+          if constexpr (VERIFY) {
+            float T = sm.rt[r];
+            softmax_combine_t(M, S, A, T, m, s, arg, t);
+            sm.rt[r] = T;
+          } else {
+            softmax_combine(M, S, A, m, s, arg);
+          }
           sm.rm[r] = M;
           sm.rs[r] = S;
           sm.ra[r] = A;
@@ -129,6 +163,10 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
       a.part_m[o] = sm.rm[tid];
       a.part_s[o] = sm.rs[tid];
       a.part_a[o] = sm.ra[tid];
+      if constexpr (VERIFY) {
+        a.part_t[o] = sm.rt[tid];
+        a.part_x[o] = sm.rx[tid];
+      }
     }
     __syncthreads();
   }
@@ -145,7 +183,8 @@ cudaError_t launch_lmhead_simt(const SimtArgs& a, cudaStream_t st) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, lmhead_simt_kernel, a);
+  return a.part_t != nullptr ? cudaLaunchKernelEx(&cfg, lmhead_simt_kernel<true>, a)
+                             : cudaLaunchKernelEx(&cfg, lmhead_simt_kernel<false>, a);
 }
 
 }  // namespace bd

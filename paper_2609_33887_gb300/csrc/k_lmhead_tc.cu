@@ -14,6 +14,9 @@
 //               thread), 32 columns at a time
 // Every wait is bounded; on timeout the CTA raises DEV_TIMEOUT in the status
 // word, drains its copies and MMAs, frees TMEM and returns.
+// The verification instantiation (VERIFY = true) also carries the entropy
+// accumulator sum exp(l - m) (l - m) log2(e) and the logit of the row's draft
+// entry (typical-acceptance appendix).
 #include <atomic>
 
 #include "kernels.h"
@@ -42,7 +45,7 @@ struct Ctl {
 
 }  // namespace
 
-template <int STAGES>
+template <int STAGES, bool VERIFY>
 __global__ void __launch_bounds__(TC_THREADS, 1)
     lmhead_tc_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, TcArgs a) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -177,6 +180,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     while (ok && it.next_unit()) {
       float m = -INFINITY, s = 0.f;
       int arg = 0x7fffffff;
+      float t = 0.f, lx = -INFINITY;  // VERIFY only
+      int xd = -1;
+      if constexpr (VERIFY) {
+        const int row = it.m_tile * BM + row_in_tile;
+        if (row < n_rows) xd = a.draft_row[row];
+      }
       for (int vt = it.vt; vt < it.vt_end; ++vt) {
         if (!mbar_wait_warp(smem_u32(&ctl->tfull[acc]), acc_phase, abort_flag, a.status)) {
           ok = false;
@@ -203,6 +212,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             for (int j = 0; j < 32; ++j)
               if (col0 + j >= a.V || col0 + j == a.mask_id) v[j] = -INFINITY;
           }
+          if constexpr (VERIFY) {
+            if (static_cast<unsigned>(xd - col0) < 32u) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (col0 + j == xd) lx = v[j];
+            }
+          }
           float cm = v[0];
 #pragma unroll
           for (int j = 1; j < 32; ++j) cm = fmaxf(cm, v[j]);
@@ -212,18 +228,45 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             for (int j = 31; j >= 0; --j)
               if (v[j] == cm) jj = j;
             arg = col0 + jj;
-            s = (m == -INFINITY) ? 0.f : s * ex2_approx((m - cm) * LOG2E);
+            if constexpr (VERIFY) {
+              if (m == -INFINITY) {
+                s = 0.f;
+                t = 0.f;
+              } else {
+                const float dm = (m - cm) * LOG2E;
+                const float f = ex2_approx(dm);
+                t = f * fmaf(dm, s, t);
+                s *= f;
+              }
+            } else {
+              s = (m == -INFINITY) ? 0.f : s * ex2_approx((m - cm) * LOG2E);
+            }
             m = cm;
           }
           if (m != -INFINITY) {
             const float mc = m * LOG2E;
-            float s0 = 0.f, s1 = 0.f;
+            if constexpr (VERIFY) {
+              float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
-            for (int j = 0; j < 32; j += 2) {
-              s0 += ex2_approx(fmaf(v[j], LOG2E, -mc));
-              s1 += ex2_approx(fmaf(v[j + 1], LOG2E, -mc));
+              for (int j = 0; j < 32; j += 2) {
+                const float u0 = fmaf(v[j], LOG2E, -mc), u1 = fmaf(v[j + 1], LOG2E, -mc);
+                const float e0 = ex2_approx(u0), e1 = ex2_approx(u1);
+                s0 += e0;
+                s1 += e1;
+                t0 = fmaf(e0, fmaxf(u0, -256.f), t0);
+                t1 = fmaf(e1, fmaxf(u1, -256.f), t1);
+              }
+              s += s0 + s1;
+              t += t0 + t1;
+            } else {
+              float s0 = 0.f, s1 = 0.f;
+#pragma unroll
+              for (int j = 0; j < 32; j += 2) {
+                s0 += ex2_approx(fmaf(v[j], LOG2E, -mc));
+                s1 += ex2_approx(fmaf(v[j + 1], LOG2E, -mc));
+              }
+              s += s0 + s1;
             }
-            s += s0 + s1;
           }
         }
         tc_fence_before();
@@ -241,6 +284,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         a.part_m[o] = m;
         a.part_s[o] = s;
         a.part_a[o] = arg;
+        if constexpr (VERIFY) {
+          a.part_t[o] = t;
+          a.part_x[o] = lx;
+        }
       }
     }
   }
@@ -255,7 +302,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
 size_t tc_smem_bytes(int stages) { return static_cast<size_t>(stages) * STAGE_BYTES + sizeof(Ctl) + 1024; }
 
-template <int STAGES>
+template <int STAGES, bool VERIFY>
 static cudaError_t launch_stages(const CUtensorMap& tmA, const CUtensorMap& tmB, const TcArgs& a,
                                  cudaStream_t st) {
   const size_t smem = tc_smem_bytes(STAGES);
@@ -267,7 +314,7 @@ static cudaError_t launch_stages(const CUtensorMap& tmA, const CUtensorMap& tmB,
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if ((opted_in.load() & bit) == 0) {
-    e = cudaFuncSetAttribute(lmhead_tc_kernel<STAGES>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(lmhead_tc_kernel<STAGES, VERIFY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(smem));
     if (e != cudaSuccess) return e;
     opted_in.fetch_or(bit);
@@ -282,16 +329,17 @@ static cudaError_t launch_stages(const CUtensorMap& tmA, const CUtensorMap& tmB,
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, lmhead_tc_kernel<STAGES>, tmA, tmB, a);
+  return cudaLaunchKernelEx(&cfg, lmhead_tc_kernel<STAGES, VERIFY>, tmA, tmB, a);
 }
 
 cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, const TcArgs& a, int stages,
                              cudaStream_t st) {
+  const bool verify = a.part_t != nullptr;
   switch (stages) {
     case 3:
-      return launch_stages<3>(tmA, tmB, a, st);
+      return verify ? launch_stages<3, true>(tmA, tmB, a, st) : launch_stages<3, false>(tmA, tmB, a, st);
     default:
-      return launch_stages<4>(tmA, tmB, a, st);
+      return verify ? launch_stages<4, true>(tmA, tmB, a, st) : launch_stages<4, false>(tmA, tmB, a, st);
   }
 }
 

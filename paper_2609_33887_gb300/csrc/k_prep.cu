@@ -130,6 +130,34 @@ cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_fla
 }
 
 // ---------------------------------------------------------------------------
+// Verification rows need no compaction: every row is live. Row
+// r = q * (n_draft + 1) + i verifies draft token i of request q (i < n_draft);
+// the last row of a request verifies nothing.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restrict__ draft, int n_req, int n_draft,
+                                                          int* __restrict__ idx, int* __restrict__ draft_row,
+                                                          int* __restrict__ n_rows) {
+  griddep_launch_dependents();
+  const int R = n_req * (n_draft + 1);
+  for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
+    const int q = r / (n_draft + 1), i = r % (n_draft + 1);
+    idx[r] = r;
+    draft_row[r] = i < n_draft ? draft[q * n_draft + i] : -1;
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) *n_rows = R;
+}
+
+cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,
+                               cudaStream_t st) {
+  const int R = n_req * (n_draft + 1);
+  int grid = (R + 255) / 256;
+  if (grid < 1) grid = 1;
+  if (grid > 1024) grid = 1024;
+  prep_verify_kernel<<<grid, 256, 0, st>>>(draft, n_req, n_draft, idx, draft_row, n_rows);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
 // FP8 E4M3 -> bf16. Every e4m3 value (subnormals included) is exactly
 // representable in f16 and in bf16, so the decode is exact; the per-row
 // scale is applied later, to the fp32 logit.

@@ -39,6 +39,12 @@ struct TcArgs {
   float* part_s;
   int* part_a;
   uint32_t* status;
+  // verification path only (part_t != nullptr selects it): the draft token of
+  // each row (-1: none), and per partial the entropy accumulator t and the
+  // draft token's logit (-inf where the part does not hold it)
+  const int* draft_row = nullptr;
+  float* part_t = nullptr;
+  float* part_x = nullptr;
 };
 constexpr int TC_BM = 128;
 constexpr int TC_BN = 256;
@@ -75,6 +81,9 @@ struct SimtArgs {
   float* part_m;
   float* part_s;
   int* part_a;
+  const int* draft_row = nullptr;  // verification path, as in TcArgs
+  float* part_t = nullptr;
+  float* part_x = nullptr;
 };
 constexpr int SIMT_BM = 32;
 constexpr int SIMT_BN = 256;
@@ -100,5 +109,33 @@ struct CommitArgs {
   int32_t* out_counts;
 };
 cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st);
+
+// Verification path (speculative decoding, typical acceptance). Rows are
+// r = q * (n_draft + 1) + i; row i < n_draft of request q verifies draft
+// token draft[q * n_draft + i], the last row of a request gives its bonus token.
+// Prep: idx[r] = r, draft_row[r] = that draft token or -1, *n_rows = R.
+cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,
+                               cudaStream_t st);
+
+struct VerifyArgs {
+  const int* draft_row;
+  const int* n_rows;
+  BandPlan plan;
+  int P;  // rows
+  const float* part_m;
+  const float* part_s;
+  const int* part_a;
+  const float* part_t;
+  const float* part_x;
+  int n_req, n_draft, E;
+  float eps[31];
+  float sqrt_eps[31];
+  int32_t* out_tokens;
+  float* out_p_draft;
+  float* out_entropy;
+  uint32_t* out_accept;
+  int32_t* out_accepted;
+};
+cudaError_t launch_merge_verify(const VerifyArgs& a, cudaStream_t st);
 
 }  // namespace bd

@@ -40,7 +40,7 @@ def test_header_declares_the_abi():
     assert declared_functions() == sorted([
         "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status",
         "bd_shutdown",
-        "bd_status_string", "bd_version", "bd_workspace_size",
+        "bd_status_string", "bd_version", "bd_workspace_size", "bd_verify_step", "bd_verify_workspace_size",
         "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
         "bd_redline_select", "bd_redline_sweep", "bd_redline_critical_count", "bd_redline_power",
         "bd_redline_min_calibration", "bd_redline_tpf"])
@@ -167,3 +167,48 @@ def test_sweep_argument_checks(lib, kw, code):
 def test_sweep_empty_window_is_a_no_op(lib):
     assert _sweep(lib, n_seq=0, ptrs=(None, None, None), step=(None, None), cache=None, n_committed=None) == B.BD_OK
     assert lib.bd_commit_sweep(None, FAKE, FAKE, 0, 0, FAKE, FAKE, None, 0) == B.BD_ERR_NULL
+
+
+# ------------------------------------------------ verification argument checks --
+# every case fails a check before any CUDA call (none may reach a launch)
+def _verify(lib, n_req=4, n_draft=4, rows=None, eps=(0.1, 0.3), d=128, V=1000, hdt=B.BD_BF16, wdt=B.BD_BF16,
+            draft=FAKE, outs=(FAKE,) * 5, counts=None, variant=0, hptr=FAKE):
+    R = n_req * (n_draft + 1) if rows is None else rows
+    h = B.bd_hidden(hptr, hdt, R, d, d)
+    w = B.bd_weight(FAKE, wdt, V, d, d, None)
+    dr = B.bd_draft(n_req, n_draft, draft)
+    arr = (ctypes.c_float * max(1, len(eps)))(*eps)
+    eg = B.bd_eps_grid(ctypes.cast(arr, ctypes.POINTER(ctypes.c_float)), len(eps))
+    ex = B.bd_exec()
+    ex.variant = variant
+    ex.out_counts = counts
+    return lib.bd_verify_step(ctypes.byref(h), ctypes.byref(w), ctypes.byref(dr), ctypes.byref(eg), *outs,
+                              ctypes.byref(ex))
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(eps=()), B.BD_ERR_TAU),
+    (dict(eps=(0.1,) * 32), B.BD_ERR_TAU),
+    (dict(eps=(0.0,)), B.BD_ERR_TAU),
+    (dict(eps=(1.5,)), B.BD_ERR_TAU),
+    (dict(eps=(math.nan,)), B.BD_ERR_TAU),
+    (dict(n_draft=0), B.BD_ERR_SHAPE),
+    (dict(n_draft=33), B.BD_ERR_SHAPE),
+    (dict(rows=19), B.BD_ERR_SHAPE),
+    (dict(V=0), B.BD_ERR_SHAPE),
+    (dict(hdt=B.BD_F32), B.BD_ERR_DTYPE),
+    (dict(variant=2, hdt=B.BD_F32, wdt=B.BD_F32), B.BD_ERR_DTYPE),
+    (dict(variant=5), B.BD_ERR_ARG),
+    (dict(counts=FAKE), B.BD_ERR_ARG),
+    (dict(draft=None), B.BD_ERR_NULL),
+    (dict(draft=FAKE + 2), B.BD_ERR_ALIGN),
+    (dict(hptr=FAKE + 4), B.BD_ERR_ALIGN),
+    (dict(outs=(FAKE, FAKE, None, FAKE, FAKE)), B.BD_ERR_NULL),
+    (dict(outs=(FAKE, FAKE, FAKE, FAKE + 2, FAKE)), B.BD_ERR_ALIGN),
+])
+def test_verify_argument_checks(lib, kw, code):
+    assert _verify(lib, **kw) == code
+
+
+def test_verify_empty_batch_is_a_no_op(lib):
+    assert _verify(lib, n_req=0, draft=None, hptr=None, outs=(None,) * 5) == B.BD_OK
