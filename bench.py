@@ -52,6 +52,7 @@ def parse_args():
                     help="launch every step eagerly instead of replaying the K steps as one CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-verify", action="store_true", help="skip the speculative-verification measurement")
     return ap.parse_args()
 
 
@@ -290,6 +291,70 @@ def redline_timing(with_oracle: bool) -> dict:
     return out
 
 
+def verify_timing(dev, stream) -> dict:
+    """Speculative-decoding verification (bd_verify_step) at the Llama-3.1-8B
+    shape: 64 requests of 4 drafts (320 rows), d = 4096, V = 128256, bf16, the
+    paper's eleven typical-acceptance settings. Device time per step (CUDA
+    events around 200 back-to-back steps), the LM-head kernel's own time and
+    roofline, and the accepted tokens per target forward of each setting on
+    these synthetic drafts (agreement 0.905)."""
+    import statistics as st_
+
+    import paper_2609_33887_gb300 as bdc
+    from paper_2609_33887_gb300 import bdcommit as B
+    from workloads.verify_inputs import VERIFY_CONFIGS, generate_verify
+
+    cfg = VERIFY_CONFIGS[0]
+    wl = generate_verify(cfg).to(dev)
+    R = cfg.rows
+    ws = torch.empty(bdc.bd_verify_workspace_size(wl.hidden, wl.weight, None, wl.draft, cfg.n_req, cfg.n_draft,
+                                                  cfg.eps), dtype=torch.uint8, device=dev)
+    outs = {"tokens": torch.empty(R, dtype=torch.int32, device=dev),
+            "p_draft": torch.empty(R, dtype=torch.float32, device=dev),
+            "entropy": torch.empty(R, dtype=torch.float32, device=dev),
+            "accept": torch.empty(R, dtype=torch.int32, device=dev),
+            "accepted": torch.empty((cfg.n_req, len(cfg.eps) + 1), dtype=torch.int32, device=dev)}
+
+    def step(ev=None):
+        rc = B.bd_verify_step(wl.hidden, wl.weight, None, wl.draft, cfg.n_req, cfg.n_draft, cfg.eps, outs["tokens"],
+                              outs["p_draft"], outs["entropy"], outs["accept"], outs["accepted"], stream=stream,
+                              workspace=ws, lmhead_events=ev)
+        if rc != 0:
+            raise B.BdError(rc, "bd_verify_step")
+
+    for _ in range(5):
+        step()
+    n = 200
+    (e0, e1), = timing_events(1, stream)
+    e0.record(stream)
+    for _ in range(n):
+        step()
+    e1.record(stream)
+    lm = timing_events(20, stream)
+    for ev in lm:
+        step(ev)
+    torch.cuda.synchronize()
+    st = B.bd_get_device_status(stream)
+    if st != 0:
+        raise B.BdError(st, "verify")
+    ms = e0.elapsed_time(e1) / n
+    lm_s = st_.mean(a.elapsed_time(b) for a, b in lm) / 1e3
+    hbm_gbs, tc_tflops, _, src = peaks()
+    flops = 2.0 * R * cfg.d * cfg.V
+    abytes = cfg.V * cfg.d * 2 + R * cfg.d * 2 + R * 20
+    bound = "tensor" if flops / (tc_tflops * 1e12) >= abytes / (hbm_gbs * 1e9) else "hbm"
+    achieved = flops / lm_s / 1e12 if bound == "tensor" else abytes / lm_s / 1e9
+    peak = tc_tflops if bound == "tensor" else hbm_gbs
+    acc = outs["accepted"].float().mean(dim=0).cpu().tolist()
+    tpf = {("lossless" if k == len(cfg.eps) else f"eps={cfg.eps[k]}"): 1.0 + acc[k] for k in range(len(acc))}
+    return {"workload": cfg.name, "rows": R, "requests": cfg.n_req, "ms_per_step": ms,
+            "rows_per_s": R / (ms / 1e3), "lmhead_us": lm_s * 1e6,
+            "roofline": {"bound": bound, "achieved": achieved, "peak": peak,
+                         "unit": "TFLOP/s" if bound == "tensor" else "GB/s", "frac": achieved / peak,
+                         "peak_source": src, "algorithmic_flops": flops, "algorithmic_bytes": abytes},
+            "tokens_per_forward": tpf, "data": "synthetic drafts, agreement 0.905 with the planted argmax"}
+
+
 def run_ours(args):
     import paper_2609_33887_gb300 as bdc
     from paper_2609_33887_gb300 import bdcommit as B
@@ -510,6 +575,7 @@ def run_ours(args):
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
     redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
+    verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
 
     if rank == 0:
         line = {
@@ -529,6 +595,7 @@ def run_ours(args):
             "clocks": clocks,
             "redline": redline,
             "sweep": sweep,
+            "verify": verify,
         }
         print(json.dumps(line), flush=True)
     if pg:
