@@ -76,17 +76,54 @@ def decode_e4m3(raw: np.ndarray) -> np.ndarray:
     return out
 
 
-def weights_f64(raw: np.ndarray, dtype: str, scale: Optional[np.ndarray] = None) -> np.ndarray:
+def decode_e2m1(codes: np.ndarray) -> np.ndarray:
+    """FP4 E2M1 codes (0..15) -> float64, per the OCP microscaling 4-bit float:
+    1 sign bit, 2 exponent bits (bias 1), 1 mantissa bit; exponent field 0
+    encodes the subnormal m * 0.5; no infinities or NaN. The magnitudes of
+    codes 0..7 are 0, 0.5, 1, 1.5, 2, 3, 4, 6."""
+    c = np.asarray(codes, dtype=np.int64) & 0xF
+    sign = np.where(c & 0x8, -1.0, 1.0)
+    e = (c >> 1) & 0x3
+    m = (c & 0x1).astype(np.float64)
+    normal = (1.0 + m / 2.0) * np.exp2(e.astype(np.float64) - 1.0)
+    return sign * np.where(e == 0, m * 0.5, normal)
+
+
+def decode_nvfp4(codes: np.ndarray, block_scale: np.ndarray, d: int) -> np.ndarray:
+    """NVFP4 rows -> float64 [rows, d] (the 4-bit weight lever).
+
+    Row layout: element k of a row is the E2M1 code in the low nibble of byte
+    k // 2 when k is even, the high nibble when k is odd (codes [rows,
+    ceil(d / 2)]); each run of 16 elements shares one E4M3 scale, element k
+    using block_scale[:, k // 16] (block_scale [rows, ceil(d / 16)]). Value =
+    e2m1(code) * e4m3(block scale)."""
+    codes = np.asarray(codes, dtype=np.uint8)
+    k = np.arange(d)
+    byte = codes[:, k // 2].astype(np.int64)
+    nib = np.where(k % 2 == 0, byte & 0xF, byte >> 4)
+    bs = decode_e4m3(np.asarray(block_scale, dtype=np.uint8)[:, k // 16])
+    return decode_e2m1(nib) * bs
+
+
+def weights_f64(raw, dtype: str, scale: Optional[np.ndarray] = None, d: Optional[int] = None) -> np.ndarray:
     """Stored LM-head rows [rows, d] -> float64 values.
 
     f32 and bf16 rows are used as stored. e4m3 rows are the stored code times
     the row's (output channel's) float32 scale, i.e. exactly the dequantised
-    weights the library is handed, not the matrix before quantisation.
+    weights the library is handed, not the matrix before quantisation. nvfp4
+    rows are given as the pair (codes, block scales) and need the width d;
+    their values are decode_nvfp4 times the optional per-row float32 scale.
     "f64" rows are values already decoded by this function (a caller that
     evaluates many samples of one head decodes it once).
     """
     if dtype == "f64":
         return np.asarray(raw, dtype=np.float64)
+    if dtype == "nvfp4":
+        codes, bscale = raw
+        w = decode_nvfp4(codes, bscale, int(d))
+        if scale is not None:
+            w = w * np.asarray(scale, dtype=np.float32).astype(np.float64)[:, None]
+        return w
     if dtype == "f32":
         return np.asarray(raw, dtype=np.float32).astype(np.float64)
     if dtype == "bf16":
@@ -119,12 +156,14 @@ def lm_head_logits(h: np.ndarray, w_raw: np.ndarray, w_dtype: str,
     full dot product (a library matrix product serves as that step).
     """
     h = np.asarray(h, dtype=np.float64)
-    V = w_raw.shape[0]
+    packed = isinstance(w_raw, tuple)  # nvfp4: (codes, block scales)
+    V = w_raw[0].shape[0] if packed else w_raw.shape[0]
     out = np.empty((h.shape[0], V), dtype=np.float64)
     for r0 in range(0, V, chunk_rows):
         r1 = min(V, r0 + chunk_rows)
         sc = None if w_scale is None else w_scale[r0:r1]
-        w = weights_f64(w_raw[r0:r1], w_dtype, sc)
+        rows = tuple(x[r0:r1] for x in w_raw) if packed else w_raw[r0:r1]
+        w = weights_f64(rows, w_dtype, sc, d=h.shape[1])
         out[:, r0:r1] = h @ w.T
     return out
 
