@@ -64,3 +64,29 @@ def test_mask_fraction_is_close_to_the_stated_rate():
     wl = generate(c)
     frac = wl.pos_masked.float().mean().item()
     assert abs(frac - 0.6) < 0.07
+
+
+def test_nvfp4_head_quantisation():
+    """The NVFP4 head: per row the largest block scale is 448 (E4M3 max), and the
+    decoded head is close to the N(0, 1/d) draw it quantises (4-bit codes with
+    16-element blocks: relative RMS error well under 15%)."""
+    import math
+
+    import numpy as np
+    import torch
+
+    from oracle import commit_oracle as C
+    from workloads.generate import quantize_nvfp4
+
+    V, d = 512, 200
+    w = torch.randn(V, d, generator=torch.Generator().manual_seed(3)) / math.sqrt(d)
+    codes, bs, rs = quantize_nvfp4(w)
+    assert codes.shape == (V, 100) and bs.shape == (V, 13) and rs.shape == (V,)
+    bsv = C.decode_e4m3(bs.numpy())
+    assert np.allclose(bsv.max(axis=1), 448.0)
+    deq = C.weights_f64((codes.numpy(), bs.numpy()), "nvfp4", rs.numpy(), d=d)
+    err = np.sqrt(np.mean((deq - w.numpy()) ** 2)) / np.sqrt(np.mean(w.numpy() ** 2))
+    assert err < 0.15, err
+    # odd widths leave the last high nibble empty
+    codes, bs, rs = quantize_nvfp4(w[:, :33])
+    assert codes.shape == (V, 17) and np.all((codes[:, -1].numpy() >> 4) == 0)

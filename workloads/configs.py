@@ -48,7 +48,7 @@ class WorkloadConfig:
     d: int
     V: int
     hidden_dtype: str  # "f32" | "bf16"
-    weight_dtype: str  # "f32" | "bf16" | "e4m3"
+    weight_dtype: str  # "f32" | "bf16" | "e4m3" | "nvfp4"
     boost: str  # "fixed_half" | "single" | "tied_mix" | "none"
     boost_frac: float
     boost_lo: float
@@ -107,8 +107,15 @@ CONFIGS = (
 )
 
 
+# The 4-bit weight lever on the bench window (not one of the five workloads):
+# the b8x2x32 window and head shape with an NVFP4 head.
+EXTRA_CONFIGS = (
+    dataclasses.replace(CONFIGS[1], name="b8x2x32_d2048_v151936_nvfp4", weight_dtype="nvfp4"),
+)
+
+
 def by_name(name: str) -> WorkloadConfig:
-    for c in CONFIGS:
+    for c in CONFIGS + EXTRA_CONFIGS:
         if c.name == name:
             return c
     raise KeyError(name)

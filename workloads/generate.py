@@ -31,12 +31,13 @@ _TORCH_DTYPE = {"f32": torch.float32, "bf16": torch.bfloat16}
 class Workload:
     cfg: WorkloadConfig
     hidden: torch.Tensor  # [P, d], float32 or bfloat16
-    weight: torch.Tensor  # [V, d], float32, bfloat16 or float8_e4m3fn
-    weight_scale: Optional[torch.Tensor]  # [V] float32 for e4m3 weights, else None
+    weight: torch.Tensor  # [V, d], float32, bfloat16 or float8_e4m3fn; nvfp4: uint8 codes [V, ceil(d/2)]
+    weight_scale: Optional[torch.Tensor]  # [V] float32 for e4m3 and nvfp4 weights, else None
     pos_masked: torch.Tensor  # [P] uint8, 1 = still masked
     block_flags: torch.Tensor  # [n_seq * n_slots] uint8
     tau: Tuple[float, ...]
     mask_token_id: int
+    weight_block_scale: Optional[torch.Tensor] = None  # nvfp4: uint8 E4M3 codes [V, ceil(d/16)]
 
     @property
     def P(self) -> int:
@@ -52,6 +53,7 @@ class Workload:
             block_flags=self.block_flags.to(device),
             tau=self.tau,
             mask_token_id=self.mask_token_id,
+            weight_block_scale=None if self.weight_block_scale is None else self.weight_block_scale.to(device),
         )
 
 
@@ -121,13 +123,18 @@ def generate(cfg: WorkloadConfig) -> Workload:
         for r0 in range(0, V, step):
             r1 = min(V, r0 + step)
             stored[r0:r1] = (weight[r0:r1] / scale[r0:r1, None]).to(torch.float8_e4m3fn)
+    elif cfg.weight_dtype == "nvfp4":
+        stored, bscale, scale = quantize_nvfp4(weight)
     else:
         raise ValueError(cfg.weight_dtype)
-    del weight
 
-    # 4. planted boosts
+    # 4. planted boosts (along the unquantised rows for a 4-bit head)
     if cfg.boost != "none":
-        _plant(cfg, g, hidden, stored, scale)
+        if cfg.weight_dtype == "nvfp4":
+            _plant(cfg, g, hidden, weight, None)
+        else:
+            _plant(cfg, g, hidden, stored, scale)
+    del weight
 
     hidden = hidden.to(_TORCH_DTYPE[cfg.hidden_dtype]).contiguous()
     return Workload(
@@ -139,7 +146,48 @@ def generate(cfg: WorkloadConfig) -> Workload:
         block_flags=block_flags,
         tau=tuple(float(t) for t in cfg.tau),
         mask_token_id=cfg.mask_token_id,
+        weight_block_scale=bscale if cfg.weight_dtype == "nvfp4" else None,
     )
+
+
+_E2M1 = torch.tensor([0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0])
+
+
+def quantize_nvfp4(weight: torch.Tensor, chunk: int = 4096):
+    """[V, d] float32 -> NVFP4 (codes uint8 [V, ceil(d/2)], E4M3 block scales uint8
+    [V, ceil(d/16)], row scales float32 [V]). Per row, the row scale makes the
+    largest block scale 448 (the largest E4M3 value); a block's scale is its
+    absolute maximum / (6 * row scale) rounded to E4M3; each element is
+    x / (block scale * row scale) rounded to the nearest E2M1 value, ties to
+    the even code. Element k sits in the low nibble of byte k // 2 when k is even."""
+    V, d = weight.shape
+    nb = (d + 15) // 16
+    dp = nb * 16
+    codes = torch.zeros(V, (d + 1) // 2, dtype=torch.uint8)
+    bscale = torch.zeros(V, nb, dtype=torch.uint8)
+    rscale = torch.zeros(V, dtype=torch.float32)
+    for r0 in range(0, V, chunk):
+        r1 = min(V, r0 + chunk)
+        w = torch.zeros(r1 - r0, dp)
+        w[:, :d] = weight[r0:r1]
+        blk = w.view(r1 - r0, nb, 16)
+        amax = blk.abs().amax(dim=2)
+        rs = (amax.amax(dim=1) / (6.0 * 448.0)).clamp_min(1e-30)
+        bs8 = (amax / (6.0 * rs[:, None])).to(torch.float8_e4m3fn)
+        bsv = bs8.float()
+        denom = (bsv * rs[:, None]).clamp_min(1e-38)
+        q = (blk / denom[:, :, None]).clamp(-6.0, 6.0)
+        mag = q.abs().reshape(-1, 1)
+        dist = (mag - _E2M1[None, :]).abs() + (torch.arange(8) % 2)[None, :] * 1e-7  # ties to the even code
+        idx = dist.argmin(dim=1)
+        sign = ((q.reshape(-1) < 0) & (idx > 0)).to(torch.int64)
+        code = (idx | (sign << 3)).view(r1 - r0, dp)[:, :d]
+        if d % 2:
+            code = torch.cat([code, torch.zeros(r1 - r0, 1, dtype=code.dtype)], dim=1)
+        codes[r0:r1] = (code[:, 0::2] | (code[:, 1::2] << 4)).to(torch.uint8)
+        bscale[r0:r1] = bs8.view(torch.uint8)
+        rscale[r0:r1] = rs
+    return codes.contiguous(), bscale.contiguous(), rscale.contiguous()
 
 
 def _plant(cfg, g, hidden, stored, scale):
