@@ -57,7 +57,8 @@ typedef enum {
 typedef enum {
   BD_F32 = 0,  /* IEEE binary32 */
   BD_BF16 = 1, /* bfloat16 */
-  BD_E4M3 = 2  /* FP8 E4M3 (OCP "fn" variant: no infinities), weights only */
+  BD_E4M3 = 2, /* FP8 E4M3 (OCP "fn" variant: no infinities), weights only */
+  BD_NVFP4 = 3 /* 4-bit E2M1 codes with an E4M3 scale per 16 elements (NVFP4), weights only */
 } bd_dtype;
 
 /* Block flag bits (bd_mask_state.block_flags). */
@@ -86,15 +87,26 @@ typedef struct {
  *   dtype BD_E4M3 : with BD_BF16 hidden states; `scale` is a device float32
  *                   array [vocab] and the weight of row v is code * scale[v]
  *                   (per-output-channel scaling, the FP8 precision lever).
- *   For BD_BF16 / BD_E4M3 the pointer must be 16-byte aligned and
- *   ld * element size a multiple of 16 (TMA row stride rule). */
+ *   dtype BD_NVFP4: with BD_BF16 hidden states (the 4-bit weight lever).
+ *                   `data` holds E2M1 codes, two per byte: element k of a row
+ *                   is the low nibble of byte k / 2 for even k, the high
+ *                   nibble for odd k; `ld` counts BYTES (>= ceil(dim / 2));
+ *                   `block_scale` [vocab, block_ld] holds E4M3 codes, element
+ *                   k using block_scale[v * block_ld + k / 16] (block_ld >=
+ *                   ceil(dim / 16)); `scale` is an optional float32 [vocab]
+ *                   per-row scale (NULL = 1). Weight (v, k) =
+ *                   e2m1(code) * e4m3(block scale) * scale[v].
+ *   For BD_BF16 / BD_E4M3 / BD_NVFP4 the pointer must be 16-byte aligned and
+ *   ld * element size (bytes for BD_NVFP4) a multiple of 16. */
 typedef struct {
   const void* data;
   int32_t dtype;
   int64_t vocab;
   int64_t dim;
   int64_t ld;
-  const float* scale; /* required iff dtype == BD_E4M3, else ignored */
+  const float* scale;         /* required for BD_E4M3, optional for BD_NVFP4, else ignored */
+  const uint8_t* block_scale; /* BD_NVFP4 only */
+  int64_t block_ld;           /* BD_NVFP4 only */
 } bd_weight;
 
 /* Which positions are still masked and which slots hold active blocks

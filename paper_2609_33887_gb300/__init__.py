@@ -14,6 +14,7 @@ from .bdcommit import (
     BD_SWEEP_ADMIT,
     BD_SWEEP_ELIGIBLE_OLDEST,
     BdError,
+    Nvfp4Head,
     bd_commit_step,
     bd_commit_step_ex,
     bd_commit_sweep,
@@ -37,6 +38,7 @@ __all__ = [
     "BD_SWEEP_ADMIT",
     "BD_SWEEP_ELIGIBLE_OLDEST",
     "BdError",
+    "Nvfp4Head",
     "bd_commit_step",
     "bd_commit_step_ex",
     "bd_commit_sweep",

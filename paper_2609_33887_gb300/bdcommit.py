@@ -11,6 +11,7 @@ from __future__ import annotations
 import ctypes
 import os
 from ctypes import POINTER, c_float, c_int, c_int32, c_int64, c_size_t, c_void_p
+from dataclasses import dataclass
 from typing import Optional, Sequence
 
 import torch
@@ -35,6 +36,7 @@ BD_ERR_ARG = -10
 BD_F32 = 0
 BD_BF16 = 1
 BD_E4M3 = 2
+BD_NVFP4 = 3
 
 BD_BLOCK_ACTIVE = 1
 BD_BLOCK_FALLBACK_ELIGIBLE = 2
@@ -54,7 +56,7 @@ class bd_hidden(ctypes.Structure):
 
 class bd_weight(ctypes.Structure):
     _fields_ = [("data", c_void_p), ("dtype", c_int32), ("vocab", c_int64), ("dim", c_int64), ("ld", c_int64),
-                ("scale", c_void_p)]
+                ("scale", c_void_p), ("block_scale", c_void_p), ("block_ld", c_int64)]
 
 
 class bd_mask_state(ctypes.Structure):
@@ -150,11 +152,28 @@ def make_hidden(hidden: torch.Tensor) -> bd_hidden:
     return bd_hidden(_ptr(hidden), _DT[hidden.dtype], hidden.shape[0], hidden.shape[1], hidden.stride(0))
 
 
-def make_weight(weight: torch.Tensor, scale: Optional[torch.Tensor] = None) -> bd_weight:
+@dataclass
+class Nvfp4Head:
+    """An NVFP4 LM head as the library reads it: codes uint8 [vocab, ceil(dim/2)]
+    (two E2M1 codes per byte, low nibble first), block_scale uint8
+    [vocab, ceil(dim/16)] (E4M3 codes, one per 16 elements) and the width dim.
+    The optional per-row float32 scale is passed as the weight scale."""
+    codes: torch.Tensor
+    block_scale: torch.Tensor
+    dim: int
+
+
+def make_weight(weight, scale: Optional[torch.Tensor] = None) -> bd_weight:
+    if isinstance(weight, Nvfp4Head):
+        c, b = weight.codes, weight.block_scale
+        if c.dtype != torch.uint8 or b.dtype != torch.uint8 or c.dim() != 2 or b.dim() != 2 \
+                or c.stride(1) != 1 or b.stride(1) != 1:
+            raise ValueError("NVFP4 codes and block scales must be 2-D uint8 tensors with contiguous rows")
+        return bd_weight(_ptr(c), BD_NVFP4, c.shape[0], weight.dim, c.stride(0), _ptr(scale), _ptr(b), b.stride(0))
     if weight.dim() != 2 or weight.stride(1) != 1:
         raise ValueError("weight must be a 2-D [vocab, dim] tensor with contiguous rows")
     return bd_weight(_ptr(weight), _DT[weight.dtype], weight.shape[0], weight.shape[1], weight.stride(0),
-                     _ptr(scale))
+                     _ptr(scale), None, 0)
 
 
 def make_mask_state(pos_masked: torch.Tensor, block_flags: torch.Tensor, n_seq: int, n_slots: int,

@@ -82,7 +82,24 @@ struct Call {
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }
+int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }  // NVFP4: ld counts bytes
+
+bool decoded_head(const Call& c) { return c.tc && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4); }
+
+// Decodes an FP8 or NVFP4 head into the bf16 workspace copy the tensor-core
+// kernels read (both decodes are exact); wsrc / wld then describe that copy.
+int decode_head(const Call& c, const bd_weight* weight, void* wq, int sm_count, cudaStream_t st, const void** wsrc,
+                int64_t* wld) {
+  const int V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+  cudaError_t e = c.wdt == BD_E4M3
+                      ? bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
+                                                sm_count, st)
+                      : bd::launch_dequant_nvfp4(static_cast<const uint8_t*>(weight->data), c.ldw,
+                                                 weight->block_scale, weight->block_ld, V, d, wq, c.ldq, sm_count, st);
+  *wsrc = wq;
+  *wld = c.ldq;
+  return e == cudaSuccess ? BD_OK : BD_ERR_CUDA;
+}
 
 int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
@@ -103,18 +120,19 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   if (h->rows != P) return BD_ERR_SHAPE;
   if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
   if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
-  if (h->ld < h->cols || w->ld < w->dim) return BD_ERR_SHAPE;
+  if (h->ld < h->cols || w->ld < (w->dtype == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim)) return BD_ERR_SHAPE;
   if (ms->mask_token_id < -1 || ms->mask_token_id >= w->vocab) return BD_ERR_ARG;
   if (ms->mask_token_id >= 0 && w->vocab < 2) return BD_ERR_SHAPE;  // nothing left to predict
   const int hdt = h->dtype, wdt = w->dtype;
   const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
-  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3);
+  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3 || wdt == BD_NVFP4);
   if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
   const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
   if (tc && !combo_bf16) return BD_ERR_DTYPE;
   if (P > 0) {
     if (!h->data || !w->data || !ms->pos_masked || !ms->block_flags) return BD_ERR_NULL;
     if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
+    if (wdt == BD_NVFP4 && !w->block_scale) return BD_ERR_NULL;
   }
   if (tc) {
     if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
@@ -122,7 +140,8 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   } else {
     if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
   }
-  if (w->scale && wdt == BD_E4M3 && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  if (w->scale && (wdt == BD_E4M3 || wdt == BD_NVFP4) && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  if (wdt == BD_NVFP4 && w->block_ld < (w->dim + 15) / 16) return BD_ERR_SHAPE;
   c->P = P;
   c->d = w->dim;
   c->V = w->vocab;
@@ -203,7 +222,7 @@ Layout make_layout(const Call& c, const BandPlan& p) {
   l.ps = take(4 * slots * P, 256);
   l.pa = take(4 * slots * P, 256);
   l.hc = c.tc ? take(2 * static_cast<size_t>(c.ldc) * P, 1024) : 0;
-  l.wq = (c.tc && c.wdt == BD_E4M3) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
+  l.wq = decoded_head(c) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
   l.total = (off + 255) / 256 * 256;
   return l;
 }
@@ -270,13 +289,9 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
     void* hc = ws + lay.hc;
     const void* wsrc = weight->data;
     int64_t wld = c.ldw;
-    if (c.wdt == BD_E4M3) {
-      void* wq = ws + lay.wq;
-      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
-                                               sm_count, st));
+    if (decoded_head(c)) {
+      rc = decode_head(c, weight, ws + lay.wq, sm_count, st, &wsrc, &wld);
       if (rc != BD_OK) return rc;
-      wsrc = wq;
-      wld = c.ldq;
     }
     if (c.pair) {
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
@@ -294,7 +309,7 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   if (c.tc) {
     bd::TcArgs a;
     a.n_rows = n_rows;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
     a.V = V;
     a.d = d;
     a.P = P;
@@ -314,7 +329,9 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
     a.w = weight->data;
     a.ldw = c.ldw;
     a.wdtype = c.wdt;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.wbs = weight->block_scale;
+    a.ldbs = weight->block_ld;
+    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
     a.idx = idx;
     a.n_rows = n_rows;
     a.V = V;
@@ -579,16 +596,17 @@ int check_verify(const bd_hidden* h, const bd_weight* w, const bd_draft* dr, con
   if (R > MAX_POSITIONS || h->rows != R) return BD_ERR_SHAPE;
   if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
   if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
-  if (h->ld < h->cols || w->ld < w->dim) return BD_ERR_SHAPE;
+  if (h->ld < h->cols || w->ld < (w->dtype == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim)) return BD_ERR_SHAPE;
   const int hdt = h->dtype, wdt = w->dtype;
   const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
-  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3);
+  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3 || wdt == BD_NVFP4);
   if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
   const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
   if (tc && !combo_bf16) return BD_ERR_DTYPE;
   if (R > 0) {
     if (!h->data || !w->data || !dr->draft) return BD_ERR_NULL;
     if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
+    if (wdt == BD_NVFP4 && !w->block_scale) return BD_ERR_NULL;
     if (!aligned(dr->draft, 4)) return BD_ERR_ALIGN;
   }
   if (tc) {
@@ -597,7 +615,8 @@ int check_verify(const bd_hidden* h, const bd_weight* w, const bd_draft* dr, con
   } else {
     if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
   }
-  if (w->scale && wdt == BD_E4M3 && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  if (w->scale && (wdt == BD_E4M3 || wdt == BD_NVFP4) && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  if (wdt == BD_NVFP4 && w->block_ld < (w->dim + 15) / 16) return BD_ERR_SHAPE;
   Call& c = vc->c;
   c = Call{};
   c.P = R;
@@ -645,7 +664,7 @@ VerifyLayout make_verify_layout(const Call& c, const BandPlan& p) {
   l.pa = take(4 * slots * R, 256);
   l.pt = take(4 * slots * R, 256);
   l.px = take(4 * slots * R, 256);
-  l.wq = (c.tc && c.wdt == BD_E4M3) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
+  l.wq = decoded_head(c) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
   l.total = (off + 255) / 256 * 256;
   return l;
 }
@@ -673,13 +692,9 @@ int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& l
   if (c.tc) {
     const void* wsrc = weight->data;
     int64_t wld = c.ldw;
-    if (c.wdt == BD_E4M3) {
-      void* wq = ws + lay.wq;
-      rc = cuda_status(bd::launch_dequant_e4m3(static_cast<const uint8_t*>(weight->data), c.ldw, V, d, wq, c.ldq,
-                                               sm_count, st));
+    if (decoded_head(c)) {
+      rc = decode_head(c, weight, ws + lay.wq, sm_count, st, &wsrc, &wld);
       if (rc != BD_OK) return rc;
-      wsrc = wq;
-      wld = c.ldq;
     }
     if (c.pair) {
       for (int i = 0; i < 8; ++i)
@@ -695,7 +710,7 @@ int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& l
   if (c.tc) {
     bd::TcArgs a;
     a.n_rows = n_rows;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
     a.V = V;
     a.d = d;
     a.P = R;
@@ -718,7 +733,9 @@ int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& l
     a.w = weight->data;
     a.ldw = c.ldw;
     a.wdtype = c.wdt;
-    a.wscale = c.wdt == BD_E4M3 ? weight->scale : nullptr;
+    a.wbs = weight->block_scale;
+    a.ldbs = weight->block_ld;
+    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
     a.idx = idx;
     a.n_rows = n_rows;
     a.V = V;

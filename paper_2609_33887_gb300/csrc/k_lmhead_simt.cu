@@ -35,6 +35,18 @@ __device__ __forceinline__ float load_w(const void* p, int64_t i, int dt) {
   return e4m3_to_float(static_cast<const uint8_t*>(p)[i]);
 }
 
+// NVFP4 element (v, k): the E2M1 nibble k of row v (low nibble first) times
+// the E4M3 scale of its 16-element block; the value is built from the code's
+// bit fields (sign, 2-bit exponent with bias 1, 1-bit mantissa).
+__device__ __forceinline__ float load_w_nvfp4(const void* p, const uint8_t* bs, int v, int k, int64_t ldw,
+                                              int64_t ldbs) {
+  const uint8_t byte = static_cast<const uint8_t*>(p)[static_cast<int64_t>(v) * ldw + k / 2];
+  const uint32_t c = (k & 1) ? (byte >> 4) : (byte & 0xFu);
+  const uint32_t e = (c >> 1) & 3u, m = c & 1u;
+  const uint32_t mag = e == 0 ? (m ? 0x3F000000u : 0u) : (((126u + e) << 23) | (m << 22));
+  return __uint_as_float(mag | ((c & 8u) << 28)) * e4m3_to_float(bs[static_cast<int64_t>(v) * ldbs + k / 16]);
+}
+
 struct SimtSmem {
   float hs[SIMT_BM][KC + 1];
   union {
@@ -90,7 +102,9 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
           const int vr = e / KC, kk = e % KC;
           const int vv = vt * SIMT_BN + vr;
           float x = 0.f;
-          if (vv < a.V && k0 + kk < a.d) x = load_w(a.w, static_cast<int64_t>(vv) * a.ldw + k0 + kk, a.wdtype);
+          if (vv < a.V && k0 + kk < a.d)
+            x = a.wdtype == BD_NVFP4 ? load_w_nvfp4(a.w, a.wbs, vv, k0 + kk, a.ldw, a.ldbs)
+                                     : load_w(a.w, static_cast<int64_t>(vv) * a.ldw + k0 + kk, a.wdtype);
           sm.u.ws[vr][kk] = x;
         }
         __syncthreads();

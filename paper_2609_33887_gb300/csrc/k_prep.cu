@@ -1,6 +1,6 @@
 // Preparation kernels of the commit step: compaction of the still-masked
 // positions of active blocks, packing of their hidden rows, and the FP8 e4m3
-// -> bf16 weight decode of the precision lever.
+// and NVFP4 -> bf16 weight decodes of the precision levers.
 #include "kernels.h"
 
 namespace bd {
@@ -210,6 +210,63 @@ cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, voi
                                 cudaStream_t st) {
   int grid = sm_count * 16;
   dequant_e4m3_kernel<<<grid, 256, 0, st>>>(w, ldw, V, d, static_cast<__nv_bfloat16*>(out), ldo);
+  return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------------------
+// NVFP4 -> bf16. An E2M1 code is 1 sign bit, 2 exponent bits (bias 1) and 1
+// mantissa bit; its value (1 + m/2) * 2^(e-1), or m/2 for e = 0, is built
+// directly as a binary32 bit pattern. Times the E4M3 block scale the product
+// has at most 5 significant bits, so the bf16 result is exact; the per-row
+// scale is applied later, to the fp32 logit.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float e2m1_value(uint32_t c) {
+  const uint32_t e = (c >> 1) & 3u, m = c & 1u;
+  const uint32_t mag = e == 0 ? (m ? 0x3F000000u : 0u) : (((126u + e) << 23) | (m << 22));
+  return __uint_as_float(mag | ((c & 8u) << 28));
+}
+
+__device__ __forceinline__ float e4m3_value(uint8_t c) {
+  uint32_t h2;
+  asm("cvt.rn.f16x2.e4m3x2 %0, %1;" : "=r"(h2) : "h"(static_cast<uint16_t>(c)));
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(h2 & 0xffffu)));
+}
+
+__global__ void __launch_bounds__(256) dequant_nvfp4_kernel(const uint8_t* __restrict__ codes, int64_t ldw,
+                                                            const uint8_t* __restrict__ bs, int64_t ldbs, int V,
+                                                            int d, __nv_bfloat16* __restrict__ out, int64_t ldo) {
+  // one thread per 16-element block: 8 code bytes (8-byte aligned: ldw % 16 == 0)
+  const int nblk = (d + 15) / 16;
+  const int64_t total = static_cast<int64_t>(V) * nblk;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int v = static_cast<int>(t / nblk);
+    const int b = static_cast<int>(t % nblk);
+    const int k0 = b * 16;
+    const uint2 q = __ldg(reinterpret_cast<const uint2*>(codes + static_cast<int64_t>(v) * ldw + k0 / 2));
+    const float sc = e4m3_value(bs[static_cast<int64_t>(v) * ldbs + b]);
+    __nv_bfloat16 o[16];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const uint32_t byte = ((j < 4 ? q.x : q.y) >> (8 * (j & 3))) & 0xFFu;
+      o[2 * j] = __float2bfloat16_rn(e2m1_value(byte & 0xFu) * sc);
+      o[2 * j + 1] = __float2bfloat16_rn(e2m1_value(byte >> 4) * sc);
+    }
+    __nv_bfloat16* dst = out + static_cast<int64_t>(v) * ldo + k0;
+    if (k0 + 16 <= d) {
+      // ldo % 8 == 0 and k0 % 16 == 0 keep both stores 16-byte aligned
+      reinterpret_cast<uint4*>(dst)[0] = *reinterpret_cast<const uint4*>(&o[0]);
+      reinterpret_cast<uint4*>(dst)[1] = *reinterpret_cast<const uint4*>(&o[8]);
+    } else {
+      for (int j = 0; k0 + j < d; ++j) dst[j] = o[j];
+    }
+  }
+}
+
+cudaError_t launch_dequant_nvfp4(const uint8_t* codes, int64_t ldw, const uint8_t* bs, int64_t ldbs, int V, int d,
+                                 void* out, int64_t ldo, int sm_count, cudaStream_t st) {
+  int grid = sm_count * 16;
+  dequant_nvfp4_kernel<<<grid, 256, 0, st>>>(codes, ldw, bs, ldbs, V, d, static_cast<__nv_bfloat16*>(out), ldo);
   return cudaGetLastError();
 }
 

@@ -28,6 +28,11 @@ cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_fla
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
                                 int sm_count, cudaStream_t st);
 
+// Decodes NVFP4 rows to bf16 (exact: every E2M1 x E4M3 product is a bf16):
+// out[v][k] = e2m1(nibble k of codes[v]) * e4m3(bs[v][k / 16]).
+cudaError_t launch_dequant_nvfp4(const uint8_t* codes, int64_t ldw, const uint8_t* bs, int64_t ldbs, int V, int d,
+                                 void* out, int64_t ldo, int sm_count, cudaStream_t st);
+
 // a1+a2 on the tensor cores: tcgen05 LM-head GEMM with the online softmax
 // epilogue. tmA describes hc [P, d] bf16, tmB the head [V, d] bf16.
 struct TcArgs {
@@ -72,7 +77,9 @@ struct SimtArgs {
   int hdtype;  // BD_F32 / BD_BF16
   const void* w;
   int64_t ldw;
-  int wdtype;  // BD_F32 / BD_BF16 / BD_E4M3
+  int wdtype;  // BD_F32 / BD_BF16 / BD_E4M3 / BD_NVFP4
+  const uint8_t* wbs;  // BD_NVFP4 block scales [V, ldbs]
+  int64_t ldbs;
   const float* wscale;
   const int* idx;
   const int* n_rows;

@@ -14,7 +14,8 @@ import numpy as np
 
 GAP_TOL = 1e-3
 TAU_TOL = 2e-3
-CONF_TOL = {"f32": 2e-3, "bf16": 2e-3, "e4m3": 1e-2}
+# NVFP4 heads decode exactly to bf16 on the device and take the bf16 path's arithmetic
+CONF_TOL = {"f32": 2e-3, "bf16": 2e-3, "e4m3": 1e-2, "nvfp4": 2e-3}
 
 
 @dataclass

@@ -212,3 +212,24 @@ def test_verify_argument_checks(lib, kw, code):
 
 def test_verify_empty_batch_is_a_no_op(lib):
     assert _verify(lib, n_req=0, draft=None, hptr=None, outs=(None,) * 5) == B.BD_OK
+
+
+# ------------------------------------------------------- NVFP4 head checks --
+def _nvfp4_call(lib, ld=64, bs=FAKE, bld=4, d=128, hdt=B.BD_BF16, variant=0):
+    h, _w, ms, tg, _keep = _args(d=d, hdt=hdt)
+    w = B.bd_weight(FAKE, B.BD_NVFP4, 1000, d, ld, None, bs, bld)
+    ex = B.bd_exec()
+    ex.variant = variant
+    return lib.bd_commit_step_ex(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+                                 FAKE, FAKE, FAKE, ctypes.byref(ex))
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(bs=None), B.BD_ERR_NULL),
+    (dict(bld=7, d=128), B.BD_ERR_SHAPE),      # ceil(128 / 16) = 8 scales per row
+    (dict(ld=63), B.BD_ERR_SHAPE),             # fewer than ceil(128 / 2) bytes per row
+    (dict(ld=72, bld=8), B.BD_ERR_ALIGN),      # row stride not a multiple of 16 bytes
+    (dict(hdt=B.BD_F32, bld=8), B.BD_ERR_DTYPE),
+])
+def test_nvfp4_argument_checks(lib, kw, code):
+    assert _nvfp4_call(lib, **kw) == code
