@@ -52,7 +52,8 @@ def parse_args():
                     help="launch every step eagerly instead of replaying the K steps as one CUDA graph")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-verify", action="store_true", help="skip the speculative-verification measurement")
+    ap.add_argument("--no-verify", action="store_true",
+                    help="skip the speculative-verification and NVFP4-head measurements")
     return ap.parse_args()
 
 
@@ -355,6 +356,60 @@ def verify_timing(dev, stream) -> dict:
             "tokens_per_forward": tpf, "data": "synthetic drafts, agreement 0.905 with the planted argmax"}
 
 
+def nvfp4_timing(dev, stream) -> dict:
+    """The bench window (8 x 2 x 32, d = 2048, V = 151936) with the head in
+    NVFP4 (the 4-bit weight lever): device time per commit step (CUDA events
+    around 200 back-to-back steps), the LM-head kernel's own time, and the
+    step against the 4-bit algorithmic bytes (codes V*d/2, block scales
+    V*d/16, row scales 4V, the masked rows and 13 B per window position)."""
+    import statistics as st_
+
+    import paper_2609_33887_gb300 as bdc
+    from paper_2609_33887_gb300 import bdcommit as B
+
+    cfg = by_name("b8x2x32_d2048_v151936_nvfp4")
+    wl = generate(cfg).to(dev)
+    head = bdc.Nvfp4Head(wl.weight, wl.weight_block_scale, cfg.d)
+    P, T = cfg.P, len(cfg.tau)
+    ws = torch.empty(bdc.bd_workspace_size(wl.hidden, head, wl.weight_scale, wl.pos_masked, wl.block_flags,
+                                           cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau),
+                     dtype=torch.uint8, device=dev)
+    tokens = torch.empty(P, dtype=torch.int32, device=dev)
+    conf = torch.empty(P, dtype=torch.float32, device=dev)
+    commit = torch.empty(P, dtype=torch.int32, device=dev)
+
+    def step(ev=None):
+        rc = B.bd_commit_step_ex(wl.hidden, head, wl.weight_scale, wl.pos_masked, wl.block_flags, cfg.n_seq,
+                                 cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau, tokens, conf, commit,
+                                 stream=stream, workspace=ws, lmhead_events=ev)
+        if rc != 0:
+            raise B.BdError(rc, "nvfp4 step")
+
+    for _ in range(5):
+        step()
+    n = 200
+    (e0, e1), = timing_events(1, stream)
+    e0.record(stream)
+    for _ in range(n):
+        step()
+    e1.record(stream)
+    lm = timing_events(20, stream)
+    for ev in lm:
+        step(ev)
+    torch.cuda.synchronize()
+    st = B.bd_get_device_status(stream)
+    if st != 0:
+        raise B.BdError(st, "nvfp4")
+    ms = e0.elapsed_time(e1) / n
+    lm_us = st_.mean(a.elapsed_time(b) for a, b in lm) * 1e3
+    n_masked = int(((wl.pos_masked != 0) & (torch.repeat_interleave(wl.block_flags & 1, cfg.block_len) != 0)).sum())
+    abytes = cfg.V * cfg.d // 2 + cfg.V * ((cfg.d + 15) // 16) + 4 * cfg.V + n_masked * cfg.d * 2 + P * 13
+    hbm_gbs, _, _, src = peaks()
+    return {"workload": cfg.name, "ms_per_step": ms, "positions_per_s": n_masked / (ms / 1e3),
+            "lmhead_us": lm_us, "algorithmic_bytes": abytes,
+            "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs, "peak_source": src}
+
+
 def run_ours(args):
     import paper_2609_33887_gb300 as bdc
     from paper_2609_33887_gb300 import bdcommit as B
@@ -576,6 +631,7 @@ def run_ours(args):
 
     redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
     verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
+    nvfp4 = nvfp4_timing(dev, stream) if rank == 0 and not args.no_verify else None
 
     if rank == 0:
         line = {
@@ -596,6 +652,7 @@ def run_ours(args):
             "redline": redline,
             "sweep": sweep,
             "verify": verify,
+            "nvfp4": nvfp4,
         }
         print(json.dumps(line), flush=True)
     if pg:

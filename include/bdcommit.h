@@ -195,6 +195,15 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
  * outputs are then invalid), or BD_ERR_CUDA if the synchronisation failed. */
 int bd_get_device_status(void* stream);
 
+/* Failure-detection self-test (the paper has no counterpart). Queues on
+ * `stream` one small kernel that waits, through the same bounded wait the
+ * tensor-core kernels use, on a barrier that nothing ever completes; after the
+ * wait limit (about 1 s) it records the timeout in the device status word of
+ * the current device and returns. The next bd_get_device_status then returns
+ * BD_ERR_TIMEOUT and clears the word; the context stays usable. No fault, trap
+ * or hang is involved. Returns BD_OK once queued (or BD_ERR_DEVICE / BD_ERR_CUDA). */
+int bd_selftest_timeout(void* stream);
+
 /* Static English text for a status code. Never NULL. */
 const char* bd_status_string(int status);
 

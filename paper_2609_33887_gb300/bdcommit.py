@@ -125,6 +125,7 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
         "bd_commit_sweep": (c_int, [POINTER(bd_window), c_void_p, c_void_p, c_int32, ctypes.c_uint32, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),
         "bd_get_device_status": (c_int, [c_void_p]),
+        "bd_selftest_timeout": (c_int, [c_void_p]),
         "bd_status_string": (ctypes.c_char_p, [c_int]),
         "bd_shutdown": (c_int, []),
         "bd_version": (c_int, []),
@@ -213,6 +214,11 @@ def bd_shutdown() -> int:
 
 def bd_get_device_status(stream=None) -> int:
     return int(load_library().bd_get_device_status(_stream_handle(stream)))
+
+
+def bd_selftest_timeout(stream=None) -> int:
+    """Queue the failure-detection self-test: a bounded wait that runs out (about 1 s)."""
+    return int(load_library().bd_selftest_timeout(_stream_handle(stream)))
 
 
 def bd_workspace_size(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,

@@ -461,6 +461,13 @@ int bd_get_device_status(void* stream) {
   return BD_OK;
 }
 
+int bd_selftest_timeout(void* stream) {
+  DevCtx* ctx = nullptr;
+  int rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  return cuda_status(bd::launch_timeout_selftest(ctx->status, static_cast<cudaStream_t>(stream)));
+}
+
 int bd_shutdown(void) {
   std::lock_guard<std::mutex> lk(g_mu);
   int cur = 0;

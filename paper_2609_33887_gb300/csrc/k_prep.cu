@@ -171,36 +171,44 @@ __device__ __forceinline__ uint32_t e4m3x2_to_bf16x2(uint16_t two) {
   return *reinterpret_cast<uint32_t*>(&b);
 }
 
+// One warp per row (grid-stride over rows). The row is cut into 8-element
+// chunks; lane l takes chunks l, l + 32, ..., so every warp load reads 256
+// contiguous code bytes and every warp store writes 512 contiguous output
+// bytes; four chunks per lane are in flight at once. No index needs a division.
 __global__ void __launch_bounds__(256) dequant_e4m3_kernel(const uint8_t* __restrict__ w, int64_t ldw, int V, int d,
                                                            __nv_bfloat16* __restrict__ out, int64_t ldo) {
-  // one thread per 16 codes of a row; rows are 16-byte aligned (ldw % 16 == 0)
-  const int per_row = (d + 15) / 16;
-  const int64_t total = static_cast<int64_t>(V) * per_row;
-  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int v = static_cast<int>(t / per_row);
-    const int c0 = static_cast<int>(t % per_row) * 16;
-    const uint8_t* src = w + static_cast<int64_t>(v) * ldw + c0;
-    __nv_bfloat16* dst = out + static_cast<int64_t>(v) * ldo + c0;
-    if (c0 + 16 <= d) {
-      uint4 q = __ldg(reinterpret_cast<const uint4*>(src));
-      const uint16_t* q2 = reinterpret_cast<const uint16_t*>(&q);
-      uint4 o0, o1;
-      o0.x = e4m3x2_to_bf16x2(q2[0]);
-      o0.y = e4m3x2_to_bf16x2(q2[1]);
-      o0.z = e4m3x2_to_bf16x2(q2[2]);
-      o0.w = e4m3x2_to_bf16x2(q2[3]);
-      o1.x = e4m3x2_to_bf16x2(q2[4]);
-      o1.y = e4m3x2_to_bf16x2(q2[5]);
-      o1.z = e4m3x2_to_bf16x2(q2[6]);
-      o1.w = e4m3x2_to_bf16x2(q2[7]);
-      // ldo % 8 == 0 and c0 % 16 == 0 keep both stores 16-byte aligned
-      reinterpret_cast<uint4*>(dst)[0] = o0;
-      reinterpret_cast<uint4*>(dst)[1] = o1;
-    } else {
-      for (int i = 0; c0 + i < d; ++i) {
-        uint32_t b2 = e4m3x2_to_bf16x2(static_cast<uint16_t>(src[i]));
-        dst[i] = *reinterpret_cast<__nv_bfloat16*>(&b2);
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  const int nchunk = (d + 7) / 8;
+  for (int v = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); v < V; v += warps) {
+    const uint8_t* src_row = w + static_cast<int64_t>(v) * ldw;
+    __nv_bfloat16* dst_row = out + static_cast<int64_t>(v) * ldo;
+    for (int c0 = lane; c0 < nchunk; c0 += 128) {
+      uint2 q[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + 32 * u;
+        // 8 codes at 8c: inside the row (ldw % 16 == 0 and ldw >= d)
+        if (c < nchunk) q[u] = __ldg(reinterpret_cast<const uint2*>(src_row + 8 * c));
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + 32 * u;
+        if (c >= nchunk) break;
+        uint4 o;
+        o.x = e4m3x2_to_bf16x2(static_cast<uint16_t>(q[u].x & 0xFFFFu));
+        o.y = e4m3x2_to_bf16x2(static_cast<uint16_t>(q[u].x >> 16));
+        o.z = e4m3x2_to_bf16x2(static_cast<uint16_t>(q[u].y & 0xFFFFu));
+        o.w = e4m3x2_to_bf16x2(static_cast<uint16_t>(q[u].y >> 16));
+        __nv_bfloat16* dst = dst_row + 8 * c;
+        if (8 * c + 8 <= d) {
+          *reinterpret_cast<uint4*>(dst) = o;  // ldo % 8 == 0: 16-byte aligned
+        } else {
+          const __nv_bfloat16* ov = reinterpret_cast<const __nv_bfloat16*>(&o);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (8 * c + j < d) dst[j] = ov[j];
+        }
       }
     }
   }
@@ -208,7 +216,7 @@ __global__ void __launch_bounds__(256) dequant_e4m3_kernel(const uint8_t* __rest
 
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo, int sm_count,
                                 cudaStream_t st) {
-  int grid = sm_count * 16;
+  int grid = sm_count * 8;
   dequant_e4m3_kernel<<<grid, 256, 0, st>>>(w, ldw, V, d, static_cast<__nv_bfloat16*>(out), ldo);
   return cudaGetLastError();
 }
@@ -232,40 +240,62 @@ __device__ __forceinline__ float e4m3_value(uint8_t c) {
   return __half2float(__ushort_as_half(static_cast<unsigned short>(h2 & 0xffffu)));
 }
 
+// One warp per row (grid-stride over rows). The row is cut into 8-element
+// chunks (4 code bytes, 16 output bytes); lane l takes chunks l, l + 32, ...,
+// so every warp load reads 128 contiguous code bytes and every warp store
+// writes 512 contiguous output bytes; four chunks per lane are in flight at
+// once. Chunk c uses block scale c / 2. No index needs a division.
 __global__ void __launch_bounds__(256) dequant_nvfp4_kernel(const uint8_t* __restrict__ codes, int64_t ldw,
                                                             const uint8_t* __restrict__ bs, int64_t ldbs, int V,
                                                             int d, __nv_bfloat16* __restrict__ out, int64_t ldo) {
-  // one thread per 16-element block: 8 code bytes (8-byte aligned: ldw % 16 == 0)
-  const int nblk = (d + 15) / 16;
-  const int64_t total = static_cast<int64_t>(V) * nblk;
-  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < total;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int v = static_cast<int>(t / nblk);
-    const int b = static_cast<int>(t % nblk);
-    const int k0 = b * 16;
-    const uint2 q = __ldg(reinterpret_cast<const uint2*>(codes + static_cast<int64_t>(v) * ldw + k0 / 2));
-    const float sc = e4m3_value(bs[static_cast<int64_t>(v) * ldbs + b]);
-    __nv_bfloat16 o[16];
+  const int lane = threadIdx.x & 31;
+  const int warps = gridDim.x * (blockDim.x >> 5);
+  const int nchunk = (d + 7) / 8;
+  for (int v = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); v < V; v += warps) {
+    const uint8_t* crow = codes + static_cast<int64_t>(v) * ldw;
+    const uint8_t* brow = bs + static_cast<int64_t>(v) * ldbs;
+    __nv_bfloat16* orow = out + static_cast<int64_t>(v) * ldo;
+    for (int c0 = lane; c0 < nchunk; c0 += 128) {
+      uint32_t q[4];
+      uint8_t sb[4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const uint32_t byte = ((j < 4 ? q.x : q.y) >> (8 * (j & 3))) & 0xFFu;
-      o[2 * j] = __float2bfloat16_rn(e2m1_value(byte & 0xFu) * sc);
-      o[2 * j + 1] = __float2bfloat16_rn(e2m1_value(byte >> 4) * sc);
-    }
-    __nv_bfloat16* dst = out + static_cast<int64_t>(v) * ldo + k0;
-    if (k0 + 16 <= d) {
-      // ldo % 8 == 0 and k0 % 16 == 0 keep both stores 16-byte aligned
-      reinterpret_cast<uint4*>(dst)[0] = *reinterpret_cast<const uint4*>(&o[0]);
-      reinterpret_cast<uint4*>(dst)[1] = *reinterpret_cast<const uint4*>(&o[8]);
-    } else {
-      for (int j = 0; k0 + j < d; ++j) dst[j] = o[j];
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + 32 * u;
+        // 4 code bytes at 4c: inside the row (ldw % 16 == 0 and ldw >= ceil(d / 2))
+        if (c < nchunk) {
+          q[u] = __ldg(reinterpret_cast<const uint32_t*>(crow + 4 * c));
+          sb[u] = brow[c >> 1];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = c0 + 32 * u;
+        if (c >= nchunk) break;
+        const float sc = e4m3_value(sb[u]);
+        uint32_t ow[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const uint32_t byte = (q[u] >> (8 * j)) & 0xFFu;
+          __nv_bfloat162 pr = __floats2bfloat162_rn(e2m1_value(byte & 0xFu) * sc, e2m1_value(byte >> 4) * sc);
+          ow[j] = *reinterpret_cast<uint32_t*>(&pr);
+        }
+        __nv_bfloat16* dst = orow + 8 * c;
+        if (8 * c + 8 <= d) {
+          *reinterpret_cast<uint4*>(dst) = make_uint4(ow[0], ow[1], ow[2], ow[3]);  // ldo % 8 == 0
+        } else {
+          const __nv_bfloat16* ov = reinterpret_cast<const __nv_bfloat16*>(ow);
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (8 * c + j < d) dst[j] = ov[j];
+        }
+      }
     }
   }
 }
 
 cudaError_t launch_dequant_nvfp4(const uint8_t* codes, int64_t ldw, const uint8_t* bs, int64_t ldbs, int V, int d,
                                  void* out, int64_t ldo, int sm_count, cudaStream_t st) {
-  int grid = sm_count * 16;
+  int grid = sm_count * 8;
   dequant_nvfp4_kernel<<<grid, 256, 0, st>>>(codes, ldw, bs, ldbs, V, d, static_cast<__nv_bfloat16*>(out), ldo);
   return cudaGetLastError();
 }

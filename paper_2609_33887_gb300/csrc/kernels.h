@@ -145,4 +145,8 @@ struct VerifyArgs {
 };
 cudaError_t launch_merge_verify(const VerifyArgs& a, cudaStream_t st);
 
+// One CTA that runs the bounded mbarrier wait on a barrier nothing completes
+// (failure-detection self-test): sets DEV_TIMEOUT in *status after the limit.
+cudaError_t launch_timeout_selftest(uint32_t* status, cudaStream_t st);
+
 }  // namespace bd

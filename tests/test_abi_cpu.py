@@ -38,7 +38,7 @@ def declared_functions():
 
 def test_header_declares_the_abi():
     assert declared_functions() == sorted([
-        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status",
+        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status", "bd_selftest_timeout",
         "bd_shutdown",
         "bd_status_string", "bd_version", "bd_workspace_size", "bd_verify_step", "bd_verify_workspace_size",
         "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
