@@ -44,7 +44,7 @@ constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
 constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
 constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns
 constexpr int EPI_WARPS = 4;
-constexpr int TR = 33;  // padded row of the transpose buffers
+constexpr int TR = 34;  // padded row of the transpose buffers: 8-byte aligned rows, conflict-free column reads
 constexpr int MAX_CHUNKS = 8;
 
 struct PairCtl {
@@ -290,14 +290,26 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         const int vrow0 = vt * 256 + static_cast<int>(rank) * 128 + quarter * 32;  // vocabulary row of lane 0
         const int my_v = vrow0 + lane;
         const bool dead = my_v >= a.V || my_v == a.mask_id;
-        const float sc = (a.wscale != nullptr && !dead) ? __ldg(a.wscale + my_v) : 1.f;
+        const bool scaled = a.wscale != nullptr;
+        const float sc = (scaled && !dead) ? __ldg(a.wscale + my_v) : 1.f;
 #pragma unroll
         for (int c = 0; c < MAX_CHUNKS; ++c) {
           if (c < nch) {
             float v[32];
             tmem_ld32(tmem_base + lane_addr + acc * 256 + c * 32, v);
+            // this lane's row of the transpose, two floats per store; the mask
+            // entry and rows past V are -inf, the e4m3 row scale applies to live rows
+            float2* row = reinterpret_cast<float2*>(tr + lane * TR);
+            if (dead) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) tr[lane * TR + j] = dead ? -INFINITY : v[j] * sc;
+              for (int j = 0; j < 16; ++j) row[j] = make_float2(-INFINITY, -INFINITY);
+            } else if (scaled) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) row[j] = make_float2(v[2 * j] * sc, v[2 * j + 1] * sc);
+            } else {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) row[j] = make_float2(v[2 * j], v[2 * j + 1]);
+            }
             __syncwarp();
             float x[32];
 #pragma unroll
