@@ -105,6 +105,49 @@ int64_t round_up(int64_t x, int64_t a) { return (x + a - 1) / a * a; }
 
 int env_int(const char* name, int dflt, int lo, int hi);
 
+// Checks shared by every entry point that runs the LM head: the head and the
+// `rows` hidden rows, their dtypes and alignment, and the kernel choice. Fills
+// the head fields of *c (d, V, dtypes, tc / pair, leading dimensions).
+int check_head(const bd_hidden* h, const bd_weight* w, int64_t rows, int variant, Call* c) {
+  if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
+  if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
+  if (h->ld < h->cols || w->ld < (w->dtype == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim)) return BD_ERR_SHAPE;
+  const int hdt = h->dtype, wdt = w->dtype;
+  const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
+  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3 || wdt == BD_NVFP4);
+  if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
+  const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
+  if (tc && !combo_bf16) return BD_ERR_DTYPE;
+  if (rows > 0) {
+    if (!h->data || !w->data) return BD_ERR_NULL;
+    if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
+    if (wdt == BD_NVFP4 && !w->block_scale) return BD_ERR_NULL;
+  }
+  if (tc) {
+    if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
+    if (!aligned(w->data, 16) || (w->ld * esize(wdt)) % 16 != 0) return BD_ERR_ALIGN;
+  } else {
+    if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
+  }
+  if (w->scale && (wdt == BD_E4M3 || wdt == BD_NVFP4) && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
+  if (wdt == BD_NVFP4 && w->block_ld < (w->dim + 15) / 16) return BD_ERR_SHAPE;
+  c->d = w->dim;
+  c->V = w->vocab;
+  c->hdt = hdt;
+  c->wdt = wdt;
+  c->tc = tc;
+  // automatic choice: the CTA-pair kernel (vocabulary on M, token dimension
+  // padded only to a multiple of 32) wins while the window is small; at large
+  // windows both kernels saturate the tensor pipe under the power cap and the
+  // one-CTA kernel runs slightly faster
+  c->pair = tc && (variant == 3 || (variant == 0 && rows <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
+  c->ldh = h->ld;
+  c->ldw = w->ld;
+  c->ldc = round_up(c->d, 8);
+  c->ldq = round_up(c->d, 8);
+  return BD_OK;
+}
+
 int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, const bd_tau_grid* tg,
                int variant, Call* c) {
   if (!h || !w || !ms || !tg) return BD_ERR_NULL;
@@ -118,52 +161,17 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   const int64_t P = n_blocks * ms->block_len;
   if (P > MAX_POSITIONS) return BD_ERR_SHAPE;
   if (h->rows != P) return BD_ERR_SHAPE;
-  if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
-  if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
-  if (h->ld < h->cols || w->ld < (w->dtype == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim)) return BD_ERR_SHAPE;
+  if (const int rc = check_head(h, w, P, variant, c)) return rc;
   if (ms->mask_token_id < -1 || ms->mask_token_id >= w->vocab) return BD_ERR_ARG;
   if (ms->mask_token_id >= 0 && w->vocab < 2) return BD_ERR_SHAPE;  // nothing left to predict
-  const int hdt = h->dtype, wdt = w->dtype;
-  const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
-  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3 || wdt == BD_NVFP4);
-  if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
-  const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
-  if (tc && !combo_bf16) return BD_ERR_DTYPE;
-  if (P > 0) {
-    if (!h->data || !w->data || !ms->pos_masked || !ms->block_flags) return BD_ERR_NULL;
-    if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
-    if (wdt == BD_NVFP4 && !w->block_scale) return BD_ERR_NULL;
-  }
-  if (tc) {
-    if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
-    if (!aligned(w->data, 16) || (w->ld * esize(wdt)) % 16 != 0) return BD_ERR_ALIGN;
-  } else {
-    if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
-  }
-  if (w->scale && (wdt == BD_E4M3 || wdt == BD_NVFP4) && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
-  if (wdt == BD_NVFP4 && w->block_ld < (w->dim + 15) / 16) return BD_ERR_SHAPE;
+  if (P > 0 && (!ms->pos_masked || !ms->block_flags)) return BD_ERR_NULL;
   c->P = P;
-  c->d = w->dim;
-  c->V = w->vocab;
   c->n_seq = ms->n_seq;
   c->n_slots = ms->n_slots;
   c->L = ms->block_len;
   c->n_blocks = static_cast<int>(n_blocks);
   c->mask_id = ms->mask_token_id;
   c->T = tg->T;
-  c->hdt = hdt;
-  c->wdt = wdt;
-  c->tc = tc;
-  // automatic choice: the CTA-pair kernel (vocabulary on M, token dimension
-  // padded only to a multiple of 32) wins while the window is small; at large
-  // windows both kernels saturate the tensor pipe under the power cap and the
-  // one-CTA kernel runs slightly faster
-  c->pair = tc && (variant == 3 || (variant == 0 && P <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
-
-  c->ldh = h->ld;
-  c->ldw = w->ld;
-  c->ldc = round_up(c->d, 8);
-  c->ldq = round_up(c->d, 8);
   return BD_OK;
 }
 
@@ -258,67 +266,62 @@ int cuda_status(cudaError_t e) {
 }
 
 
-// The launch sequence of one commit step (a0..a4) on `st`, working in `ws`
-// laid out by `lay`; kernel timeouts are reported in `status`.
-int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws, uint32_t* status, int sm_count,
-             const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
-             const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
-             int32_t* out_counts, void* ev_begin, void* ev_end, cudaStream_t st) {
-  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
-  int* idx = reinterpret_cast<int*>(ws + lay.idx);
-  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
-  float* pm = reinterpret_cast<float*>(ws + lay.pm);
-  float* ps = reinterpret_cast<float*>(ws + lay.ps);
-  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+// Partial-slot arrays of the LM head; t and x only on the verification path.
+struct Partials {
+  float* m;
+  float* s;
+  int* a;
+  float* t;
+  float* x;
+};
+
+// a1 + a2: decodes an FP8 / NVFP4 head if needed, builds the tensor maps over
+// `rows` (the packed rows of the commit step, or the caller's rows for
+// verification) and launches the LM-head kernel the plan chose, between the
+// optional timing events. The SIMT kernel reads hidden->data through idx.
+int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, const bd_weight* weight,
+                  const void* rows, int64_t ld_rows, void* wq, const int* idx, const int* n_rows,
+                  const int* draft_row, const Partials& part, uint32_t* status, int sm_count, void* ev_begin,
+                  void* ev_end, cudaStream_t st) {
   const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
-
-  if (out_counts) {
-    if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
-      return BD_ERR_CUDA;
-  }
-
-  // a0: compaction of the masked positions of active blocks (+ packing of their rows)
-  int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
-                                            c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
-                                            c.ldc, idx, rowpos, n_rows, sm_count, st));
-  if (rc != BD_OK) return rc;
-
+  const float* wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
   CUtensorMap tmA, tmB;
   bd::PairTokenMaps tmTok;
   if (c.tc) {
-    void* hc = ws + lay.hc;
     const void* wsrc = weight->data;
     int64_t wld = c.ldw;
     if (decoded_head(c)) {
-      rc = decode_head(c, weight, ws + lay.wq, sm_count, st, &wsrc, &wld);
+      const int rc = decode_head(c, weight, wq, sm_count, st, &wsrc, &wld);
       if (rc != BD_OK) return rc;
     }
     if (c.pair) {
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
       for (int i = 0; i < 8; ++i)
-        if (!encode_bf16_2d(&tmTok.m[i], hc, c.d, c.P, c.ldc, 64, 16 * (i + 1))) return BD_ERR_CUDA;
+        if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 16 * (i + 1))) return BD_ERR_CUDA;
       if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
     } else {
-      if (!encode_bf16_2d(&tmA, hc, c.d, c.P, c.ldc, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
+      if (!encode_bf16_2d(&tmA, rows, c.d, c.P, ld_rows, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
       if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
     }
   }
-
-  // a1 + a2: LM head with the online softmax epilogue
   if (ev_begin && record_event(ev_begin, st) != cudaSuccess) return BD_ERR_CUDA;
+  int rc;
   if (c.tc) {
     bd::TcArgs a;
     a.n_rows = n_rows;
-    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
+    a.wscale = wscale;
     a.V = V;
     a.d = d;
     a.P = P;
     a.mask_id = c.mask_id;
     a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
+    a.part_m = part.m;
+    a.part_s = part.s;
+    a.part_a = part.a;
     a.status = status;
+    a.draft_row = draft_row;
+    a.part_t = part.t;
+    a.part_x = part.x;
     rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, a, st))
                 : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
   } else {
@@ -331,7 +334,7 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
     a.wdtype = c.wdt;
     a.wbs = weight->block_scale;
     a.ldbs = weight->block_ld;
-    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
+    a.wscale = wscale;
     a.idx = idx;
     a.n_rows = n_rows;
     a.V = V;
@@ -339,13 +342,47 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
     a.P = P;
     a.mask_id = c.mask_id;
     a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
+    a.part_m = part.m;
+    a.part_s = part.s;
+    a.part_a = part.a;
+    a.draft_row = draft_row;
+    a.part_t = part.t;
+    a.part_x = part.x;
     rc = cuda_status(bd::launch_lmhead_simt(a, st));
   }
   if (rc != BD_OK) return rc;
   if (ev_end && record_event(ev_end, st) != cudaSuccess) return BD_ERR_CUDA;
+  return BD_OK;
+}
+
+// The launch sequence of one commit step (a0..a4) on `st`, working in `ws`
+// laid out by `lay`; kernel timeouts are reported in `status`.
+int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws, uint32_t* status, int sm_count,
+             const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+             const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+             int32_t* out_counts, void* ev_begin, void* ev_end, cudaStream_t st) {
+  int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
+  int* idx = reinterpret_cast<int*>(ws + lay.idx);
+  int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
+  float* pm = reinterpret_cast<float*>(ws + lay.pm);
+  float* ps = reinterpret_cast<float*>(ws + lay.ps);
+  int* pa = reinterpret_cast<int*>(ws + lay.pa);
+  const int P = static_cast<int>(c.P), d = static_cast<int>(c.d);
+
+  if (out_counts) {
+    if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
+      return BD_ERR_CUDA;
+  }
+
+  // a0: compaction of the masked positions of active blocks (+ packing of their rows)
+  int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
+                                            c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
+                                            c.ldc, idx, rowpos, n_rows, sm_count, st));
+  if (rc != BD_OK) return rc;
+
+  rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, c.ldc, ws + lay.wq, idx, n_rows, nullptr,
+                     Partials{pm, ps, pa, nullptr, nullptr}, status, sm_count, ev_begin, ev_end, st);
+  if (rc != BD_OK) return rc;
 
   // a3 + a4: merge and the multi-threshold commit
   bd::CommitArgs ca;
@@ -601,48 +638,19 @@ int check_verify(const bd_hidden* h, const bd_weight* w, const bd_draft* dr, con
   if (dr->n_req < 0 || dr->n_draft < 1 || dr->n_draft > 32) return BD_ERR_SHAPE;
   const int64_t R = int64_t(dr->n_req) * (dr->n_draft + 1);
   if (R > MAX_POSITIONS || h->rows != R) return BD_ERR_SHAPE;
-  if (w->vocab < 1 || w->vocab > MAX_VOCAB) return BD_ERR_SHAPE;
-  if (w->dim < 1 || w->dim > MAX_DIM || h->cols != w->dim) return BD_ERR_SHAPE;
-  if (h->ld < h->cols || w->ld < (w->dtype == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim)) return BD_ERR_SHAPE;
-  const int hdt = h->dtype, wdt = w->dtype;
-  const bool combo_f32 = hdt == BD_F32 && wdt == BD_F32;
-  const bool combo_bf16 = hdt == BD_BF16 && (wdt == BD_BF16 || wdt == BD_E4M3 || wdt == BD_NVFP4);
-  if (!combo_f32 && !combo_bf16) return BD_ERR_DTYPE;
-  const bool tc = variant >= 2 || (variant == 0 && combo_bf16);
-  if (tc && !combo_bf16) return BD_ERR_DTYPE;
-  if (R > 0) {
-    if (!h->data || !w->data || !dr->draft) return BD_ERR_NULL;
-    if (wdt == BD_E4M3 && !w->scale) return BD_ERR_NULL;
-    if (wdt == BD_NVFP4 && !w->block_scale) return BD_ERR_NULL;
-    if (!aligned(dr->draft, 4)) return BD_ERR_ALIGN;
-  }
-  if (tc) {
-    if (!aligned(h->data, 16) || (h->ld * 2) % 16 != 0) return BD_ERR_ALIGN;
-    if (!aligned(w->data, 16) || (w->ld * esize(wdt)) % 16 != 0) return BD_ERR_ALIGN;
-  } else {
-    if (!aligned(h->data, esize(hdt)) || !aligned(w->data, esize(wdt))) return BD_ERR_ALIGN;
-  }
-  if (w->scale && (wdt == BD_E4M3 || wdt == BD_NVFP4) && !aligned(w->scale, 4)) return BD_ERR_ALIGN;
-  if (wdt == BD_NVFP4 && w->block_ld < (w->dim + 15) / 16) return BD_ERR_SHAPE;
   Call& c = vc->c;
   c = Call{};
+  if (const int rc = check_head(h, w, R, variant, &c)) return rc;
+  if (R > 0 && !dr->draft) return BD_ERR_NULL;
+  if (R > 0 && !aligned(dr->draft, 4)) return BD_ERR_ALIGN;
   c.P = R;
-  c.d = w->dim;
-  c.V = w->vocab;
   c.n_seq = dr->n_req;
   c.n_slots = 1;
   c.L = dr->n_draft + 1;
   c.n_blocks = dr->n_req;
   c.mask_id = -1;  // the target's full distribution
   c.T = eg->E;
-  c.hdt = hdt;
-  c.wdt = wdt;
-  c.tc = tc;
-  c.pair = tc && (variant == 3 || (variant == 0 && R <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
-  c.ldh = h->ld;
-  c.ldw = w->ld;
   c.ldc = h->ld;  // the rows are read in place
-  c.ldq = round_up(c.d, 8);
   vc->n_req = dr->n_req;
   vc->n_draft = dr->n_draft;
   return BD_OK;
@@ -689,77 +697,14 @@ int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& l
   int* pa = reinterpret_cast<int*>(ws + lay.pa);
   float* pt = reinterpret_cast<float*>(ws + lay.pt);
   float* px = reinterpret_cast<float*>(ws + lay.px);
-  const int R = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
+  const int R = static_cast<int>(c.P);
 
   int rc = cuda_status(bd::launch_prep_verify(draft->draft, vc.n_req, vc.n_draft, idx, draft_row, n_rows, st));
   if (rc != BD_OK) return rc;
 
-  CUtensorMap tmA, tmB;
-  bd::PairTokenMaps tmTok;
-  if (c.tc) {
-    const void* wsrc = weight->data;
-    int64_t wld = c.ldw;
-    if (decoded_head(c)) {
-      rc = decode_head(c, weight, ws + lay.wq, sm_count, st, &wsrc, &wld);
-      if (rc != BD_OK) return rc;
-    }
-    if (c.pair) {
-      for (int i = 0; i < 8; ++i)
-        if (!encode_bf16_2d(&tmTok.m[i], hidden->data, c.d, c.P, c.ldh, 64, 16 * (i + 1))) return BD_ERR_CUDA;
-      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
-    } else {
-      if (!encode_bf16_2d(&tmA, hidden->data, c.d, c.P, c.ldh, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
-      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
-    }
-  }
-
-  if (ev_begin && record_event(ev_begin, st) != cudaSuccess) return BD_ERR_CUDA;
-  if (c.tc) {
-    bd::TcArgs a;
-    a.n_rows = n_rows;
-    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
-    a.V = V;
-    a.d = d;
-    a.P = R;
-    a.mask_id = -1;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    a.status = status;
-    a.draft_row = draft_row;
-    a.part_t = pt;
-    a.part_x = px;
-    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, a, st))
-                : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
-  } else {
-    bd::SimtArgs a;
-    a.hidden = hidden->data;
-    a.ldh = c.ldh;
-    a.hdtype = c.hdt;
-    a.w = weight->data;
-    a.ldw = c.ldw;
-    a.wdtype = c.wdt;
-    a.wbs = weight->block_scale;
-    a.ldbs = weight->block_ld;
-    a.wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
-    a.idx = idx;
-    a.n_rows = n_rows;
-    a.V = V;
-    a.d = d;
-    a.P = R;
-    a.mask_id = -1;
-    a.plan = plan;
-    a.part_m = pm;
-    a.part_s = ps;
-    a.part_a = pa;
-    a.draft_row = draft_row;
-    a.part_t = pt;
-    a.part_x = px;
-    rc = cuda_status(bd::launch_lmhead_simt(a, st));
-  }
+  rc = launch_lmhead(c, plan, hidden, weight, hidden->data, c.ldh, ws + lay.wq, idx, n_rows, draft_row,
+                     Partials{pm, ps, pa, pt, px}, status, sm_count, ev_begin, ev_end, st);
   if (rc != BD_OK) return rc;
-  if (ev_end && record_event(ev_end, st) != cudaSuccess) return BD_ERR_CUDA;
 
   bd::VerifyArgs va;
   va.draft_row = draft_row;
