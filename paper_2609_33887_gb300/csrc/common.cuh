@@ -263,6 +263,21 @@ __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, vo
   }
 }
 
+// True in exactly one lane of a converged warp (elect.sync). A role that
+// issues asynchronous work (TMA copies, MMAs, commits) runs its loop in the
+// whole warp, with warp-uniform barrier waits, and lets the elected lane
+// issue: a single divergent lane that waits and issues pays a much larger
+// per-instruction issue cost.
+__device__ __forceinline__ bool elect_one() {
+  uint32_t pred;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "elect.sync _|p, 0xffffffff;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(pred));
+  return pred != 0;
+}
+
 // Bounded wait that ignores the abort flag (used only to drain work in flight
 // before the CTA exits).
 __device__ __forceinline__ bool mbar_drain(uint32_t bar, uint32_t parity) {

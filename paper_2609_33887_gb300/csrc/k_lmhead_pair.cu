@@ -23,8 +23,10 @@
 // combined once per unit, and each CTA writes its own partial per token.
 //
 // CTA layout (192 threads): warp 0 TMA producer, warp 1 TMEM allocation (both
-// CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue. Every wait is
-// bounded (see common.cuh).
+// CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue. The producer and
+// issuer loops run in the whole warp and one elected lane issues, which keeps
+// the MMA issue rate at the tensor pipe's rate (N = 160: 80 cycles per MMA).
+// Every wait is bounded (see common.cuh).
 //
 // The verification instantiation (VERIFY = true, speculative decoding) also
 // carries, per token, the entropy accumulator sum exp(l - m) (l - m) log2(e)
@@ -160,24 +162,26 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      const uint64_t pol_w = policy_evict_first();  // head rows: streamed
-      const uint64_t pol_h = policy_evict_last();   // token rows: re-read for every v-tile
-      const uint32_t full0_leader = mapa_shared(smem_u32(&ctl->full[0]), 0);
-      uint32_t stage = 0, phase = 0;
-      uint32_t issued_mask = 0, issued_phase = 0;
-      TileIter it;
-      it.init(a.plan, n_rows, pair);
-      bool ok = true;
-      while (ok && it.next_unit()) {
-        const int tok0 = it.m_tile * NT + static_cast<int>(rank) * half;
-        for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
-          const int vrow = vt * 256 + static_cast<int>(rank) * 128;
-          for (int kb = 0; kb < nk; ++kb) {
-            if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
-              ok = false;
-              break;
-            }
+    // the whole warp walks the stages (warp-uniform waits); one lane issues
+    const bool leader = elect_one();
+    const uint64_t pol_w = policy_evict_first();  // head rows: streamed
+    const uint64_t pol_h = policy_evict_last();   // token rows: re-read for every v-tile
+    const uint32_t full0_leader = mapa_shared(smem_u32(&ctl->full[0]), 0);
+    uint32_t stage = 0, phase = 0;
+    uint32_t issued_mask = 0, issued_phase = 0;
+    TileIter it;
+    it.init(a.plan, n_rows, pair);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      const int tok0 = it.m_tile * NT + static_cast<int>(rank) * half;
+      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+        const int vrow = vt * 256 + static_cast<int>(rank) * 128;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait_warp(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          if (leader) {
             if (rank == 0) mbar_expect_tx(smem_u32(&ctl->full[stage]), tx_total);
             const uint32_t fb = full0_leader + 8u * stage;
             const uint32_t sa = smem_base + stage * SB;
@@ -185,24 +189,27 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             tma_load_2d_pair(sa + A_BLOCK, &tmW, fb, kb * BK + 64, vrow, pol_w);
             tma_load_2d_pair(sa + 2 * A_BLOCK, tm_tok, fb, kb * BK, tok0, pol_h);
             tma_load_2d_pair(sa + 2 * A_BLOCK + B_BLOCK, tm_tok, fb, kb * BK + 64, tok0, pol_h);
-            issued_mask |= 1u << stage;
-            issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-            if (++stage == STAGES) {
-              stage = 0;
-              phase ^= 1u;
-            }
+          }
+          __syncwarp();
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
           }
         }
       }
-      // The even CTA's full barriers count both CTAs' bytes: once they have
-      // flipped for the last issue of every stage, no copy is in flight.
-      if (rank == 0)
-        for (int s = 0; s < STAGES; ++s)
-          if (issued_mask & (1u << s)) mbar_drain(smem_u32(&ctl->full[s]), (issued_phase >> s) & 1u);
     }
+    // The even CTA's full barriers count both CTAs' bytes: once they have
+    // flipped for the last issue of every stage, no copy is in flight.
+    if (rank == 0 && leader)
+      for (int s = 0; s < STAGES; ++s)
+        if (issued_mask & (1u << s)) mbar_drain(smem_u32(&ctl->full[s]), (issued_phase >> s) & 1u);
+    __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------ MMA issuer (even CTA)
-    if (rank == 0 && lane == 0) {
+    if (rank == 0) {
+      const bool leader = elect_one();
       const uint32_t idesc = idesc_bf16_f32(256, NT);
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
@@ -211,43 +218,50 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
       bool ok = true;
       while (ok && it.next_unit()) {
         for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
-          if (!mbar_wait(smem_u32(&ctl->tempty[acc]), acc_phase ^ 1u, abort_flag, a.status)) {
+          if (!mbar_wait_warp(smem_u32(&ctl->tempty[acc]), acc_phase ^ 1u, abort_flag, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + acc * 256;
           for (int kb = 0; kb < nk; ++kb) {
-            if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
+            if (!mbar_wait_warp(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            const uint32_t sa = smem_base + stage * SB;
+            if (leader) {
+              const uint32_t sa = smem_base + stage * SB;
 #pragma unroll
-            for (int j = 0; j < 2; ++j) {
-              const uint64_t adesc = sw128_kmajor_desc(sa + j * A_BLOCK);
-              const uint64_t bdesc = sw128_kmajor_desc(sa + 2 * A_BLOCK + j * B_BLOCK);
+              for (int j = 0; j < 2; ++j) {
+                const uint64_t adesc = sw128_kmajor_desc(sa + j * A_BLOCK);
+                const uint64_t bdesc = sw128_kmajor_desc(sa + 2 * A_BLOCK + j * B_BLOCK);
 #pragma unroll
-              for (int k = 0; k < 4; ++k)
-                umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                for (int k = 0; k < 4; ++k)
+                  umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+              }
+              umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), 0x3);
             }
-            umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), 0x3);
+            __syncwarp();
             if (++stage == STAGES) {
               stage = 0;
               phase ^= 1u;
             }
           }
           if (!ok) break;
-          umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
+          if (leader) umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
+          __syncwarp();
           if (++acc == 2) {
             acc = 0;
             acc_phase ^= 1u;
           }
         }
       }
-      umma_commit_pair_mc(smem_u32(&ctl->drain), 0x1);
-      mbar_drain(smem_u32(&ctl->drain), 0);
+      if (leader) {
+        umma_commit_pair_mc(smem_u32(&ctl->drain), 0x1);
+        mbar_drain(smem_u32(&ctl->drain), 0);
+      }
+      __syncwarp();
     }
   } else {
     // ------------------------------------------------------ epilogue

@@ -7,11 +7,13 @@
 // CTA layout (192 threads, one CTA per SM, persistent over the band plan):
 //   warp 0      TMA producer: A (packed hidden rows) and B (head rows) tiles
 //               of 64 columns (128 B, 128-byte swizzle) into a STAGES ring
-//   warp 1      allocates 512 TMEM columns; lane 0 issues tcgen05.mma
+//   warp 1      allocates 512 TMEM columns; an elected lane issues tcgen05.mma
 //               (M=128, N=256, K=16) into one of two 256-column fp32
 //               accumulators, so the epilogue of tile i overlaps tile i+1
 //   warps 2..5  epilogue: warp w reads TMEM lanes 32*(w%4)..+31 (one row per
 //               thread), 32 columns at a time
+// The producer and issuer loops run in the whole warp (warp-uniform waits) and
+// one elected lane issues the copies and MMAs.
 // Every wait is bounded; on timeout the CTA raises DEV_TIMEOUT in the status
 // word, drains its copies and MMAs, frees TMEM and returns.
 // The verification instantiation (VERIFY = true) also carries the entropy
@@ -87,61 +89,67 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer
-    if (lane == 0) {
-      const uint64_t pol_a = policy_evict_last();   // hidden rows: re-read by every part
-      const uint64_t pol_b = policy_evict_first();  // head rows: streamed once per band
-      uint32_t stage = 0, phase = 0;
-      uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / parity of last issue
-      TileIter it;
-      it.init(a.plan, n_rows);
-      bool ok = true;
-      while (ok && it.next_unit()) {
-        for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
-          for (int kb = 0; kb < nk; ++kb) {
-            if (!mbar_wait(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
-              ok = false;
-              break;
-            }
+    // the whole warp walks the stages (warp-uniform waits); one lane issues
+    const bool leader = elect_one();
+    const uint64_t pol_a = policy_evict_last();   // hidden rows: re-read by every part
+    const uint64_t pol_b = policy_evict_first();  // head rows: streamed once per band
+    uint32_t stage = 0, phase = 0;
+    uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / parity of last issue
+    TileIter it;
+    it.init(a.plan, n_rows);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait_warp(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          if (leader) {
             const uint32_t fb = smem_u32(&ctl->full[stage]);
             mbar_expect_tx(fb, STAGE_BYTES);
             const uint32_t sa = smem_base + stage * STAGE_BYTES;
             tma_load_2d(sa, &tmA, fb, kb * BK, it.m_tile * BM, pol_a);
             tma_load_2d(sa + A_BYTES, &tmB, fb, kb * BK, vt * BN, pol_b);
-            issued_mask |= 1u << stage;
-            issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
-            if (++stage == STAGES) {
-              stage = 0;
-              phase ^= 1u;
-            }
+          }
+          __syncwarp();
+          issued_mask |= 1u << stage;
+          issued_phase = (issued_phase & ~(1u << stage)) | (phase << stage);
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
           }
         }
       }
-      // Wait for the last load issued into every stage (immediate unless aborted).
+    }
+    // Wait for the last load issued into every stage (immediate unless aborted).
+    if (leader)
       for (int s = 0; s < STAGES; ++s)
         if (issued_mask & (1u << s)) mbar_drain(smem_u32(&ctl->full[s]), (issued_phase >> s) & 1u);
-    }
+    __syncwarp();
   } else if (warp == 1) {
     // ------------------------------------------------------ MMA issuer
-    if (lane == 0) {
-      uint32_t stage = 0, phase = 0;
-      uint32_t acc = 0, acc_phase = 0;
-      TileIter it;
-      it.init(a.plan, n_rows);
-      bool ok = true;
-      while (ok && it.next_unit()) {
-        for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
-          if (!mbar_wait(smem_u32(&ctl->tempty[acc]), acc_phase ^ 1u, abort_flag, a.status)) {
+    const bool leader = elect_one();
+    uint32_t stage = 0, phase = 0;
+    uint32_t acc = 0, acc_phase = 0;
+    TileIter it;
+    it.init(a.plan, n_rows);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+        if (!mbar_wait_warp(smem_u32(&ctl->tempty[acc]), acc_phase ^ 1u, abort_flag, a.status)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + acc * BN;
+        for (int kb = 0; kb < nk; ++kb) {
+          if (!mbar_wait_warp(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + acc * BN;
-          for (int kb = 0; kb < nk; ++kb) {
-            if (!mbar_wait(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
+          if (leader) {
             const uint32_t sa = smem_base + stage * STAGE_BYTES;
             const uint64_t adesc = sw128_kmajor_desc(sa);
             const uint64_t bdesc = sw128_kmajor_desc(sa + A_BYTES);
@@ -151,23 +159,28 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, IDESC, (kb | k) != 0);
             }
             umma_commit(smem_u32(&ctl->empty[stage]));
-            if (++stage == STAGES) {
-              stage = 0;
-              phase ^= 1u;
-            }
           }
-          if (!ok) break;
-          umma_commit(smem_u32(&ctl->tfull[acc]));
-          if (++acc == 2) {
-            acc = 0;
-            acc_phase ^= 1u;
+          __syncwarp();
+          if (++stage == STAGES) {
+            stage = 0;
+            phase ^= 1u;
           }
         }
+        if (!ok) break;
+        if (leader) umma_commit(smem_u32(&ctl->tfull[acc]));
+        __syncwarp();
+        if (++acc == 2) {
+          acc = 0;
+          acc_phase ^= 1u;
+        }
       }
-      // All MMAs issued by this thread have completed once `drain` flips.
+    }
+    // All MMAs issued by the elected thread have completed once `drain` flips.
+    if (leader) {
       umma_commit(smem_u32(&ctl->drain));
       mbar_drain(smem_u32(&ctl->drain), 0);
     }
+    __syncwarp();
   } else {
     // ------------------------------------------------------ epilogue
     const int quarter = warp & 3;
