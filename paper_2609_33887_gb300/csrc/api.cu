@@ -78,13 +78,14 @@ struct Call {
   int64_t ldh, ldw;
   int64_t ldc;      // packed hidden rows (bf16), elements
   int64_t ldq;      // decoded e4m3 head (bf16), elements
+  bool fused;       // pair kernel decodes an E4M3 / NVFP4 head itself (no bf16 copy)
 };
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }  // NVFP4: ld counts bytes
 
-bool decoded_head(const Call& c) { return c.tc && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4); }
+bool decoded_head(const Call& c) { return c.tc && !c.fused && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4); }
 
 // Decodes an FP8 or NVFP4 head into the bf16 workspace copy the tensor-core
 // kernels read (both decodes are exact); wsrc / wld then describe that copy.
@@ -145,6 +146,12 @@ int check_head(const bd_hidden* h, const bd_weight* w, int64_t rows, int variant
   c->ldw = w->ld;
   c->ldc = round_up(c->d, 8);
   c->ldq = round_up(c->d, 8);
+  // the pair kernel reads E4M3 / NVFP4 codes (and block scales) with TMA when
+  // their rows start on 16-byte boundaries; otherwise the head is decoded to a
+  // bf16 copy first
+  c->fused = c->pair && (wdt == BD_E4M3 || wdt == BD_NVFP4) && env_int("BD_FUSED_DECODE", 1, 0, 1) != 0 &&
+             aligned(w->data, 16) && w->ld % 16 == 0 && (wdt == BD_NVFP4 ? (w->dim + 1) / 2 : w->dim) >= 16 &&
+             (wdt != BD_NVFP4 || (aligned(w->block_scale, 16) && w->block_ld % 16 == 0));
   return BD_OK;
 }
 
@@ -247,6 +254,19 @@ bool encode_bf16_2d(CUtensorMap* m, const void* base, int64_t inner, int64_t row
   return r == CUDA_SUCCESS;
 }
 
+// [rows, inner_bytes] bytes with row stride ld_bytes, boxes of box_inner bytes x box_rows.
+bool encode_u8_2d(CUtensorMap* m, const void* base, int64_t inner_bytes, int64_t rows, int64_t ld_bytes,
+                  uint32_t box_inner, uint32_t box_rows, bool swizzle128) {
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner_bytes), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld_bytes)};
+  cuuint32_t box[2] = {box_inner, box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void*>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
 // Records `ev` on `st`. Inside a stream capture a plain record would only add
 // a dependency edge; the external flag makes it an event node of the graph,
 // so replays still time the kernel.
@@ -287,6 +307,18 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
   const float* wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
   CUtensorMap tmA, tmB;
   bd::PairTokenMaps tmTok;
+  bd::PairQuantMaps tmQ;
+  std::memset(&tmB, 0, sizeof(tmB));
+  std::memset(&tmQ, 0, sizeof(tmQ));
+  const int hf = !c.fused ? bd::HF_BF16 : c.wdt == BD_NVFP4 ? bd::HF_NVFP4 : bd::HF_E4M3;
+  if (c.fused) {
+    // codes: 128 bytes of a row per box (128 NVFP4 / E4M3 ... columns of d: 256 / 128)
+    const int64_t code_bytes = c.wdt == BD_NVFP4 ? (c.d + 1) / 2 : c.d;
+    if (!encode_u8_2d(&tmQ.codes, weight->data, code_bytes, c.V, c.ldw, 128, 128, true)) return BD_ERR_CUDA;
+    if (c.wdt == BD_NVFP4 &&
+        !encode_u8_2d(&tmQ.scales, weight->block_scale, (c.d + 15) / 16, c.V, weight->block_ld, 16, 128, false))
+      return BD_ERR_CUDA;
+  }
   if (c.tc) {
     const void* wsrc = weight->data;
     int64_t wld = c.ldw;
@@ -298,7 +330,7 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
       for (int i = 0; i < 8; ++i)
         if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 16 * (i + 1))) return BD_ERR_CUDA;
-      if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
+      if (!c.fused && !encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
     } else {
       if (!encode_bf16_2d(&tmA, rows, c.d, c.P, ld_rows, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
       if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
@@ -322,7 +354,7 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
     a.draft_row = draft_row;
     a.part_t = part.t;
     a.part_x = part.x;
-    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, a, st))
+    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, c.fused ? &tmQ : nullptr, hf, a, st))
                 : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
   } else {
     bd::SimtArgs a;

@@ -32,7 +32,17 @@
 // carries, per token, the entropy accumulator sum exp(l - m) (l - m) log2(e)
 // and the logit of the token's draft entry (typical-acceptance appendix); its
 // larger combine buffers cost shared memory, so it may run one stage fewer.
+//
+// Quantised heads (HF = HF_E4M3, HF_NVFP4: the precision levers) are decoded
+// inside the kernel, so HBM carries the stored head only: a raw-code producer
+// warp streams this CTA's head codes (and NVFP4 block scales) with TMA into a
+// small ring, and four converter warps decode them exactly into the bf16
+// operand tile of the stage, in the tile's 128-byte-swizzled layout. The
+// operand stage is full when both CTAs' converters (eight warp arrivals) and
+// the token rows' transaction bytes have landed. E4M3 raw stages hold 128
+// columns of d, NVFP4 raw stages 256 (128 bytes of codes per row either way).
 #include <atomic>
+#include <cstring>
 
 #include "kernels.h"
 
@@ -40,7 +50,12 @@ namespace bd {
 
 namespace {
 
-constexpr int BK = 128;                  // columns of d per pipeline stage (two 64-column swizzle atoms)
+// columns of d per operand stage: two 64-column swizzle atoms for bf16 heads;
+// one for quantised heads, whose small stages leave room for a deep raw ring
+template <int HF>
+__host__ __device__ constexpr int stage_k() {
+  return HF == HF_BF16 ? 128 : 64;
+}
 constexpr int MAX_STAGES = 8;
 constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
 constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
@@ -48,6 +63,28 @@ constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns
 constexpr int EPI_WARPS = 4;
 constexpr int TR = 34;  // padded row of the transpose buffers: 8-byte aligned rows, conflict-free column reads
 constexpr int MAX_CHUNKS = 8;
+constexpr int MAX_RAW = 8;
+constexpr int QUANT_STAGES = 4;  // operand stages next to the raw ring (quantised heads)
+constexpr int CONV_WARPS = 8;                            // converter warps 6..13 (quantised heads)
+constexpr int CONV_THREADS = CONV_WARPS * 32;
+constexpr int RAW_PRODUCER = 2 + EPI_WARPS + CONV_WARPS;  // warp streaming the quantised codes
+
+template <int HF>
+__host__ __device__ constexpr int pair_threads() {
+  return HF == HF_BF16 ? TC_THREADS : (RAW_PRODUCER + 1) * 32;
+}
+// Raw ring of a quantised head: stages of 128 head rows x 128 bytes of codes
+// (SW128), plus 16 bytes of NVFP4 block scales per row.
+constexpr uint32_t RAW_CODE_BYTES = 128 * 128;
+template <int HF>
+__host__ __device__ constexpr uint32_t raw_bytes() {
+  return HF == HF_NVFP4 ? RAW_CODE_BYTES + 128 * 16 : RAW_CODE_BYTES;
+}
+// operand stages per raw stage (a raw stage holds 256 NVFP4 or 128 E4M3 columns)
+template <int HF>
+__host__ __device__ constexpr int raw_k() {
+  return (HF == HF_NVFP4 ? 256 : 128) / stage_k<HF>();
+}
 
 struct PairCtl {
   uint64_t full[MAX_STAGES];
@@ -56,6 +93,8 @@ struct PairCtl {
   uint64_t tempty[2];
   uint64_t drain;
   uint64_t epi_sync;  // rendezvous of the 128 epilogue threads (bounded, unlike bar.sync)
+  uint64_t rfull[MAX_RAW];   // quantised heads: raw codes landed (TMA transaction bytes)
+  uint64_t rempty[MAX_RAW];  // ... and consumed by the converter warps
   uint32_t tmem_base;
   int abort_flag;
 };
@@ -92,26 +131,115 @@ __host__ __device__ constexpr size_t stage_area() {
   return SMEM_BYTES - 1024 - sizeof(PairTail<VERIFY>);
 }
 
-// Stage layout for a token group of NT rows (NT/2 in each CTA):
-//   [A block 0 | A block 1 | B block 0 | B block 1], A = 128 head rows,
-//   B = NT/2 token rows, each block 64 columns wide and 1 KB aligned.
+// Stage layout for a token group of NT rows (NT/2 in each CTA), one block per
+// 64-column atom: [A block 0 (| A block 1) | B block 0 (| B block 1)],
+// A = 128 head rows, B = NT/2 token rows, each block 1 KB aligned.
+template <int HF>
 __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
-  return 2 * A_BLOCK + 2 * static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES;
+  // quantised heads: one CTA multiplies its 128 head rows by all NT token rows
+  return HF == HF_BF16 ? 2 * (A_BLOCK + static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES)
+                       : A_BLOCK + static_cast<uint32_t>(nt) * ATOM_ROWS_BYTES;
 }
-template <bool VERIFY>
+// Operand stages: as many as fit (at most MAX_STAGES) for bf16 heads; for
+// quantised heads at most QUANT_STAGES next to a raw ring of at least three
+// stages, which takes the rest of the area.
+template <int HF, bool VERIFY>
 __host__ __device__ constexpr int stage_count(int nt) {
-  return static_cast<int>(stage_area<VERIFY>() / stage_bytes(nt)) < MAX_STAGES
-             ? static_cast<int>(stage_area<VERIFY>() / stage_bytes(nt))
+  return HF != HF_BF16
+             ? (static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt)) < QUANT_STAGES
+                    ? static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt))
+                    : QUANT_STAGES)
+         : static_cast<int>(stage_area<VERIFY>() / stage_bytes<HF>(nt)) < MAX_STAGES
+             ? static_cast<int>(stage_area<VERIFY>() / stage_bytes<HF>(nt))
              : MAX_STAGES;
 }
-static_assert(stage_count<false>(256) >= 3 && stage_count<true>(256) >= 3, "three stages at NT = 256");
-static_assert(stage_count<false>(160) == 4, "four stages at NT = 160 on the commit path");
+template <int HF, bool VERIFY>
+__host__ __device__ constexpr int raw_count(int nt) {
+  return HF == HF_BF16 ? 0
+         : static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
+                            raw_bytes<HF>()) < MAX_RAW
+             ? static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
+                                raw_bytes<HF>())
+             : MAX_RAW;
+}
+static_assert(stage_count<HF_BF16, false>(256) >= 3 && stage_count<HF_BF16, true>(256) >= 3, "three stages at NT = 256");
+static_assert(stage_count<HF_BF16, false>(160) == 4, "four stages at NT = 160 on the commit path");
+static_assert(stage_count<HF_NVFP4, false>(160) == 4 && stage_count<HF_E4M3, false>(160) == 4 &&
+                  stage_count<HF_NVFP4, true>(160) == 4 && stage_count<HF_E4M3, true>(160) == 4,
+              "four operand stages at NT = 160 for quantised heads");
+static_assert(stage_count<HF_NVFP4, true>(256) >= 3 && stage_count<HF_E4M3, true>(256) >= 3 &&
+                  raw_count<HF_NVFP4, true>(256) >= 3 && raw_count<HF_E4M3, true>(256) >= 3,
+              "three operand and three raw stages at NT = 256");
+
+// Decodes this thread's share of one operand stage (128 head rows x 64
+// columns, global columns kcol0..) from the raw stage at raw_base into the
+// bf16 A tile at a_base (one SW128 atom). h: which 64-column part of the raw
+// stage. Columns at or past d decode to zero. ct: 0..CONV_THREADS-1.
+template <int HF>
+__device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t a_base, int ct, int kcol0, int d) {
+  static_assert(HF == HF_BF16 || stage_k<HF>() == 64, "one atom per quantised operand stage");
+  if constexpr (HF == HF_NVFP4) {
+#pragma unroll
+    for (int i = 0; i < 256 / CONV_THREADS; ++i) {
+      const int ci = ct + CONV_THREADS * i;
+      const int row = ci >> 1, j = ci & 1;  // 32-column chunk j of the stage
+      const int c = h * 2 + j;              // its 16 bytes of codes within the raw row
+      const uint4 q = ld_shared_v4(raw_base + row * 128 + ((c ^ (row & 7)) << 4));
+      const uint32_t s01 = e4m3x2_to_f16x2(ld_shared_u16(raw_base + RAW_CODE_BYTES + row * 16 + c * 2));
+      const uint32_t sc[2] = {__byte_perm(s01, 0, 0x1010), __byte_perm(s01, 0, 0x3232)};
+      const uint32_t words[4] = {q.x, q.y, q.z, q.w};
+      uint32_t w[16];
+#pragma unroll
+      for (int b = 0; b < 16; ++b)  // byte b: elements 2b (low nibble), 2b + 1; 16 elements per block scale
+        w[b] = f16x2_to_bf16x2(hmul2_u32(e2m1x2_to_f16x2(__byte_perm(words[b >> 2], 0, 0x4440 + (b & 3))), sc[b >> 3]));
+      const int col0 = kcol0 + j * 32;
+      if (col0 + 32 > d) {
+#pragma unroll
+        for (int b = 0; b < 16; ++b) {
+          if (col0 + 2 * b >= d) w[b] = 0u;
+          else if (col0 + 2 * b + 1 >= d) w[b] &= 0xFFFFu;
+        }
+      }
+      const uint32_t rowbase = a_base + row * 128;
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        st_shared_v4(rowbase + (((j * 4 + u) ^ (row & 7)) << 4), w[4 * u], w[4 * u + 1], w[4 * u + 2], w[4 * u + 3]);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 512 / CONV_THREADS; ++i) {
+      const int ci = ct + CONV_THREADS * i;
+      const int row = ci >> 2, j = ci & 3;  // 16-column chunk j of the stage
+      const int c = h * 4 + j;              // its 16 bytes of codes within the raw row
+      const uint4 q = ld_shared_v4(raw_base + row * 128 + ((c ^ (row & 7)) << 4));
+      const uint32_t words[4] = {q.x, q.y, q.z, q.w};
+      uint32_t w[8];
+#pragma unroll
+      for (int b = 0; b < 8; ++b)  // bytes 2b, 2b + 1: elements 2b, 2b + 1
+        w[b] = f16x2_to_bf16x2(e4m3x2_to_f16x2(__byte_perm(words[b >> 1], 0, (b & 1) ? 0x4432 : 0x4410)));
+      const int col0 = kcol0 + j * 16;
+      if (col0 + 16 > d) {
+#pragma unroll
+        for (int b = 0; b < 8; ++b) {
+          if (col0 + 2 * b >= d) w[b] = 0u;
+          else if (col0 + 2 * b + 1 >= d) w[b] &= 0xFFFFu;
+        }
+      }
+      const uint32_t rowbase = a_base + row * 128;
+#pragma unroll
+      for (int u = 0; u < 2; ++u)
+        st_shared_v4(rowbase + (((j * 2 + u) ^ (row & 7)) << 4), w[4 * u], w[4 * u + 1], w[4 * u + 2], w[4 * u + 3]);
+    }
+  }
+}
 
 }  // namespace
 
-template <bool VERIFY>
-__global__ void __launch_bounds__(TC_THREADS, 1)
-    lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW, TcArgs a) {
+template <int HF, bool VERIFY>
+__global__ void __launch_bounds__(pair_threads<HF>(), 1)
+    lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW,
+                       const __grid_constant__ PairQuantMaps tmQ, TcArgs a) {
+  constexpr bool QUANT = HF != HF_BF16;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   PairTail<VERIFY>* tail = reinterpret_cast<PairTail<VERIFY>*>(smem + stage_area<VERIFY>());
@@ -120,18 +248,30 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const uint32_t rank = cluster_ctarank();  // 0: the CTA that issues the MMAs
+  // 0: the CTA that issues the pair's MMAs (bf16 heads); quantised heads: the
+  // half of the v-tile this CTA takes on its own
+  const uint32_t rank = QUANT ? (blockIdx.x & 1u) : cluster_ctarank();
   const int pair = blockIdx.x >> 1;
 
   if (threadIdx.x == 0) {
-    prefetch_tmap(&tmW);
+    if constexpr (QUANT) {
+      prefetch_tmap(&tmQ.codes);
+      if constexpr (HF == HF_NVFP4) prefetch_tmap(&tmQ.scales);
+      for (int r = 0; r < MAX_RAW; ++r) {
+        mbar_init(smem_u32(&ctl->rfull[r]), 1);
+        mbar_init(smem_u32(&ctl->rempty[r]), CONV_WARPS);
+      }
+    } else {
+      prefetch_tmap(&tmW);
+    }
     for (int s = 0; s < MAX_STAGES; ++s) {
-      mbar_init(smem_u32(&ctl->full[s]), 1);
+      // quantised heads: the token bytes' arrival plus the CTA's converter warps
+      mbar_init(smem_u32(&ctl->full[s]), QUANT ? 1 + CONV_WARPS : 1);
       mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&ctl->tfull[i]), 1);
-      mbar_init(smem_u32(&ctl->tempty[i]), 2 * EPI_WARPS);
+      mbar_init(smem_u32(&ctl->tempty[i]), QUANT ? EPI_WARPS : 2 * EPI_WARPS);
     }
     mbar_init(smem_u32(&ctl->drain), 1);
     mbar_init(smem_u32(&ctl->epi_sync), EPI_WARPS * 32);
@@ -139,25 +279,39 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc_pair(smem_u32(&ctl->tmem_base), TMEM_COLS);
-    tmem_relinquish_pair();
+    if constexpr (QUANT) {
+      tmem_alloc(smem_u32(&ctl->tmem_base), TMEM_COLS);
+      tmem_relinquish();
+    } else {
+      tmem_alloc_pair(smem_u32(&ctl->tmem_base), TMEM_COLS);
+      tmem_relinquish_pair();
+    }
   }
   tc_fence_before();
-  cluster_sync_all();  // barriers initialised and TMEM allocated in both CTAs
+  if constexpr (QUANT)
+    __syncthreads();
+  else
+    cluster_sync_all();  // barriers initialised and TMEM allocated in both CTAs
   tc_fence_after();
   const uint32_t tmem_base = ctl->tmem_base;
   volatile int* abort_flag = &ctl->abort_flag;
 
   griddep_wait();  // the packed rows and N come from the preceding kernel
   const int n_rows = *a.n_rows;
+  constexpr int BK = stage_k<HF>();
+  constexpr int NATOM = BK / 64;
   const int nk = cdiv(a.d, BK);
   const int NT = pair_group_rows(n_rows);
   const int half = NT / 2;
   const int nch = NT / 32;
-  const uint32_t SB = stage_bytes(NT);
+  const uint32_t SB = stage_bytes<HF>(NT);
   const uint32_t B_BLOCK = static_cast<uint32_t>(half) * ATOM_ROWS_BYTES;
-  const int STAGES = stage_count<VERIFY>(NT);
-  const uint32_t tx_total = 2u * SB;  // both CTAs' bytes land on the even CTA's barrier
+  const int STAGES = stage_count<HF, VERIFY>(NT);
+  const int RSTAGES = raw_count<HF, VERIFY>(NT);
+  // bf16 heads: both CTAs' bytes land on the even CTA's barrier; quantised
+  // heads: this CTA's token rows only
+  const uint32_t tx_total = QUANT ? static_cast<uint32_t>(NT) * ATOM_ROWS_BYTES : 2u * SB;
+  const uint32_t raw_base = smem_base + static_cast<uint32_t>(STAGES) * SB;  // quantised heads' raw ring
   const CUtensorMap* tm_tok = &tmH.m[half / 16 - 1];  // box of exactly `half` rows
 
   if (warp == 0) {
@@ -173,7 +327,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     it.init(a.plan, n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
-      const int tok0 = it.m_tile * NT + static_cast<int>(rank) * half;
+      const int tok0 = it.m_tile * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
         const int vrow = vt * 256 + static_cast<int>(rank) * 128;
         for (int kb = 0; kb < nk; ++kb) {
@@ -182,13 +336,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             break;
           }
           if (leader) {
-            if (rank == 0) mbar_expect_tx(smem_u32(&ctl->full[stage]), tx_total);
-            const uint32_t fb = full0_leader + 8u * stage;
             const uint32_t sa = smem_base + stage * SB;
-            tma_load_2d_pair(sa, &tmW, fb, kb * BK, vrow, pol_w);
-            tma_load_2d_pair(sa + A_BLOCK, &tmW, fb, kb * BK + 64, vrow, pol_w);
-            tma_load_2d_pair(sa + 2 * A_BLOCK, tm_tok, fb, kb * BK, tok0, pol_h);
-            tma_load_2d_pair(sa + 2 * A_BLOCK + B_BLOCK, tm_tok, fb, kb * BK + 64, tok0, pol_h);
+            if constexpr (QUANT) {
+              // all NT token rows of the group, as two boxes of NT/2 rows
+              const uint32_t fb = smem_u32(&ctl->full[stage]);
+              mbar_expect_tx(fb, tx_total);
+              tma_load_2d(sa + A_BLOCK, tm_tok, fb, kb * BK, tok0, pol_h);
+              tma_load_2d(sa + A_BLOCK + B_BLOCK, tm_tok, fb, kb * BK, tok0 + half, pol_h);
+            } else {
+              if (rank == 0) mbar_expect_tx(smem_u32(&ctl->full[stage]), tx_total);
+              const uint32_t fb = full0_leader + 8u * stage;
+#pragma unroll
+              for (int j = 0; j < NATOM; ++j) {
+                tma_load_2d_pair(sa + j * A_BLOCK, &tmW, fb, kb * BK + 64 * j, vrow, pol_w);
+                tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + 64 * j, tok0, pol_h);
+              }
+            }
           }
           __syncwarp();
           issued_mask |= 1u << stage;
@@ -207,10 +370,10 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         if (issued_mask & (1u << s)) mbar_drain(smem_u32(&ctl->full[s]), (issued_phase >> s) & 1u);
     __syncwarp();
   } else if (warp == 1) {
-    // ------------------------------------------------------ MMA issuer (even CTA)
-    if (rank == 0) {
+    // ------------------------------------------------------ MMA issuer (even CTA; every CTA for quantised heads)
+    if (rank == 0 || QUANT) {
       const bool leader = elect_one();
-      const uint32_t idesc = idesc_bf16_f32(256, NT);
+      const uint32_t idesc = idesc_bf16_f32(QUANT ? 128 : 256, NT);
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
@@ -233,14 +396,21 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             if (leader) {
               const uint32_t sa = smem_base + stage * SB;
 #pragma unroll
-              for (int j = 0; j < 2; ++j) {
+              for (int j = 0; j < NATOM; ++j) {
                 const uint64_t adesc = sw128_kmajor_desc(sa + j * A_BLOCK);
-                const uint64_t bdesc = sw128_kmajor_desc(sa + 2 * A_BLOCK + j * B_BLOCK);
+                const uint64_t bdesc = sw128_kmajor_desc(sa + NATOM * A_BLOCK + j * B_BLOCK);
 #pragma unroll
-                for (int k = 0; k < 4; ++k)
-                  umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                for (int k = 0; k < 4; ++k) {
+                  if constexpr (QUANT)
+                    umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                  else
+                    umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                }
               }
-              umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), 0x3);
+              if constexpr (QUANT)
+                umma_commit(smem_u32(&ctl->empty[stage]));
+              else
+                umma_commit_pair_mc(smem_u32(&ctl->empty[stage]), 0x3);
             }
             __syncwarp();
             if (++stage == STAGES) {
@@ -249,7 +419,12 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
             }
           }
           if (!ok) break;
-          if (leader) umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
+          if (leader) {
+            if constexpr (QUANT)
+              umma_commit(smem_u32(&ctl->tfull[acc]));
+            else
+              umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
+          }
           __syncwarp();
           if (++acc == 2) {
             acc = 0;
@@ -258,10 +433,92 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         }
       }
       if (leader) {
-        umma_commit_pair_mc(smem_u32(&ctl->drain), 0x1);
+        if constexpr (QUANT)
+          umma_commit(smem_u32(&ctl->drain));
+        else
+          umma_commit_pair_mc(smem_u32(&ctl->drain), 0x1);
         mbar_drain(smem_u32(&ctl->drain), 0);
       }
       __syncwarp();
+    }
+  } else if (QUANT && warp == RAW_PRODUCER) {
+    // ------------------------------------------------------ raw-code producer (quantised heads)
+    const bool leader = elect_one();
+    const uint64_t pol = policy_evict_first();
+    const int RS = RSTAGES;
+    const int nkr = cdiv(nk, raw_k<HF>());
+    uint32_t r = 0, rph = 0;
+    uint32_t issued_mask = 0, issued_phase = 0;
+    TileIter it;
+    it.init(a.plan, n_rows, pair);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+        const int vrow = vt * 256 + static_cast<int>(rank) * 128;
+        for (int kr = 0; kr < nkr; ++kr) {
+          if (!mbar_wait_warp(smem_u32(&ctl->rempty[r]), rph ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          if (leader) {
+            const uint32_t fb = smem_u32(&ctl->rfull[r]);
+            const uint32_t dst = raw_base + r * raw_bytes<HF>();
+            mbar_expect_tx(fb, raw_bytes<HF>());
+            tma_load_2d(dst, &tmQ.codes, fb, kr * 128, vrow, pol);
+            if constexpr (HF == HF_NVFP4) tma_load_2d(dst + RAW_CODE_BYTES, &tmQ.scales, fb, kr * 16, vrow, pol);
+          }
+          __syncwarp();
+          issued_mask |= 1u << r;
+          issued_phase = (issued_phase & ~(1u << r)) | (rph << r);
+          if (++r == static_cast<uint32_t>(RS)) {
+            r = 0;
+            rph ^= 1u;
+          }
+        }
+      }
+    }
+    if (leader)
+      for (int q = 0; q < RS; ++q)
+        if (issued_mask & (1u << q)) mbar_drain(smem_u32(&ctl->rfull[q]), (issued_phase >> q) & 1u);
+    __syncwarp();
+  } else if (QUANT && warp >= 2 + EPI_WARPS) {
+    // ------------------------------------------------------ converters (quantised heads)
+    const int ct = threadIdx.x - (2 + EPI_WARPS) * 32;  // 0..CONV_THREADS-1
+    const int RS = RSTAGES;
+    constexpr int RK = raw_k<HF>();
+    uint32_t r = 0, rph = 0, stage = 0, phase = 0;
+    TileIter it;
+    it.init(a.plan, n_rows, pair);
+    bool ok = true;
+    while (ok && it.next_unit()) {
+      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+        for (int kb = 0; kb < nk; ++kb) {
+          const int h = kb % RK;
+          if (h == 0 && !mbar_wait_warp(smem_u32(&ctl->rfull[r]), rph, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          if (!mbar_wait_warp(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
+            ok = false;
+            break;
+          }
+          convert_stage<HF>(raw_base + r * raw_bytes<HF>(), h, smem_base + stage * SB, ct, kb * BK, a.d);
+          fence_proxy_async_smem();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&ctl->full[stage]));
+          if (h == RK - 1 || kb == nk - 1) {
+            if (lane == 0) mbar_arrive(smem_u32(&ctl->rempty[r]));
+            if (++r == static_cast<uint32_t>(RS)) {
+              r = 0;
+              rph ^= 1u;
+            }
+          }
+          if (++stage == static_cast<uint32_t>(STAGES)) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+      }
     }
   } else {
     // ------------------------------------------------------ epilogue
@@ -389,7 +646,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) {
-          if (rank == 0)
+          if (rank == 0 || QUANT)
             mbar_arrive(tempty_local0 + 8u * acc);
           else
             mbar_arrive_cluster(tempty_leader0 + 8u * acc);
@@ -455,14 +712,22 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   __syncwarp();
   griddep_launch_dependents();
   tc_fence_before();
-  cluster_sync_all();  // both CTAs done: no MMA, copy or remote arrival is pending
+  if constexpr (QUANT)
+    __syncthreads();
+  else
+    cluster_sync_all();  // both CTAs done: no MMA, copy or remote arrival is pending
   tc_fence_after();
-  if (warp == 1) tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  if (warp == 1) {
+    if constexpr (QUANT)
+      tmem_dealloc(tmem_base, TMEM_COLS);
+    else
+      tmem_dealloc_pair(tmem_base, TMEM_COLS);
+  }
 }
 
 size_t pair_smem_bytes() { return SMEM_BYTES; }
 
-template <bool VERIFY>
+template <int HF, bool VERIFY>
 static cudaError_t pair_opt_in() {
   static std::atomic<uint64_t> opted_in{0};
   int dev = 0;
@@ -470,7 +735,7 @@ static cudaError_t pair_opt_in() {
   if (e != cudaSuccess) return e;
   const uint64_t bit = 1ull << (dev & 63);
   if ((opted_in.load() & bit) == 0) {
-    e = cudaFuncSetAttribute(lmhead_pair_kernel<VERIFY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    e = cudaFuncSetAttribute(lmhead_pair_kernel<HF, VERIFY>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(SMEM_BYTES));
     if (e != cudaSuccess) return e;
     opted_in.fetch_or(bit);
@@ -478,48 +743,68 @@ static cudaError_t pair_opt_in() {
   return cudaSuccess;
 }
 
-static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int pairs, cudaStream_t st,
-                        bool programmatic) {
+static void pair_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int pairs, int threads, cudaStream_t st,
+                        bool programmatic, bool cluster = true) {
   *cfg = cudaLaunchConfig_t{};
   cfg->gridDim = dim3(2 * pairs, 1, 1);
-  cfg->blockDim = dim3(TC_THREADS, 1, 1);
+  cfg->blockDim = dim3(threads, 1, 1);
   cfg->dynamicSmemBytes = SMEM_BYTES;
   cfg->stream = st;
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
   cfg->attrs = attr;
-  cfg->numAttrs = 1;
+  cfg->numAttrs = 0;
+  if (cluster) {
+    attr[cfg->numAttrs].id = cudaLaunchAttributeClusterDimension;
+    attr[cfg->numAttrs].val.clusterDim.x = 2;
+    attr[cfg->numAttrs].val.clusterDim.y = 1;
+    attr[cfg->numAttrs].val.clusterDim.z = 1;
+    ++cfg->numAttrs;
+  }
   if (programmatic) {
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
-    cfg->numAttrs = 2;
+    attr[cfg->numAttrs].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[cfg->numAttrs].val.programmaticStreamSerializationAllowed = 1;
+    ++cfg->numAttrs;
   }
 }
 
 cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs) {
-  cudaError_t e = pair_opt_in<false>();
+  cudaError_t e = pair_opt_in<HF_BF16, false>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
-  pair_config(&cfg, attr, sm_count / 2, nullptr, false);
+  pair_config(&cfg, attr, sm_count / 2, pair_threads<HF_BF16>(), nullptr, false);
   int n = 0;
-  e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel<false>, &cfg);
+  e = cudaOccupancyMaxActiveClusters(&n, lmhead_pair_kernel<HF_BF16, false>, &cfg);
   if (e != cudaSuccess) return e;
   *pairs = n < 1 ? 1 : n;
   return cudaSuccess;
 }
 
-cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const TcArgs& a, cudaStream_t st) {
-  const bool verify = a.part_t != nullptr;
-  cudaError_t e = verify ? pair_opt_in<true>() : pair_opt_in<false>();
+template <int HF, bool VERIFY>
+static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps& tmQ,
+                               const TcArgs& a, cudaStream_t st) {
+  cudaError_t e = pair_opt_in<HF, VERIFY>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
-  pair_config(&cfg, attr, a.plan.G, st, true);
-  return verify ? cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<true>, tmH, tmW, a)
-                : cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<false>, tmH, tmW, a);
+  pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, HF == HF_BF16);
+  return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, a);
+}
+
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ, int hf,
+                               const TcArgs& a, cudaStream_t st) {
+  const bool verify = a.part_t != nullptr;
+  PairQuantMaps none;
+  std::memset(&none, 0, sizeof(none));
+  const PairQuantMaps& q = tmQ ? *tmQ : none;
+  switch (hf) {
+    case HF_E4M3:
+      return verify ? launch_pair<HF_E4M3, true>(tmH, tmW, q, a, st) : launch_pair<HF_E4M3, false>(tmH, tmW, q, a, st);
+    case HF_NVFP4:
+      return verify ? launch_pair<HF_NVFP4, true>(tmH, tmW, q, a, st)
+                    : launch_pair<HF_NVFP4, false>(tmH, tmW, q, a, st);
+    default:
+      return verify ? launch_pair<HF_BF16, true>(tmH, tmW, q, a, st) : launch_pair<HF_BF16, false>(tmH, tmW, q, a, st);
+  }
 }
 
 }  // namespace bd

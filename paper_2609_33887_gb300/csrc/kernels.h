@@ -66,9 +66,22 @@ cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, con
 struct PairTokenMaps {
   CUtensorMap m[8];
 };
+// Head formats of the pair kernel: bf16 rows staged as they are, or E4M3 /
+// NVFP4 codes decoded to bf16 inside the kernel (codes: [V, ld] bytes with
+// 128 x 128-byte SW128 boxes; NVFP4 block scales: [V, block_ld] bytes with
+// 16 x 128-byte boxes).
+enum : int { HF_BF16 = 0, HF_E4M3 = 1, HF_NVFP4 = 2 };
+struct PairQuantMaps {
+  CUtensorMap codes;
+  CUtensorMap scales;
+};
 size_t pair_smem_bytes();
 cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs);
-cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const TcArgs& a, cudaStream_t st);
+// hf: HF_BF16 (tmW describes the bf16 head; tmQ unused, may be null) or
+// HF_E4M3 / HF_NVFP4 (tmQ describes the codes, and the NVFP4 block scales;
+// tmW unused). E4M3 and NVFP4 need the TcArgs row scale wscale.
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ, int hf,
+                               const TcArgs& a, cudaStream_t st);
 
 // a1+a2 with fp32 FMA on the CUDA cores (exact fp32 path; any dtype combo).
 struct SimtArgs {

@@ -2,7 +2,10 @@
 
 The library decodes every E2M1 x E4M3 product exactly to bf16 and applies the
 per-row scale to the fp32 logit, so the bf16 path's tolerances apply (tokens
-and commit bits exact away from near-ties, confidence within 2e-3).
+and commit bits exact away from near-ties, confidence within 2e-3). The CTA-pair
+kernel decodes the codes itself when code and block-scale rows start on
+16-byte boundaries (BD_FUSED_DECODE, default on), and otherwise from a bf16
+copy decoded beforehand; both are checked.
 """
 
 import numpy as np
@@ -38,10 +41,11 @@ def padded_rows(t, multiple=16):
     return out[:, : t.shape[1]]
 
 
-def run(wl, variant=0):
+def run(wl, variant=0, pad_scales=False):
     cfg = wl.cfg
     g = wl.to("cuda")
-    head = bdc.Nvfp4Head(padded_rows(g.weight), g.weight_block_scale, cfg.d)
+    scales = padded_rows(g.weight_block_scale) if pad_scales else g.weight_block_scale
+    head = bdc.Nvfp4Head(padded_rows(g.weight), scales, cfg.d)
     tokens, conf, commit, counts = bdc.commit_step(
         g.hidden, head, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, wl.tau,
         weight_scale=g.weight_scale, mask_token_id=wl.mask_token_id, counts=True, variant=variant)
@@ -51,9 +55,9 @@ def run(wl, variant=0):
             "commit": commit.cpu().numpy().view(np.uint32), "counts": counts.cpu().numpy()}
 
 
-def check(wl, variant=0, blocks=None):
+def check(wl, variant=0, blocks=None, pad_scales=False):
     ref = oracle_on_workload(wl, blocks=blocks)
-    rep = compare(run(wl, variant), ref, wl.tau, "nvfp4", wl.cfg.block_len, wl.cfg.n_slots)
+    rep = compare(run(wl, variant, pad_scales), ref, wl.tau, "nvfp4", wl.cfg.block_len, wl.cfg.n_slots)
     assert rep.ok(), rep.failures
     return rep
 
@@ -70,6 +74,17 @@ SMALL = {
 @pytest.mark.parametrize("variant", [0, 1, 2, 3])
 def test_small(name, variant):
     rep = check(generate(SMALL[name]), variant)
+    assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("name", sorted(SMALL))
+@pytest.mark.parametrize("fused", [True, False])
+def test_pair_fused_and_decoded(name, fused, monkeypatch):
+    """The pair kernel decoding the codes in shared memory (16-byte aligned code
+    and scale rows, K tails included) and the same kernel on the decoded copy."""
+    if not fused:
+        monkeypatch.setenv("BD_FUSED_DECODE", "0")
+    rep = check(generate(SMALL[name]), variant=3, pad_scales=True)
     assert rep.n_live > 0
 
 

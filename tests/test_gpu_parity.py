@@ -100,6 +100,16 @@ def test_small_one_cta_tensor_core_variant(name):
     check(wl, variant=2)
 
 
+@pytest.mark.parametrize("name", ["e4m3", "e4m3_ktail"])
+@pytest.mark.parametrize("fused", [True, False])
+def test_e4m3_pair_fused_and_decoded(name, fused, monkeypatch):
+    # the pair kernel decodes E4M3 codes in shared memory (rows of 16-byte
+    # multiples), or reads a bf16 copy decoded beforehand
+    if not fused:
+        monkeypatch.setenv("BD_FUSED_DECODE", "0")
+    check(generate(SMALL[name]), variant=3)
+
+
 @pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "e4m3"])
 def test_small_simt_variant(name):
     wl = generate(SMALL[name])
