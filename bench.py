@@ -404,10 +404,15 @@ def nvfp4_timing(dev, stream) -> dict:
     lm_us = st_.mean(a.elapsed_time(b) for a, b in lm) * 1e3
     n_masked = int(((wl.pos_masked != 0) & (torch.repeat_interleave(wl.block_flags & 1, cfg.block_len) != 0)).sum())
     abytes = cfg.V * cfg.d // 2 + cfg.V * ((cfg.d + 15) // 16) + 4 * cfg.V + n_masked * cfg.d * 2 + P * 13
-    hbm_gbs, _, _, src = peaks()
+    flops = 2.0 * n_masked * cfg.d * cfg.V
+    hbm_gbs, tc_tflops, _, src = peaks()
     return {"workload": cfg.name, "ms_per_step": ms, "positions_per_s": n_masked / (ms / 1e3),
-            "lmhead_us": lm_us, "algorithmic_bytes": abytes,
-            "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs, "peak_source": src}
+            "lmhead_us": lm_us, "algorithmic_bytes": abytes, "algorithmic_flops": flops,
+            "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs,
+            "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_tflops,
+            "path": "codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA); "
+                    "bound: the converter warps' instruction issue",
+            "peak_source": src}
 
 
 def run_ours(args):
