@@ -97,7 +97,14 @@ typedef struct {
  *                   per-row scale (NULL = 1). Weight (v, k) =
  *                   e2m1(code) * e4m3(block scale) * scale[v].
  *   For BD_BF16 / BD_E4M3 / BD_NVFP4 the pointer must be 16-byte aligned and
- *   ld * element size (bytes for BD_NVFP4) a multiple of 16. */
+ *   ld * element size (bytes for BD_NVFP4) a multiple of 16.
+ *   Both quantised formats decode exactly to bf16. On the CTA-pair LM-head
+ *   kernel (windows up to 8192 positions) the codes are decoded inside the
+ *   kernel, so the workspace holds no bf16 copy of the head, when a row holds
+ *   at least 16 bytes of codes and, for BD_NVFP4, `block_scale` is 16-byte
+ *   aligned with block_ld a multiple of 16; otherwise the head is first
+ *   decoded into a bf16 copy in the workspace (bd_workspace_size accounts
+ *   for it). The environment variable BD_FUSED_DECODE=0 forces the copy. */
 typedef struct {
   const void* data;
   int32_t dtype;
