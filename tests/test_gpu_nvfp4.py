@@ -88,6 +88,13 @@ def test_pair_fused_and_decoded(name, fused, monkeypatch):
     assert rep.n_live > 0
 
 
+def test_pair_fused_mask_token_in_last_tile():
+    """The in-kernel decode with a suppressed mask token inside the partial last v-tile."""
+    cfg = scaled(CONFIGS[1], n_seq=4, n_slots=2, d=256, V=2900, weight_dtype="nvfp4", mask_token_id=2899)
+    rep = check(generate(cfg), variant=3, pad_scales=True)
+    assert rep.n_live > 0
+
+
 def test_bench_window_nvfp4_head():
     """The 8 x 2 x 32 window with the 151936 x 2048 head in NVFP4, every masked position."""
     wl = generate(by_name("b8x2x32_d2048_v151936_nvfp4"))
