@@ -76,6 +76,53 @@ def decode_e4m3(raw: np.ndarray) -> np.ndarray:
     return out
 
 
+def encode_e4m3(x: np.ndarray) -> np.ndarray:
+    """float64 values -> FP8 E4M3 codes (uint8), rounding to the nearest
+    representable value with ties to the even code, magnitudes above the
+    largest finite value 448 saturating to 448 (the "satfinite" conversion the
+    W8A8 activations go through). The sign is kept, -0 included.
+
+    Written from the format's definition: the non-negative finite codes
+    0x00..0x7E are increasing in value (decode_e4m3), so a value's two
+    neighbours on that grid are found by bisection."""
+    x = np.asarray(x, dtype=np.float64)
+    grid = decode_e4m3(np.arange(0x7F, dtype=np.uint8))  # 0x00..0x7E, increasing
+    a = np.minimum(np.abs(x), grid[-1])
+    hi = np.clip(np.searchsorted(grid, a, side="left"), 0, len(grid) - 1)  # first grid value >= a
+    lo = np.maximum(hi - 1, 0)
+    d_lo = a - grid[lo]
+    d_hi = grid[hi] - a
+    take_hi = (d_hi < d_lo) | ((d_hi == d_lo) & (hi % 2 == 0))
+    code = np.where(a == grid[hi], hi, np.where(take_hi, hi, lo)).astype(np.uint8)
+    return np.where(np.signbit(x), code | 0x80, code).astype(np.uint8)
+
+
+def quantize_rows_e4m3(h: np.ndarray):
+    """Per-row E4M3 quantisation of activations (the W8A8 variant of the
+    precision lever): for row i with a = max_k |h[i, k]| (float32),
+    inv = fl32(448 / a), codes = encode_e4m3(fl32(h[i, k] * inv)) and the
+    row's dequantisation scale fl32(a / 448); an all-zero row gets codes 0 and
+    scale 0. Every float32 operation is one correctly rounded IEEE operation,
+    so a device implementation that performs the same operations produces the
+    same codes. Returns (codes uint8 [n, d], scale float32 [n])."""
+    h = np.asarray(h, dtype=np.float32)
+    amax = np.max(np.abs(h), axis=1) if h.shape[1] else np.zeros(h.shape[0], np.float32)
+    codes = np.zeros(h.shape, dtype=np.uint8)
+    scale = np.zeros(h.shape[0], dtype=np.float32)
+    nz = amax > 0
+    inv = np.zeros_like(amax)
+    inv[nz] = np.float32(448.0) / amax[nz]
+    y = (h * inv[:, None]).astype(np.float32)
+    codes[nz] = encode_e4m3(y[nz].astype(np.float64))
+    scale[nz] = amax[nz] / np.float32(448.0)
+    return codes, scale
+
+
+def dequantize_rows_e4m3(codes: np.ndarray, scale: np.ndarray) -> np.ndarray:
+    """The float64 activations the W8A8 LM head multiplies: code value times the row scale."""
+    return decode_e4m3(codes) * np.asarray(scale, dtype=np.float64)[:, None]
+
+
 def decode_e2m1(codes: np.ndarray) -> np.ndarray:
     """FP4 E2M1 codes (0..15) -> float64, per the OCP microscaling 4-bit float:
     1 sign bit, 2 exponent bits (bias 1), 1 mantissa bit; exponent field 0
@@ -136,6 +183,8 @@ def weights_f64(raw, dtype: str, scale: Optional[np.ndarray] = None, d: Optional
 
 
 def hidden_f64(raw: np.ndarray, dtype: str) -> np.ndarray:
+    if dtype == "f64":  # values already decoded (e.g. the W8A8 variant's dequantised activations)
+        return np.asarray(raw, dtype=np.float64)
     if dtype == "f32":
         return np.asarray(raw, dtype=np.float32).astype(np.float64)
     if dtype == "bf16":
