@@ -53,7 +53,7 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-verify", action="store_true",
-                    help="skip the speculative-verification and NVFP4-head measurements")
+                    help="skip the speculative-verification and precision-lever (NVFP4, E4M3, W8A8) measurements")
     return ap.parse_args()
 
 
@@ -356,21 +356,38 @@ def verify_timing(dev, stream) -> dict:
             "tokens_per_forward": tpf, "data": "synthetic drafts, agreement 0.905 with the planted argmax"}
 
 
-def nvfp4_timing(dev, stream) -> dict:
-    """The bench window (8 x 2 x 32, d = 2048, V = 151936) with the head in
-    NVFP4 (the 4-bit weight lever): device time per commit step (CUDA events
-    around 200 back-to-back steps), the LM-head kernel's own time, and the
-    step against the 4-bit algorithmic bytes (codes V*d/2, block scales
-    V*d/16, row scales 4V, the masked rows and 13 B per window position)."""
+LEVERS = {
+    # key: (workload, description of the LM-head path and what bounds it)
+    "nvfp4": ("b8x2x32_d2048_v151936_nvfp4",
+              "codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA); "
+              "bound: the converter warps' instruction issue"),
+    "e4m3": ("b8x2x32_d2048_v151936_e4m3",
+             "W8A16: E4M3 codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA)"),
+    "w8a8": ("b8x2x32_d2048_v151936_e4m3",
+             "W8A8: packed rows quantised to E4M3 per row by the compaction kernel, E4M3 x E4M3 on the "
+             "8-bit tensor path (tcgen05.mma kind::f8f6f4), both scales applied to the fp32 logits"),
+}
+
+
+def lever_timing(dev, stream, lever: str) -> dict:
+    """The bench window (8 x 2 x 32, d = 2048, V = 151936) with a quantised
+    head (the precision levers): device time per commit step (CUDA events
+    around 200 back-to-back steps), the LM-head kernel's own time, and the step
+    against the lever's algorithmic bytes (the stored head: NVFP4 codes V*d/2
+    and block scales V*d/16, or E4M3 codes V*d; row scales 4V; the masked bf16
+    rows; 13 B per window position). The tensor fraction of the W8A8 head is
+    taken against twice the measured bf16 peak (the nominal FP8 : BF16 ratio)."""
     import statistics as st_
 
     import paper_2609_33887_gb300 as bdc
     from paper_2609_33887_gb300 import bdcommit as B
 
-    cfg = by_name("b8x2x32_d2048_v151936_nvfp4")
+    name, path = LEVERS[lever]
+    cfg = by_name(name)
     wl = generate(cfg).to(dev)
-    head = bdc.Nvfp4Head(wl.weight, wl.weight_block_scale, cfg.d)
-    P, T = cfg.P, len(cfg.tau)
+    head = bdc.Nvfp4Head(wl.weight, wl.weight_block_scale, cfg.d) if lever == "nvfp4" else wl.weight
+    flags = B.BD_EXEC_FP8_ACTIVATIONS if lever == "w8a8" else 0
+    P = cfg.P
     ws = torch.empty(bdc.bd_workspace_size(wl.hidden, head, wl.weight_scale, wl.pos_masked, wl.block_flags,
                                            cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau),
                      dtype=torch.uint8, device=dev)
@@ -381,9 +398,9 @@ def nvfp4_timing(dev, stream) -> dict:
     def step(ev=None):
         rc = B.bd_commit_step_ex(wl.hidden, head, wl.weight_scale, wl.pos_masked, wl.block_flags, cfg.n_seq,
                                  cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau, tokens, conf, commit,
-                                 stream=stream, workspace=ws, lmhead_events=ev)
+                                 stream=stream, workspace=ws, lmhead_events=ev, flags=flags)
         if rc != 0:
-            raise B.BdError(rc, "nvfp4 step")
+            raise B.BdError(rc, f"{lever} step")
 
     for _ in range(5):
         step()
@@ -399,20 +416,22 @@ def nvfp4_timing(dev, stream) -> dict:
     torch.cuda.synchronize()
     st = B.bd_get_device_status(stream)
     if st != 0:
-        raise B.BdError(st, "nvfp4")
+        raise B.BdError(st, lever)
     ms = e0.elapsed_time(e1) / n
     lm_us = st_.mean(a.elapsed_time(b) for a, b in lm) * 1e3
     n_masked = int(((wl.pos_masked != 0) & (torch.repeat_interleave(wl.block_flags & 1, cfg.block_len) != 0)).sum())
-    abytes = cfg.V * cfg.d // 2 + cfg.V * ((cfg.d + 15) // 16) + 4 * cfg.V + n_masked * cfg.d * 2 + P * 13
+    head_bytes = (cfg.V * cfg.d // 2 + cfg.V * ((cfg.d + 15) // 16)) if lever == "nvfp4" else cfg.V * cfg.d
+    abytes = head_bytes + 4 * cfg.V + n_masked * cfg.d * 2 + P * 13
     flops = 2.0 * n_masked * cfg.d * cfg.V
     hbm_gbs, tc_tflops, _, src = peaks()
+    tc_peak = 2.0 * tc_tflops if lever == "w8a8" else tc_tflops
     return {"workload": cfg.name, "ms_per_step": ms, "positions_per_s": n_masked / (ms / 1e3),
             "lmhead_us": lm_us, "algorithmic_bytes": abytes, "algorithmic_flops": flops,
             "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs,
-            "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_tflops,
-            "path": "codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA); "
-                    "bound: the converter warps' instruction issue",
-            "peak_source": src}
+            "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_peak,
+            "tensor_peak_tflops": tc_peak,
+            "path": path,
+            "peak_source": src + (" (x2: nominal FP8 : BF16 ratio)" if lever == "w8a8" else "")}
 
 
 def run_ours(args):
@@ -682,7 +701,7 @@ def run_ours(args):
 
     redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
     verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
-    nvfp4 = nvfp4_timing(dev, stream) if rank == 0 and not args.no_verify else None
+    levers = {k: lever_timing(dev, stream, k) for k in LEVERS} if rank == 0 and not args.no_verify else {}
 
     if rank == 0:
         line = {
@@ -703,7 +722,9 @@ def run_ours(args):
             "redline": redline,
             "sweep": sweep,
             "verify": verify,
-            "nvfp4": nvfp4,
+            "nvfp4": levers.get("nvfp4"),
+            "e4m3": levers.get("e4m3"),
+            "w8a8": levers.get("w8a8"),
         }
         print(json.dumps(line), flush=True)
     if pg:

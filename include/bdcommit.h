@@ -61,6 +61,9 @@ typedef enum {
   BD_NVFP4 = 3 /* 4-bit E2M1 codes with an E4M3 scale per 16 elements (NVFP4), weights only */
 } bd_dtype;
 
+/* bd_exec.flags bits. */
+#define BD_EXEC_FP8_ACTIVATIONS 1
+
 /* Block flag bits (bd_mask_state.block_flags). */
 #define BD_BLOCK_ACTIVE 1u            /* the slot holds an active block (App. F) */
 #define BD_BLOCK_FALLBACK_ELIGIBLE 2u /* the block may take the top-1 fallback (App. B.2) */
@@ -162,7 +165,19 @@ typedef struct {
  *                     tensor-core kernel (tokens on the MMA M side); 3 = force the
  *                     CTA-pair tensor-core kernel (vocabulary on the M side).
  *                     2 and 3 need BF16 hidden states.
- *   flags           : reserved, must be 0. */
+ *   flags           : 0, or BD_EXEC_FP8_ACTIVATIONS (commit step only): the
+ *                     W8A8 variant of the precision lever. Needs a BD_E4M3 head
+ *                     (16-byte aligned, ld a multiple of 16, dim >= 16), BF16
+ *                     hidden states and the CTA-pair kernel (variant 0 or 3,
+ *                     windows up to 8192 positions); else BD_ERR_ARG / ALIGN.
+ *                     Each packed hidden row is quantised to E4M3 with one
+ *                     scale per row (a = max |h|, code = e4m3(h * fl32(448 /
+ *                     a)) rounding to nearest even and saturating, scale =
+ *                     fl32(a / 448); an all-zero row gets scale 0) and the LM
+ *                     head multiplies the E4M3 codes on the 8-bit tensor path
+ *                     (tcgen05.mma kind::f8f6f4), applying the head's row scale
+ *                     and the token's scale to each fp32 logit. Lossy: results
+ *                     are those of the quantised activations. */
 typedef struct {
   void* stream;
   void* workspace;

@@ -49,6 +49,9 @@ VARIANT_SIMT = 1
 VARIANT_TC_ONE_CTA = 2
 VARIANT_TC_PAIR = 3
 
+# bd_exec.flags
+BD_EXEC_FP8_ACTIVATIONS = 1  # W8A8: E4M3 token rows x E4M3 head on the 8-bit tensor path
+
 
 class bd_hidden(ctypes.Structure):
     _fields_ = [("data", c_void_p), ("dtype", c_int32), ("rows", c_int64), ("cols", c_int64), ("ld", c_int64)]
@@ -233,7 +236,7 @@ def bd_workspace_size(hidden, weight, weight_scale, pos_masked, block_flags, n_s
 
 def bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
                       mask_token_id, tau, out_tokens, out_conf, out_commit, *, stream=None, workspace=None,
-                      out_counts=None, lmhead_events=None, variant=VARIANT_AUTO) -> int:
+                      out_counts=None, lmhead_events=None, variant=VARIANT_AUTO, flags=0) -> int:
     """Queue one commit step on `stream` (default: torch's current stream).
 
     All tensors are device tensors; `tau` is a host sequence of floats.
@@ -252,7 +255,7 @@ def bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_s
         ex.lmhead_event_begin = lmhead_events[0].cuda_event
         ex.lmhead_event_end = lmhead_events[1].cuda_event
     ex.variant = variant
-    ex.flags = 0
+    ex.flags = flags
     return int(load_library().bd_commit_step_ex(
         ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
         _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit), ctypes.byref(ex)))
@@ -288,8 +291,11 @@ def bd_commit_step_static(hidden, weight, weight_scale, pos_masked, block_flags,
 
 def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_len, tau, *,
                 weight_scale=None, mask_token_id=-1, stream=None, workspace=None, counts=False,
-                variant=VARIANT_AUTO, lmhead_events=None):
+                variant=VARIANT_AUTO, lmhead_events=None, fp8_activations=False):
     """Allocate the outputs on the hidden states' device, queue the step, raise on error.
+
+    fp8_activations=True selects the W8A8 variant (an E4M3 head only): the
+    packed hidden rows are quantised to E4M3 with one scale per row.
 
     Returns (tokens int32 [P], conf float32 [P], commit int32 [P] holding the
     uint32 bit masks, counts int32 [n_seq, T] or None)."""
@@ -301,7 +307,8 @@ def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_l
     cnt = torch.empty((n_seq, len(tau)), dtype=torch.int32, device=dev) if counts else None
     rc = bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
                            mask_token_id, tau, tokens, conf, commit, stream=stream, workspace=workspace,
-                           out_counts=cnt, lmhead_events=lmhead_events, variant=variant)
+                           out_counts=cnt, lmhead_events=lmhead_events, variant=variant,
+                           flags=BD_EXEC_FP8_ACTIVATIONS if fp8_activations else 0)
     if rc != BD_OK:
         raise BdError(rc)
     return tokens, conf, commit, cnt

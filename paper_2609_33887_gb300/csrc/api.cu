@@ -79,13 +79,16 @@ struct Call {
   int64_t ldc;      // packed hidden rows (bf16), elements
   int64_t ldq;      // decoded e4m3 head (bf16), elements
   bool fused;       // pair kernel decodes an E4M3 / NVFP4 head itself (no bf16 copy)
+  bool fp8_act = false;  // W8A8: token rows quantised to E4M3, kind::f8f6f4 MMAs on the E4M3 head
 };
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }  // NVFP4: ld counts bytes
 
-bool decoded_head(const Call& c) { return c.tc && !c.fused && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4); }
+bool decoded_head(const Call& c) {
+  return c.tc && !c.fused && !c.fp8_act && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4);
+}
 
 // Decodes an FP8 or NVFP4 head into the bf16 workspace copy the tensor-core
 // kernels read (both decodes are exact); wsrc / wld then describe that copy.
@@ -216,7 +219,7 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs) {
 }
 
 struct Layout {
-  size_t hdr, idx, rowpos, pm, ps, pa, hc, wq, total;
+  size_t hdr, idx, rowpos, pm, ps, pa, hc, tsc, wq, total;
 };
 
 Layout make_layout(const Call& c, const BandPlan& p) {
@@ -236,11 +239,15 @@ Layout make_layout(const Call& c, const BandPlan& p) {
   l.pm = take(4 * slots * P, 256);
   l.ps = take(4 * slots * P, 256);
   l.pa = take(4 * slots * P, 256);
-  l.hc = c.tc ? take(2 * static_cast<size_t>(c.ldc) * P, 1024) : 0;
+  l.hc = c.tc ? take(2 * static_cast<size_t>(c.ldc) * P, 1024) : 0;  // bf16 rows, or E4M3 rows (W8A8)
+  l.tsc = take(4 * P, 256);                                             // W8A8: per-row token scales
   l.wq = decoded_head(c) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
   l.total = (off + 255) / 256 * 256;
   return l;
 }
+
+// Row stride (bytes) of the packed E4M3 token rows of the W8A8 variant.
+int64_t ld_fp8_rows(const Call& c) { return round_up(c.d, 16); }
 
 bool encode_bf16_2d(CUtensorMap* m, const void* base, int64_t inner, int64_t rows, int64_t ld_elems,
                     uint32_t box_inner, uint32_t box_rows) {
@@ -302,7 +309,7 @@ struct Partials {
 int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, const bd_weight* weight,
                   const void* rows, int64_t ld_rows, void* wq, const int* idx, const int* n_rows,
                   const int* draft_row, const Partials& part, uint32_t* status, int sm_count, void* ev_begin,
-                  void* ev_end, cudaStream_t st) {
+                  void* ev_end, cudaStream_t st, const float* tok_scale = nullptr) {
   const int P = static_cast<int>(c.P), V = static_cast<int>(c.V), d = static_cast<int>(c.d);
   const float* wscale = (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4) ? weight->scale : nullptr;
   CUtensorMap tmA, tmB;
@@ -310,7 +317,7 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
   bd::PairQuantMaps tmQ;
   std::memset(&tmB, 0, sizeof(tmB));
   std::memset(&tmQ, 0, sizeof(tmQ));
-  const int hf = !c.fused ? bd::HF_BF16 : c.wdt == BD_NVFP4 ? bd::HF_NVFP4 : bd::HF_E4M3;
+  const int hf = c.fp8_act ? bd::HF_W8A8 : !c.fused ? bd::HF_BF16 : c.wdt == BD_NVFP4 ? bd::HF_NVFP4 : bd::HF_E4M3;
   if (c.fused) {
     // codes: 128 bytes of a row per box (128 NVFP4 / E4M3 ... columns of d: 256 / 128)
     const int64_t code_bytes = c.wdt == BD_NVFP4 ? (c.d + 1) / 2 : c.d;
@@ -326,7 +333,12 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
       const int rc = decode_head(c, weight, wq, sm_count, st, &wsrc, &wld);
       if (rc != BD_OK) return rc;
     }
-    if (c.pair) {
+    if (c.pair && c.fp8_act) {
+      // W8A8: E4M3 token rows and head rows, 128-byte (128-column) boxes
+      for (int i = 0; i < 8; ++i)
+        if (!encode_u8_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 128, 16 * (i + 1), true)) return BD_ERR_CUDA;
+      if (!encode_u8_2d(&tmB, weight->data, c.d, c.V, c.ldw, 128, 128, true)) return BD_ERR_CUDA;
+    } else if (c.pair) {
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
       for (int i = 0; i < 8; ++i)
         if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 16 * (i + 1))) return BD_ERR_CUDA;
@@ -354,6 +366,7 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
     a.draft_row = draft_row;
     a.part_t = part.t;
     a.part_x = part.x;
+    a.tok_scale = tok_scale;
     rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, c.fused ? &tmQ : nullptr, hf, a, st))
                 : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
   } else {
@@ -407,13 +420,16 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   }
 
   // a0: compaction of the masked positions of active blocks (+ packing of their rows)
+  // (W8A8: the packed rows are quantised to E4M3 with one scale per row)
+  float* tsc = c.fp8_act ? reinterpret_cast<float*>(ws + lay.tsc) : nullptr;
+  const int64_t ld_rows = c.fp8_act ? ld_fp8_rows(c) : c.ldc;
   int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
                                             c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
-                                            c.ldc, idx, rowpos, n_rows, sm_count, st));
+                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc));
   if (rc != BD_OK) return rc;
 
-  rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, c.ldc, ws + lay.wq, idx, n_rows, nullptr,
-                     Partials{pm, ps, pa, nullptr, nullptr}, status, sm_count, ev_begin, ev_end, st);
+  rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, ld_rows, ws + lay.wq, idx, n_rows, nullptr,
+                     Partials{pm, ps, pa, nullptr, nullptr}, status, sm_count, ev_begin, ev_end, st, tsc);
   if (rc != BD_OK) return rc;
 
   // a3 + a4: merge and the multi-threshold commit
@@ -475,10 +491,18 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd
                       const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                       const bd_exec* exec) {
   const int variant = exec ? exec->variant : 0;
-  if (exec && exec->flags != 0) return BD_ERR_ARG;
+  const int flags = exec ? exec->flags : 0;
+  if (flags & ~BD_EXEC_FP8_ACTIVATIONS) return BD_ERR_ARG;
   Call c;
   int rc = check_args(hidden, weight, mask_state, tau_grid, variant, &c);
   if (rc != BD_OK) return rc;
+  if (flags & BD_EXEC_FP8_ACTIVATIONS) {
+    // W8A8 runs on the CTA-pair kernel with an E4M3 head read by TMA
+    if (c.wdt != BD_E4M3 || c.hdt != BD_BF16 || !c.pair) return BD_ERR_ARG;
+    if (!aligned(weight->data, 16) || weight->ld % 16 != 0 || c.d < 16) return BD_ERR_ALIGN;
+    c.fp8_act = true;
+    c.fused = false;
+  }
   if (c.P == 0) return BD_OK;
   if (!out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
   if (!aligned(out_tokens, 4) || !aligned(out_conf, 4) || !aligned(out_commit, 4)) return BD_ERR_ALIGN;
@@ -527,6 +551,7 @@ int bd_get_device_status(void* stream) {
   if (cudaMemcpy(&word, ctx->status, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return BD_ERR_CUDA;
   if (word != 0 && cudaMemset(ctx->status, 0, sizeof(word)) != cudaSuccess) return BD_ERR_CUDA;
   if (word & bd::DEV_TIMEOUT) return BD_ERR_TIMEOUT;
+  if (word & bd::DEV_BAD_LAUNCH) return BD_ERR_CUDA;
   return BD_OK;
 }
 

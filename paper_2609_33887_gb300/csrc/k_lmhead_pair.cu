@@ -50,11 +50,29 @@ namespace bd {
 
 namespace {
 
-// columns of d per operand stage: two 64-column swizzle atoms for bf16 heads;
-// one for quantised heads, whose small stages leave room for a deep raw ring
+// Heads decoded in the kernel by converter warps (E4M3 / NVFP4 codes); the
+// W8A8 variant multiplies E4M3 codes directly on the 8-bit tensor path.
+template <int HF>
+__host__ __device__ constexpr bool is_quant() {
+  return HF == HF_E4M3 || HF == HF_NVFP4;
+}
+// Instantiations that issue cta_group::2 MMAs and must run as clusters of 2
+// (the heads decoded in the kernel run one CTA per half v-tile instead).
+template <int HF>
+__host__ __device__ constexpr bool pair_cluster() {
+  return !is_quant<HF>();
+}
+// columns of d per operand stage: two 64-column bf16 swizzle atoms for bf16
+// heads; one 128-column 8-bit atom for W8A8; one bf16 atom for heads decoded
+// in the kernel, whose small stages leave room for a deep raw ring
 template <int HF>
 __host__ __device__ constexpr int stage_k() {
-  return HF == HF_BF16 ? 128 : 64;
+  return is_quant<HF>() ? 64 : 128;
+}
+// columns of one 128-byte swizzle atom
+template <int HF>
+__host__ __device__ constexpr int atom_cols() {
+  return HF == HF_W8A8 ? 128 : 64;
 }
 constexpr int MAX_STAGES = 8;
 constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
@@ -71,7 +89,7 @@ constexpr int RAW_PRODUCER = 2 + EPI_WARPS + CONV_WARPS;  // warp streaming the 
 
 template <int HF>
 __host__ __device__ constexpr int pair_threads() {
-  return HF == HF_BF16 ? TC_THREADS : (RAW_PRODUCER + 1) * 32;
+  return is_quant<HF>() ? (RAW_PRODUCER + 1) * 32 : TC_THREADS;
 }
 // Raw ring of a quantised head: stages of 128 head rows x 128 bytes of codes
 // (SW128), plus 16 bytes of NVFP4 block scales per row.
@@ -136,16 +154,16 @@ __host__ __device__ constexpr size_t stage_area() {
 // A = 128 head rows, B = NT/2 token rows, each block 1 KB aligned.
 template <int HF>
 __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
-  // quantised heads: one CTA multiplies its 128 head rows by all NT token rows
-  return HF == HF_BF16 ? 2 * (A_BLOCK + static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES)
-                       : A_BLOCK + static_cast<uint32_t>(nt) * ATOM_ROWS_BYTES;
+  // heads decoded in the kernel: one CTA multiplies its 128 head rows by all NT token rows
+  return is_quant<HF>() ? A_BLOCK + static_cast<uint32_t>(nt) * ATOM_ROWS_BYTES
+                        : (stage_k<HF>() / atom_cols<HF>()) * (A_BLOCK + static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES);
 }
 // Operand stages: as many as fit (at most MAX_STAGES) for bf16 heads; for
 // quantised heads at most QUANT_STAGES next to a raw ring of at least three
 // stages, which takes the rest of the area.
 template <int HF, bool VERIFY>
 __host__ __device__ constexpr int stage_count(int nt) {
-  return HF != HF_BF16
+  return is_quant<HF>()
              ? (static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt)) < QUANT_STAGES
                     ? static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt))
                     : QUANT_STAGES)
@@ -155,7 +173,7 @@ __host__ __device__ constexpr int stage_count(int nt) {
 }
 template <int HF, bool VERIFY>
 __host__ __device__ constexpr int raw_count(int nt) {
-  return HF == HF_BF16 ? 0
+  return !is_quant<HF>() ? 0
          : static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
                             raw_bytes<HF>()) < MAX_RAW
              ? static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
@@ -164,6 +182,8 @@ __host__ __device__ constexpr int raw_count(int nt) {
 }
 static_assert(stage_count<HF_BF16, false>(256) >= 3 && stage_count<HF_BF16, true>(256) >= 3, "three stages at NT = 256");
 static_assert(stage_count<HF_BF16, false>(160) == 4, "four stages at NT = 160 on the commit path");
+static_assert(stage_count<HF_W8A8, false>(160) == 8 && stage_count<HF_W8A8, false>(256) >= 6,
+              "W8A8: 26 KB stages at NT = 160");
 static_assert(stage_count<HF_NVFP4, false>(160) == 4 && stage_count<HF_E4M3, false>(160) == 4 &&
                   stage_count<HF_NVFP4, true>(160) == 4 && stage_count<HF_E4M3, true>(160) == 4,
               "four operand stages at NT = 160 for quantised heads");
@@ -177,7 +197,7 @@ static_assert(stage_count<HF_NVFP4, true>(256) >= 3 && stage_count<HF_E4M3, true
 // stage. Columns at or past d decode to zero. ct: 0..CONV_THREADS-1.
 template <int HF>
 __device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t a_base, int ct, int kcol0, int d) {
-  static_assert(HF == HF_BF16 || stage_k<HF>() == 64, "one atom per quantised operand stage");
+  static_assert(!is_quant<HF>() || stage_k<HF>() == 64, "one atom per quantised operand stage");
   if constexpr (HF == HF_NVFP4) {
 #pragma unroll
     for (int i = 0; i < 256 / CONV_THREADS; ++i) {
@@ -239,13 +259,23 @@ template <int HF, bool VERIFY>
 __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW,
                        const __grid_constant__ PairQuantMaps tmQ, TcArgs a) {
-  constexpr bool QUANT = HF != HF_BF16;
+  constexpr bool QUANT = is_quant<HF>();
+  constexpr bool W8A8 = HF == HF_W8A8;
+  static_assert(!(W8A8 && VERIFY), "the W8A8 variant serves the commit step");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   PairTail<VERIFY>* tail = reinterpret_cast<PairTail<VERIFY>*>(smem + stage_area<VERIFY>());
   PairCtl* ctl = &tail->ctl;
   const uint32_t smem_base = smem_u32(smem);
 
+  if constexpr (pair_cluster<HF>()) {
+    // launched without its cluster of 2 there is no peer CTA to map or to
+    // pair MMAs with: report and do nothing
+    if (cluster_nctarank() != 2) {
+      if (threadIdx.x == 0) atomicOr(a.status, DEV_BAD_LAUNCH);
+      return;
+    }
+  }
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   // 0: the CTA that issues the pair's MMAs (bf16 heads); quantised heads: the
@@ -299,7 +329,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   griddep_wait();  // the packed rows and N come from the preceding kernel
   const int n_rows = *a.n_rows;
   constexpr int BK = stage_k<HF>();
-  constexpr int NATOM = BK / 64;
+  constexpr int ACOLS = atom_cols<HF>();
+  constexpr int NATOM = BK / ACOLS;
   const int nk = cdiv(a.d, BK);
   const int NT = pair_group_rows(n_rows);
   const int half = NT / 2;
@@ -348,8 +379,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
               const uint32_t fb = full0_leader + 8u * stage;
 #pragma unroll
               for (int j = 0; j < NATOM; ++j) {
-                tma_load_2d_pair(sa + j * A_BLOCK, &tmW, fb, kb * BK + 64 * j, vrow, pol_w);
-                tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + 64 * j, tok0, pol_h);
+                tma_load_2d_pair(sa + j * A_BLOCK, &tmW, fb, kb * BK + ACOLS * j, vrow, pol_w);
+                tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + ACOLS * j, tok0, pol_h);
               }
             }
           }
@@ -373,7 +404,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     // ------------------------------------------------------ MMA issuer (even CTA; every CTA for quantised heads)
     if (rank == 0 || QUANT) {
       const bool leader = elect_one();
-      const uint32_t idesc = idesc_bf16_f32(QUANT ? 128 : 256, NT);
+      const uint32_t idesc = W8A8 ? idesc_e4m3_f32(256, NT) : idesc_bf16_f32(QUANT ? 128 : 256, NT);
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
@@ -401,8 +432,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
                 const uint64_t bdesc = sw128_kmajor_desc(sa + NATOM * A_BLOCK + j * B_BLOCK);
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
+                  // +32 bytes along K per MMA (16 bf16 / 32 E4M3 columns) = +2 in the address field
                   if constexpr (QUANT)
                     umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                  else if constexpr (W8A8)
+                    umma_f8_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
                   else
                     umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
                 }
@@ -539,6 +573,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       int arg[MAX_CHUNKS];
       float t[MAX_CHUNKS], lx[MAX_CHUNKS];  // VERIFY only
       int xd[MAX_CHUNKS];                   // VERIFY only: draft entry of this thread's token
+      float ts[MAX_CHUNKS];                 // W8A8 only: this thread's token scale (1 for an all-zero row)
 #pragma unroll
       for (int c = 0; c < MAX_CHUNKS; ++c) {
         m[c] = -INFINITY;
@@ -547,6 +582,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         t[c] = 0.f;
         lx[c] = -INFINITY;
         xd[c] = -1;
+        ts[c] = 1.f;
+        if constexpr (W8A8) {
+          const int row = it.m_tile * NT + c * 32 + lane;
+          if (c < nch && row < n_rows && a.tok_scale[row] != 0.f) ts[c] = a.tok_scale[row];
+        }
         if constexpr (VERIFY) {
           const int row = it.m_tile * NT + c * 32 + lane;
           if (c < nch && row < n_rows) xd[c] = a.draft_row[row];
@@ -585,6 +625,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             float x[32];
 #pragma unroll
             for (int r = 0; r < 32; ++r) x[r] = tr[r * TR + lane];
+            if constexpr (W8A8) {
+              // the token row's dequantisation scale (an all-zero row has logits 0 already)
+#pragma unroll
+              for (int r = 0; r < 32; ++r) x[r] *= ts[c];
+            }
             if constexpr (VERIFY) {
               const int rel = xd[c] - vrow0;
               if (rel >= 0 && rel < 32) lx[c] = tr[rel * TR + lane];
@@ -786,7 +831,7 @@ static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
-  pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, HF == HF_BF16);
+  pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, pair_cluster<HF>());
   return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, a);
 }
 
@@ -797,6 +842,9 @@ cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
   std::memset(&none, 0, sizeof(none));
   const PairQuantMaps& q = tmQ ? *tmQ : none;
   switch (hf) {
+    case HF_W8A8:
+      if (verify) return cudaErrorInvalidValue;
+      return launch_pair<HF_W8A8, false>(tmH, tmW, q, a, st);
     case HF_E4M3:
       return verify ? launch_pair<HF_E4M3, true>(tmH, tmW, q, a, st) : launch_pair<HF_E4M3, false>(tmH, tmW, q, a, st);
     case HF_NVFP4:

@@ -35,10 +35,18 @@ __device__ __forceinline__ int block_sum(int v, int* red) {
   return t;
 }
 
+// Two float32 values -> two E4M3 codes (round to nearest even, saturating at
+// 448), `lo` in the low byte.
+__device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
+  uint16_t r;
+  asm("cvt.rn.satfinite.e4m3x2.f32 %0, %1, %2;" : "=h"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
 __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags, int P, int block_len, int chunk,
     const __nv_bfloat16* __restrict__ hidden, int64_t ld, int d, __nv_bfloat16* __restrict__ hc, int64_t ldc,
-    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows) {
+    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale) {
   __shared__ int red[PREP_THREADS / 32];
   __shared__ int warp_excl[PREP_THREADS / 32];
   __shared__ int rows_s[2048];
@@ -97,8 +105,53 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
   if (hidden == nullptr) return;
   __syncthreads();
 
-  // 3. copy the chunk's live rows, one warp per row, 16-byte vectors
   const int nvec = d / 8;
+  if (tok_scale != nullptr) {
+    // 3'. W8A8: quantise the chunk's live rows to E4M3 with one scale per row,
+    // one warp per row: a = max |h|, inv = 448 / a, code = e4m3(h * inv) (round
+    // to nearest even, saturating), scale = a / 448; an all-zero row gets codes
+    // 0 and scale 0. Each float32 step is one correctly rounded operation.
+    uint8_t* hq = reinterpret_cast<uint8_t*>(hc);  // ldc counts bytes here
+    for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+      const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
+      const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      float amax = 0.f;
+      for (int v = lane; v < nvec; v += 32) {
+        const uint4 q = __ldg(s4 + v);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[j]));
+          amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+        }
+      }
+      for (int e = nvec * 8 + lane; e < d; e += 32) amax = fmaxf(amax, fabsf(__bfloat162float(src[e])));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+      const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
+      uint8_t* dst = hq + static_cast<int64_t>(prefix + i) * ldc;
+      for (int v = lane; v < nvec; v += 32) {
+        const uint4 q = __ldg(s4 + v);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        uint32_t out[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          const float2 f0 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[2 * j]));
+          const float2 f1 = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[2 * j + 1]));
+          out[j] = f32x2_to_e4m3x2(__fmul_rn(f0.x, inv), __fmul_rn(f0.y, inv)) |
+                   (f32x2_to_e4m3x2(__fmul_rn(f1.x, inv), __fmul_rn(f1.y, inv)) << 16);
+        }
+        *reinterpret_cast<uint2*>(dst + 8 * v) = make_uint2(out[0], out[1]);
+      }
+      for (int e = nvec * 8 + lane; e < d; e += 32)
+        dst[e] = static_cast<uint8_t>(f32x2_to_e4m3x2(__fmul_rn(__bfloat162float(src[e]), inv), 0.f) & 0xFFu);
+      if (lane == 0) tok_scale[prefix + i] = amax > 0.f ? __fdiv_rn(amax, 448.f) : 0.f;
+    }
+    return;
+  }
+
+  // 3. copy the chunk's live rows, one warp per row, 16-byte vectors
   for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
     const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
     const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
@@ -120,12 +173,13 @@ int prep_chunk(int P, int sm_count) {
 
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st) {
+                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale) {
   const int chunk = prep_chunk(P, sm_count);
   const int grid = (P + chunk - 1) / chunk;
   prep_rows_kernel<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
                                                   static_cast<const __nv_bfloat16*>(hidden), ld, d,
-                                                  static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows);
+                                                  static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows,
+                                                  tok_scale);
   return cudaGetLastError();
 }
 

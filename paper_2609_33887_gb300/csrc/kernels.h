@@ -20,9 +20,11 @@ struct TauParams {
 // states) and, when `hidden` is not null, packing of their bf16 rows into hc.
 // Writes idx[r] = position of compacted row r (ascending positions),
 // rowpos[p] = r or -1, hc[r] = hidden[idx[r]] and *n_rows = N.
+// With tok_scale (W8A8) the packed rows are E4M3 codes (ldc in bytes, a
+// multiple of 8) quantised per row, and tok_scale[r] receives row r's scale.
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st);
+                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale = nullptr);
 
 // Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
@@ -50,6 +52,8 @@ struct TcArgs {
   const int* draft_row = nullptr;
   float* part_t = nullptr;
   float* part_x = nullptr;
+  // W8A8 only: the dequantisation scale of each packed token row
+  const float* tok_scale = nullptr;
 };
 constexpr int TC_BM = 128;
 constexpr int TC_BN = 256;
@@ -70,7 +74,9 @@ struct PairTokenMaps {
 // NVFP4 codes decoded to bf16 inside the kernel (codes: [V, ld] bytes with
 // 128 x 128-byte SW128 boxes; NVFP4 block scales: [V, block_ld] bytes with
 // 16 x 128-byte boxes).
-enum : int { HF_BF16 = 0, HF_E4M3 = 1, HF_NVFP4 = 2 };
+// HF_W8A8: E4M3 head and E4M3 token rows (per-row scales), multiplied with
+// tcgen05.mma kind::f8f6f4 (the W8A8 variant of the precision lever).
+enum : int { HF_BF16 = 0, HF_E4M3 = 1, HF_NVFP4 = 2, HF_W8A8 = 3 };
 struct PairQuantMaps {
   CUtensorMap codes;
   CUtensorMap scales;

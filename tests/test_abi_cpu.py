@@ -121,7 +121,15 @@ def test_argument_checks(lib, kw, code):
 
 def test_variant_flags_and_outputs_checked(lib):
     assert _call(lib, variant=4) == B.BD_ERR_ARG
-    assert _call(lib, flags=1) == B.BD_ERR_ARG
+    assert _call(lib, flags=2) == B.BD_ERR_ARG
+    # W8A8 (BD_EXEC_FP8_ACTIVATIONS): E4M3 heads only, on the CTA-pair kernel, rows of 16-byte multiples
+    assert _call(lib, flags=B.BD_EXEC_FP8_ACTIVATIONS) == B.BD_ERR_ARG
+    e4 = dict(wdt=B.BD_E4M3, scale=FAKE)
+    assert _call(lib, flags=B.BD_EXEC_FP8_ACTIVATIONS | 2, **e4) == B.BD_ERR_ARG
+    assert _call(lib, variant=2, flags=B.BD_EXEC_FP8_ACTIVATIONS, **e4) == B.BD_ERR_ARG
+    assert _call(lib, variant=1, flags=B.BD_EXEC_FP8_ACTIVATIONS, **e4) == B.BD_ERR_ARG
+    assert _call(lib, flags=B.BD_EXEC_FP8_ACTIVATIONS, wld=136, **e4) == B.BD_ERR_ALIGN
+    assert _call(lib, flags=B.BD_EXEC_FP8_ACTIVATIONS, wptr=FAKE + 8, **e4) == B.BD_ERR_ALIGN
     assert _call(lib, variant=2, hdt=B.BD_F32, wdt=B.BD_F32) == B.BD_ERR_DTYPE
     assert _call(lib, outs=(None, FAKE, FAKE)) == B.BD_ERR_NULL
     assert _call(lib, outs=(FAKE + 1, FAKE, FAKE)) == B.BD_ERR_ALIGN

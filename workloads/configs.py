@@ -107,10 +107,12 @@ CONFIGS = (
 )
 
 
-# The 4-bit weight lever on the bench window (not one of the five workloads):
-# the b8x2x32 window and head shape with an NVFP4 head.
+# The precision levers on the bench window (not among the five workloads):
+# the b8x2x32 window and head shape with an NVFP4 or an E4M3 head.
 EXTRA_CONFIGS = (
     dataclasses.replace(CONFIGS[1], name="b8x2x32_d2048_v151936_nvfp4", weight_dtype="nvfp4"),
+    # the 8-bit levers on the same window: an E4M3 head (W8A16 and W8A8)
+    dataclasses.replace(CONFIGS[1], name="b8x2x32_d2048_v151936_e4m3", weight_dtype="e4m3"),
 )
 
 
