@@ -78,7 +78,7 @@ constexpr int MAX_STAGES = 8;
 constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
 constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
 constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns
-constexpr int EPI_WARPS = 4;
+constexpr int EPI_WARPS = 4;  // epilogue warps of the bf16 and decoded-head instantiations
 constexpr int TR = 34;  // padded row of the transpose buffers: 8-byte aligned rows, conflict-free column reads
 constexpr int MAX_CHUNKS = 8;
 constexpr int MAX_RAW = 8;
@@ -87,10 +87,18 @@ constexpr int CONV_WARPS = 8;                            // converter warps 6..1
 constexpr int CONV_THREADS = CONV_WARPS * 32;
 constexpr int RAW_PRODUCER = 2 + EPI_WARPS + CONV_WARPS;  // warp streaming the quantised codes
 
+// Epilogue warps: W8A8's MMAs take half the time of bf16's per tile, so two
+// warps per TMEM lane quarter (each taking every other 32-column chunk of the
+// accumulator) keep the epilogue off the critical path.
+template <int HF>
+__host__ __device__ constexpr int epi_warps() {
+  return HF == HF_W8A8 ? 2 * EPI_WARPS : EPI_WARPS;
+}
 template <int HF>
 __host__ __device__ constexpr int pair_threads() {
-  return is_quant<HF>() ? (RAW_PRODUCER + 1) * 32 : TC_THREADS;
+  return is_quant<HF>() ? (RAW_PRODUCER + 1) * 32 : (2 + epi_warps<HF>()) * 32;
 }
+static_assert(pair_threads<HF_BF16>() == TC_THREADS, "bf16 pair kernel: producer, MMA and four epilogue warps");
 // Raw ring of a quantised head: stages of 128 head rows x 128 bytes of codes
 // (SW128), plus 16 bytes of NVFP4 block scales per row.
 constexpr uint32_t RAW_CODE_BYTES = 128 * 128;
@@ -137,16 +145,16 @@ struct PairWarpBuf {
   };
 };
 
-template <bool VERIFY>
+template <bool VERIFY, int EW>
 struct PairTail {
-  PairWarpBuf<VERIFY> w[EPI_WARPS];
+  PairWarpBuf<VERIFY> w[EW];
   PairCtl ctl;
 };
 
 constexpr size_t SMEM_BYTES = 232448;  // the whole opt-in shared memory of an SM
-template <bool VERIFY>
+template <int HF, bool VERIFY>
 __host__ __device__ constexpr size_t stage_area() {
-  return SMEM_BYTES - 1024 - sizeof(PairTail<VERIFY>);
+  return SMEM_BYTES - 1024 - sizeof(PairTail<VERIFY, epi_warps<HF>()>);
 }
 
 // Stage layout for a token group of NT rows (NT/2 in each CTA), one block per
@@ -164,26 +172,26 @@ __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
 template <int HF, bool VERIFY>
 __host__ __device__ constexpr int stage_count(int nt) {
   return is_quant<HF>()
-             ? (static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt)) < QUANT_STAGES
-                    ? static_cast<int>((stage_area<VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt))
+             ? (static_cast<int>((stage_area<HF, VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt)) < QUANT_STAGES
+                    ? static_cast<int>((stage_area<HF, VERIFY>() - 3 * raw_bytes<HF>()) / stage_bytes<HF>(nt))
                     : QUANT_STAGES)
-         : static_cast<int>(stage_area<VERIFY>() / stage_bytes<HF>(nt)) < MAX_STAGES
-             ? static_cast<int>(stage_area<VERIFY>() / stage_bytes<HF>(nt))
+         : static_cast<int>(stage_area<HF, VERIFY>() / stage_bytes<HF>(nt)) < MAX_STAGES
+             ? static_cast<int>(stage_area<HF, VERIFY>() / stage_bytes<HF>(nt))
              : MAX_STAGES;
 }
 template <int HF, bool VERIFY>
 __host__ __device__ constexpr int raw_count(int nt) {
   return !is_quant<HF>() ? 0
-         : static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
+         : static_cast<int>((stage_area<HF, VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
                             raw_bytes<HF>()) < MAX_RAW
-             ? static_cast<int>((stage_area<VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
+             ? static_cast<int>((stage_area<HF, VERIFY>() - stage_count<HF, VERIFY>(nt) * stage_bytes<HF>(nt)) /
                                 raw_bytes<HF>())
              : MAX_RAW;
 }
 static_assert(stage_count<HF_BF16, false>(256) >= 3 && stage_count<HF_BF16, true>(256) >= 3, "three stages at NT = 256");
 static_assert(stage_count<HF_BF16, false>(160) == 4, "four stages at NT = 160 on the commit path");
-static_assert(stage_count<HF_W8A8, false>(160) == 8 && stage_count<HF_W8A8, false>(256) >= 6,
-              "W8A8: 26 KB stages at NT = 160");
+static_assert(stage_count<HF_W8A8, false>(160) == 7 && stage_count<HF_W8A8, false>(256) >= 5,
+              "W8A8: seven 26 KB stages at NT = 160, five 32 KB stages at NT = 256");
 static_assert(stage_count<HF_NVFP4, false>(160) == 4 && stage_count<HF_E4M3, false>(160) == 4 &&
                   stage_count<HF_NVFP4, true>(160) == 4 && stage_count<HF_E4M3, true>(160) == 4,
               "four operand stages at NT = 160 for quantised heads");
@@ -264,7 +272,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   static_assert(!(W8A8 && VERIFY), "the W8A8 variant serves the commit step");
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  PairTail<VERIFY>* tail = reinterpret_cast<PairTail<VERIFY>*>(smem + stage_area<VERIFY>());
+  constexpr int EW = epi_warps<HF>();
+  PairTail<VERIFY, EW>* tail = reinterpret_cast<PairTail<VERIFY, EW>*>(smem + stage_area<HF, VERIFY>());
   PairCtl* ctl = &tail->ctl;
   const uint32_t smem_base = smem_u32(smem);
 
@@ -301,10 +310,10 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(smem_u32(&ctl->tfull[i]), 1);
-      mbar_init(smem_u32(&ctl->tempty[i]), QUANT ? EPI_WARPS : 2 * EPI_WARPS);
+      mbar_init(smem_u32(&ctl->tempty[i]), QUANT ? EW : 2 * EW);
     }
     mbar_init(smem_u32(&ctl->drain), 1);
-    mbar_init(smem_u32(&ctl->epi_sync), EPI_WARPS * 32);
+    mbar_init(smem_u32(&ctl->epi_sync), EW * 32);
     ctl->abort_flag = 0;
     fence_mbar_init();
   }
@@ -556,8 +565,10 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     }
   } else {
     // ------------------------------------------------------ epilogue
-    const int ew = warp - 2;  // epilogue warp 0..3
+    const int ew = warp - 2;  // epilogue warp 0..EW-1
     const int quarter = warp & 3;
+    // with eight epilogue warps, warp ew takes the chunks c with c % 2 == ew / 4
+    const int chunk_par = EW == 8 ? (ew >> 2) : -1;
     const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
     float* tr = tail->w[ew].tr;
     const uint32_t tempty_local0 = smem_u32(&ctl->tempty[0]);
@@ -573,7 +584,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       int arg[MAX_CHUNKS];
       float t[MAX_CHUNKS], lx[MAX_CHUNKS];  // VERIFY only
       int xd[MAX_CHUNKS];                   // VERIFY only: draft entry of this thread's token
-      float ts[MAX_CHUNKS];                 // W8A8 only: this thread's token scale (1 for an all-zero row)
+      // W8A8: this thread's token scale ts (1 for an all-zero row). The
+      // running max m is kept in unscaled accumulator units (ts > 0 keeps
+      // the max and argmax), the exponents use k2 = ts * log2(e), and the
+      // partial max is scaled by ts when written.
+      float ts[MAX_CHUNKS], k2[MAX_CHUNKS];
 #pragma unroll
       for (int c = 0; c < MAX_CHUNKS; ++c) {
         m[c] = -INFINITY;
@@ -587,6 +602,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
           const int row = it.m_tile * NT + c * 32 + lane;
           if (c < nch && row < n_rows && a.tok_scale[row] != 0.f) ts[c] = a.tok_scale[row];
         }
+        k2[c] = ts[c] * LOG2E;
         if constexpr (VERIFY) {
           const int row = it.m_tile * NT + c * 32 + lane;
           if (c < nch && row < n_rows) xd[c] = a.draft_row[row];
@@ -605,7 +621,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         const float sc = (scaled && !dead) ? __ldg(a.wscale + my_v) : 1.f;
 #pragma unroll
         for (int c = 0; c < MAX_CHUNKS; ++c) {
-          if (c < nch) {
+          if (c < nch && (chunk_par < 0 || (c & 1) == chunk_par)) {
             float v[32];
             tmem_ld32(tmem_base + lane_addr + acc * 256 + c * 32, v);
             // this lane's row of the transpose, two floats per store; the mask
@@ -625,11 +641,6 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             float x[32];
 #pragma unroll
             for (int r = 0; r < 32; ++r) x[r] = tr[r * TR + lane];
-            if constexpr (W8A8) {
-              // the token row's dequantisation scale (an all-zero row has logits 0 already)
-#pragma unroll
-              for (int r = 0; r < 32; ++r) x[r] *= ts[c];
-            }
             if constexpr (VERIFY) {
               const int rel = xd[c] - vrow0;
               if (rel >= 0 && rel < 32) lx[c] = tr[rel * TR + lane];
@@ -656,12 +667,12 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
                   s[c] *= f;
                 }
               } else {
-                s[c] = (m[c] == -INFINITY) ? 0.f : s[c] * ex2_approx((m[c] - cm) * LOG2E);
+                s[c] = (m[c] == -INFINITY) ? 0.f : s[c] * ex2_approx((m[c] - cm) * k2[c]);
               }
               m[c] = cm;
             }
             if (m[c] != -INFINITY) {
-              const float mc = m[c] * LOG2E;
+              const float mc = m[c] * k2[c];
               if constexpr (VERIFY) {
                 // -inf logits give u = -inf, e = 0; clamping u keeps e * u at 0
                 float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
@@ -680,8 +691,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
                 float s0 = 0.f, s1 = 0.f;
 #pragma unroll
                 for (int r = 0; r < 32; r += 2) {
-                  s0 += ex2_approx(fmaf(x[r], LOG2E, -mc));
-                  s1 += ex2_approx(fmaf(x[r + 1], LOG2E, -mc));
+                  s0 += ex2_approx(fmaf(x[r], k2[c], -mc));
+                  s1 += ex2_approx(fmaf(x[r + 1], k2[c], -mc));
                 }
                 s[c] += s0 + s1;
               }
@@ -705,8 +716,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       // combine the four warps' running states and write this CTA's partials
 #pragma unroll
       for (int c = 0; c < MAX_CHUNKS; ++c) {
-        if (c < nch) {
-          tail->w[ew].st.m[c * 32 + lane] = m[c];
+        if (c < nch && (chunk_par < 0 || (c & 1) == chunk_par)) {
+          tail->w[ew].st.m[c * 32 + lane] = W8A8 ? m[c] * ts[c] : m[c];
           tail->w[ew].st.s[c * 32 + lane] = s[c];
           tail->w[ew].st.a[c * 32 + lane] = arg[c];
           if constexpr (VERIFY) {
@@ -718,16 +729,19 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       mbar_arrive(epi_sync);
       if (!mbar_wait_warp(epi_sync, epi_phase, abort_flag, a.status)) break;
       epi_phase ^= 1u;
-      for (int j = ew * 32 + lane; j < NT; j += EPI_WARPS * 32) {
-        float M = tail->w[0].st.m[j], S = tail->w[0].st.s[j];
-        int A = tail->w[0].st.a[j];
+      for (int j = ew * 32 + lane; j < NT; j += EW * 32) {
+        // the four warps (one per lane quarter) that hold token j's states
+        const int w0 = EW == 8 ? 4 * ((j >> 5) & 1) : 0;
+        float M = tail->w[w0].st.m[j], S = tail->w[w0].st.s[j];
+        int A = tail->w[w0].st.a[j];
         float T = 0.f, LX = -INFINITY;
         if constexpr (VERIFY) {
-          T = tail->w[0].st.t[j];
-          LX = tail->w[0].st.x[j];
+          T = tail->w[w0].st.t[j];
+          LX = tail->w[w0].st.x[j];
         }
 #pragma unroll
-        for (int w = 1; w < EPI_WARPS; ++w) {
+        for (int q = 1; q < 4; ++q) {
+          const int w = w0 + q;
           if constexpr (VERIFY) {
             softmax_combine_t(M, S, A, T, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j],
                               tail->w[w].st.t[j]);
