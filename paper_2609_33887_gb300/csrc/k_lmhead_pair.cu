@@ -77,7 +77,8 @@ __host__ __device__ constexpr int atom_cols() {
 constexpr int MAX_STAGES = 8;
 constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
 constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
-constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns
+constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns, or three of up to 160
+constexpr int MAX_ACC = 3;
 constexpr int EPI_WARPS = 4;  // epilogue warps of the bf16 and decoded-head instantiations
 constexpr int TR = 34;  // padded row of the transpose buffers: 8-byte aligned rows, conflict-free column reads
 constexpr int MAX_CHUNKS = 8;
@@ -115,8 +116,8 @@ __host__ __device__ constexpr int raw_k() {
 struct PairCtl {
   uint64_t full[MAX_STAGES];
   uint64_t empty[MAX_STAGES];
-  uint64_t tfull[2];
-  uint64_t tempty[2];
+  uint64_t tfull[MAX_ACC];
+  uint64_t tempty[MAX_ACC];
   uint64_t drain;
   uint64_t epi_sync;  // rendezvous of the 128 epilogue threads (bounded, unlike bar.sync)
   uint64_t rfull[MAX_RAW];   // quantised heads: raw codes landed (TMA transaction bytes)
@@ -308,7 +309,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       mbar_init(smem_u32(&ctl->full[s]), QUANT ? 1 + CONV_WARPS : 1);
       mbar_init(smem_u32(&ctl->empty[s]), 1);
     }
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < MAX_ACC; ++i) {
       mbar_init(smem_u32(&ctl->tfull[i]), 1);
       mbar_init(smem_u32(&ctl->tempty[i]), QUANT ? EW : 2 * EW);
     }
@@ -343,6 +344,10 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   const int nk = cdiv(a.d, BK);
   const int NT = pair_group_rows(n_rows);
   const int half = NT / 2;
+  // accumulators in TMEM: three of 160 columns when a group has at most 160
+  // tokens (the epilogue of one tile then overlaps two tiles of MMAs), else two of 256
+  const uint32_t NACC = NT <= 160 ? 3u : 2u;
+  const uint32_t ACC_COLS = NT <= 160 ? 160u : 256u;
   const int nch = NT / 32;
   const uint32_t SB = stage_bytes<HF>(NT);
   const uint32_t B_BLOCK = static_cast<uint32_t>(half) * ATOM_ROWS_BYTES;
@@ -426,7 +431,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + acc * 256;
+          const uint32_t d_tmem = tmem_base + acc * ACC_COLS;
           for (int kb = 0; kb < nk; ++kb) {
             if (!mbar_wait_warp(smem_u32(&ctl->full[stage]), phase, abort_flag, a.status)) {
               ok = false;
@@ -469,7 +474,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
               umma_commit_pair_mc(smem_u32(&ctl->tfull[acc]), 0x3);
           }
           __syncwarp();
-          if (++acc == 2) {
+          if (++acc == NACC) {
             acc = 0;
             acc_phase ^= 1u;
           }
@@ -623,7 +628,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         for (int c = 0; c < MAX_CHUNKS; ++c) {
           if (c < nch && (chunk_par < 0 || (c & 1) == chunk_par)) {
             float v[32];
-            tmem_ld32(tmem_base + lane_addr + acc * 256 + c * 32, v);
+            tmem_ld32(tmem_base + lane_addr + acc * ACC_COLS + c * 32, v);
             // this lane's row of the transpose, two floats per store; the mask
             // entry and rows past V are -inf, the e4m3 row scale applies to live rows
             float2* row = reinterpret_cast<float2*>(tr + lane * TR);
@@ -707,7 +712,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
           else
             mbar_arrive_cluster(tempty_leader0 + 8u * acc);
         }
-        if (++acc == 2) {
+        if (++acc == NACC) {
           acc = 0;
           acc_phase ^= 1u;
         }
