@@ -359,10 +359,10 @@ def verify_timing(dev, stream) -> dict:
 LEVERS = {
     # key: (workload, description of the LM-head path and what bounds it)
     "nvfp4": ("b8x2x32_d2048_v151936_nvfp4",
-              "codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA); "
-              "bound: the converter warps' instruction issue"),
+              "codes streamed by TMA and decoded exactly to f16 inside the LM-head kernel (f16 MMA, token rows "
+              "scaled by a power of two per row); bound: the converter warps"),
     "e4m3": ("b8x2x32_d2048_v151936_e4m3",
-             "W8A16: E4M3 codes streamed by TMA and decoded to bf16 inside the LM-head kernel (bf16 MMA)"),
+             "W8A16: E4M3 codes streamed by TMA and decoded exactly to f16 inside the LM-head kernel (f16 MMA)"),
     "w8a8": ("b8x2x32_d2048_v151936_e4m3",
              "W8A8: packed rows quantised to E4M3 per row by the compaction kernel, E4M3 x E4M3 on the "
              "8-bit tensor path (tcgen05.mma kind::f8f6f4), both scales applied to the fp32 logits"),

@@ -420,12 +420,14 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   }
 
   // a0: compaction of the masked positions of active blocks (+ packing of their rows)
-  // (W8A8: the packed rows are quantised to E4M3 with one scale per row)
-  float* tsc = c.fp8_act ? reinterpret_cast<float*>(ws + lay.tsc) : nullptr;
+  // W8A8: the packed rows are quantised to E4M3 with one scale per row; a
+  // head decoded inside the LM head: f16 rows scaled by a power of two per row
+  const int row_format = c.fp8_act ? bd::ROWS_E4M3 : c.fused ? bd::ROWS_F16_POW2 : bd::ROWS_BF16;
+  float* tsc = row_format != bd::ROWS_BF16 ? reinterpret_cast<float*>(ws + lay.tsc) : nullptr;
   const int64_t ld_rows = c.fp8_act ? ld_fp8_rows(c) : c.ldc;
   int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
                                             c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
-                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc));
+                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc, row_format));
   if (rc != BD_OK) return rc;
 
   rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, ld_rows, ws + lay.wq, idx, n_rows, nullptr,

@@ -429,6 +429,11 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
          (static_cast<uint32_t>(M >> 4) << 24);
 }
 
+// The same with f16 A and B (format code 0 in bits 7-9 and 10-12).
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4) | (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
 // Instruction descriptor of tcgen05.mma kind::f8f6f4 with E4M3 A and B
 // (format code 0 in bits 7-9 and 10-12), fp32 accumulator, both operands
 // K-major; N >> 3 in bits 17-22, M >> 4 in bits 24-28.

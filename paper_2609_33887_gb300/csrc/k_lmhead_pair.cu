@@ -202,9 +202,10 @@ static_assert(stage_count<HF_NVFP4, true>(256) >= 3 && stage_count<HF_E4M3, true
 
 // Decodes this thread's share of one operand stage (128 head rows x 64
 // columns, global columns kcol0..) from the raw stage at raw_base into the
-// bf16 A tile at a_base (one SW128 atom). h: which 64-column part of the raw
-// stage. Columns at or past d decode to zero. ct: 0..CONV_THREADS-1.
-template <int HF>
+// f16 (F16) or bf16 A tile at a_base (one SW128 atom); both are exact. h:
+// which 64-column part of the raw stage. Columns at or past d decode to zero.
+// ct: 0..CONV_THREADS-1.
+template <int HF, bool F16>
 __device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t a_base, int ct, int kcol0, int d) {
   static_assert(!is_quant<HF>() || stage_k<HF>() == 64, "one atom per quantised operand stage");
   if constexpr (HF == HF_NVFP4) {
@@ -220,7 +221,10 @@ __device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t
       uint32_t w[16];
 #pragma unroll
       for (int b = 0; b < 16; ++b)  // byte b: elements 2b (low nibble), 2b + 1; 16 elements per block scale
-        w[b] = f16x2_to_bf16x2(hmul2_u32(e2m1x2_to_f16x2(__byte_perm(words[b >> 2], 0, 0x4440 + (b & 3))), sc[b >> 3]));
+      {
+        const uint32_t hv = hmul2_u32(e2m1x2_to_f16x2(__byte_perm(words[b >> 2], 0, 0x4440 + (b & 3))), sc[b >> 3]);
+        w[b] = F16 ? hv : f16x2_to_bf16x2(hv);
+      }
       const int col0 = kcol0 + j * 32;
       if (col0 + 32 > d) {
 #pragma unroll
@@ -245,7 +249,10 @@ __device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t
       uint32_t w[8];
 #pragma unroll
       for (int b = 0; b < 8; ++b)  // bytes 2b, 2b + 1: elements 2b, 2b + 1
-        w[b] = f16x2_to_bf16x2(e4m3x2_to_f16x2(__byte_perm(words[b >> 1], 0, (b & 1) ? 0x4432 : 0x4410)));
+      {
+        const uint32_t hv = e4m3x2_to_f16x2(__byte_perm(words[b >> 1], 0, (b & 1) ? 0x4432 : 0x4410));
+        w[b] = F16 ? hv : f16x2_to_bf16x2(hv);
+      }
       const int col0 = kcol0 + j * 16;
       if (col0 + 16 > d) {
 #pragma unroll
@@ -271,6 +278,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   constexpr bool QUANT = is_quant<HF>();
   constexpr bool W8A8 = HF == HF_W8A8;
   static_assert(!(W8A8 && VERIFY), "the W8A8 variant serves the commit step");
+  // commit step with a head decoded in the kernel: f16 operands (the decode
+  // ends at f16), token rows pre-scaled by a power of two per row
+  constexpr bool F16OPS = QUANT && !VERIFY;
+  // the packed rows carry a per-row scale that multiplies their logits
+  constexpr bool TOKS = W8A8 || F16OPS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr int EW = epi_warps<HF>();
@@ -418,7 +430,9 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     // ------------------------------------------------------ MMA issuer (even CTA; every CTA for quantised heads)
     if (rank == 0 || QUANT) {
       const bool leader = elect_one();
-      const uint32_t idesc = W8A8 ? idesc_e4m3_f32(256, NT) : idesc_bf16_f32(QUANT ? 128 : 256, NT);
+      const uint32_t idesc = W8A8     ? idesc_e4m3_f32(256, NT)
+                             : F16OPS ? idesc_f16_f32(128, NT)
+                                      : idesc_bf16_f32(QUANT ? 128 : 256, NT);
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
@@ -550,7 +564,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             ok = false;
             break;
           }
-          convert_stage<HF>(raw_base + r * raw_bytes<HF>(), h, smem_base + stage * SB, ct, kb * BK, a.d);
+          convert_stage<HF, F16OPS>(raw_base + r * raw_bytes<HF>(), h, smem_base + stage * SB, ct, kb * BK, a.d);
           fence_proxy_async_smem();
           __syncwarp();
           if (lane == 0) mbar_arrive(smem_u32(&ctl->full[stage]));
@@ -589,7 +603,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       int arg[MAX_CHUNKS];
       float t[MAX_CHUNKS], lx[MAX_CHUNKS];  // VERIFY only
       int xd[MAX_CHUNKS];                   // VERIFY only: draft entry of this thread's token
-      // W8A8: this thread's token scale ts (1 for an all-zero row). The
+      // W8A8 and f16 rows: this thread's token scale ts (1 for an all-zero row). The
       // running max m is kept in unscaled accumulator units (ts > 0 keeps
       // the max and argmax), the exponents use k2 = ts * log2(e), and the
       // partial max is scaled by ts when written.
@@ -603,7 +617,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         lx[c] = -INFINITY;
         xd[c] = -1;
         ts[c] = 1.f;
-        if constexpr (W8A8) {
+        if constexpr (TOKS) {
           const int row = it.m_tile * NT + c * 32 + lane;
           if (c < nch && row < n_rows && a.tok_scale[row] != 0.f) ts[c] = a.tok_scale[row];
         }
@@ -722,7 +736,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
 #pragma unroll
       for (int c = 0; c < MAX_CHUNKS; ++c) {
         if (c < nch && (chunk_par < 0 || (c & 1) == chunk_par)) {
-          tail->w[ew].st.m[c * 32 + lane] = W8A8 ? m[c] * ts[c] : m[c];
+          tail->w[ew].st.m[c * 32 + lane] = TOKS ? m[c] * ts[c] : m[c];
           tail->w[ew].st.s[c * 32 + lane] = s[c];
           tail->w[ew].st.a[c * 32 + lane] = arg[c];
           if constexpr (VERIFY) {

@@ -20,11 +20,16 @@ struct TauParams {
 // states) and, when `hidden` is not null, packing of their bf16 rows into hc.
 // Writes idx[r] = position of compacted row r (ascending positions),
 // rowpos[p] = r or -1, hc[r] = hidden[idx[r]] and *n_rows = N.
-// With tok_scale (W8A8) the packed rows are E4M3 codes (ldc in bytes, a
-// multiple of 8) quantised per row, and tok_scale[r] receives row r's scale.
+// Packed row formats. ROWS_E4M3 (W8A8): E4M3 codes (ldc in bytes, a multiple
+// of 8) quantised per row, tok_scale[r] = row r's dequantisation scale.
+// ROWS_F16_POW2 (heads decoded to f16 in the LM head): f16 rows (ldc in
+// elements) holding the bf16 values times 2^s_r, s_r chosen so the row's
+// largest magnitude lands in [2^14, 2^15), tok_scale[r] = 2^-s_r (exact).
+enum : int { ROWS_BF16 = 0, ROWS_E4M3 = 1, ROWS_F16_POW2 = 2 };
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale = nullptr);
+                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale = nullptr,
+                             int row_format = ROWS_BF16);
 
 // Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
