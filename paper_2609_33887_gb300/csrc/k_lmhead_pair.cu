@@ -19,28 +19,41 @@
 // epilogue warp owns 32 lanes; per 32 token columns it moves its 32 x 32
 // logits through a shared-memory transpose so that each thread holds one
 // token's 32 logits, and keeps a running (max, sum of exponentials, argmax)
-// per token across the v-tiles of its unit. The four warps' states are
-// combined once per unit, and each CTA writes its own partial per token.
+// per token across the v-tiles of its unit. The warps' states are combined
+// once per unit, and each CTA writes its own partial per token. Accumulators
+// live in TMEM: three of 160 columns for groups of at most 160 tokens (the
+// epilogue of one tile overlaps two tiles of MMAs), else two of 256.
 //
-// CTA layout (192 threads): warp 0 TMA producer, warp 1 TMEM allocation (both
-// CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue. The producer and
-// issuer loops run in the whole warp and one elected lane issues, which keeps
-// the MMA issue rate at the tensor pipe's rate (N = 160: 80 cycles per MMA).
-// Every wait is bounded (see common.cuh).
+// CTA layout (bf16 heads, 192 threads): warp 0 TMA producer, warp 1 TMEM
+// allocation (both CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue.
+// The producer and issuer loops run in the whole warp and one elected lane
+// issues, which keeps the MMA issue rate at the tensor pipe's rate (N = 160:
+// 80 cycles per MMA). Every wait is bounded (see common.cuh).
 //
 // The verification instantiation (VERIFY = true, speculative decoding) also
 // carries, per token, the entropy accumulator sum exp(l - m) (l - m) log2(e)
 // and the logit of the token's draft entry (typical-acceptance appendix); its
 // larger combine buffers cost shared memory, so it may run one stage fewer.
 //
-// Quantised heads (HF = HF_E4M3, HF_NVFP4: the precision levers) are decoded
-// inside the kernel, so HBM carries the stored head only: a raw-code producer
-// warp streams this CTA's head codes (and NVFP4 block scales) with TMA into a
-// small ring, and four converter warps decode them exactly into the bf16
-// operand tile of the stage, in the tile's 128-byte-swizzled layout. The
-// operand stage is full when both CTAs' converters (eight warp arrivals) and
-// the token rows' transaction bytes have landed. E4M3 raw stages hold 128
-// columns of d, NVFP4 raw stages 256 (128 bytes of codes per row either way).
+// W8A8 (HF = HF_W8A8): E4M3 head rows times E4M3 token rows (quantised per
+// row by the compaction kernel) with tcgen05.mma kind::f8f6f4, K = 32 per
+// MMA, one 128-column (128-byte) atom per stage; an 8-bit tile takes half the
+// tensor time of a bf16 one, so the epilogue has eight warps (two per lane
+// quarter, alternate 32-column chunks; 320 threads). Each token's scale
+// multiplies its logits through the exponent's factor.
+//
+// Heads decoded in the kernel (HF = HF_E4M3, HF_NVFP4: the precision levers):
+// HBM carries the stored head only. A raw-code producer warp streams this
+// CTA's head codes (and NVFP4 block scales) with TMA into a raw ring, and
+// eight converter warps decode them exactly into the operand tile of each
+// 64-column stage, in its 128-byte-swizzled layout: f16 on the commit step
+// (the token rows then come as f16 scaled by a power of two per row, undone
+// on the logits like W8A8's scales), bf16 for verification. Each CTA
+// multiplies its 128 head rows by all NT token rows with cta_group::1 MMAs,
+// so converters signal only their own CTA; the operand stage is full when
+// its eight converter warps have arrived and the token rows' bytes have
+// landed. E4M3 raw stages hold 128 columns of d, NVFP4 raw stages 256 (128
+// bytes of codes per row either way); 480 threads.
 #include <atomic>
 #include <cstring>
 
@@ -62,8 +75,8 @@ template <int HF>
 __host__ __device__ constexpr bool pair_cluster() {
   return !is_quant<HF>();
 }
-// columns of d per operand stage: two 64-column bf16 swizzle atoms for bf16
-// heads; one 128-column 8-bit atom for W8A8; one bf16 atom for heads decoded
+// columns of d per operand stage: two 64-column 16-bit swizzle atoms for bf16
+// heads; one 128-column 8-bit atom for W8A8; one 16-bit atom for heads decoded
 // in the kernel, whose small stages leave room for a deep raw ring
 template <int HF>
 __host__ __device__ constexpr int stage_k() {
@@ -75,8 +88,8 @@ __host__ __device__ constexpr int atom_cols() {
   return HF == HF_W8A8 ? 128 : 64;
 }
 constexpr int MAX_STAGES = 8;
-constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a 64-column bf16 atom
-constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x 64 columns
+constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a swizzle atom (64 16-bit or 128 8-bit columns)
+constexpr uint32_t A_BLOCK = 128 * ATOM_ROWS_BYTES;  // this CTA's 128 head rows x one atom
 constexpr uint32_t TMEM_COLS = 512;  // two accumulators of up to 256 columns, or three of up to 160
 constexpr int MAX_ACC = 3;
 constexpr int EPI_WARPS = 4;  // epilogue warps of the bf16 and decoded-head instantiations
@@ -159,8 +172,9 @@ __host__ __device__ constexpr size_t stage_area() {
 }
 
 // Stage layout for a token group of NT rows (NT/2 in each CTA), one block per
-// 64-column atom: [A block 0 (| A block 1) | B block 0 (| B block 1)],
-// A = 128 head rows, B = NT/2 token rows, each block 1 KB aligned.
+// atom: [A block 0 (| A block 1) | B block 0 (| B block 1)], A = 128 head
+// rows, B = NT/2 token rows (all NT for heads decoded in the kernel), each
+// block 1 KB aligned.
 template <int HF>
 __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
   // heads decoded in the kernel: one CTA multiplies its 128 head rows by all NT token rows
