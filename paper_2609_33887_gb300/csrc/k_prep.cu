@@ -43,11 +43,11 @@ __device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
   return r;
 }
 
+template <int FMT>  // the packed row format (ROWS_*); one instantiation per format
 __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags, int P, int block_len, int chunk,
     const __nv_bfloat16* __restrict__ hidden, int64_t ld, int d, __nv_bfloat16* __restrict__ hc, int64_t ldc,
-    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale,
-    int row_format) {
+    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale) {
   __shared__ int red[PREP_THREADS / 32];
   __shared__ int warp_excl[PREP_THREADS / 32];
   __shared__ int rows_s[2048];
@@ -107,7 +107,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
   __syncthreads();
 
   const int nvec = d / 8;
-  if (row_format == ROWS_F16_POW2) {
+  if constexpr (FMT == ROWS_F16_POW2) {
     // 3''. f16 rows for an LM head whose operands are f16: row r holds
     // h * 2^s with s = 15 - e for max |h| in [2^(e-1), 2^e) (so the largest
     // magnitude lands in [2^14, 2^15) and every bf16 value at or above 2^-14
@@ -130,9 +130,11 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       for (int e = nvec * 8 + lane; e < d; e += 32) amax = fmaxf(amax, fabsf(__bfloat162float(src[e])));
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-      int e2 = 0;
-      frexpf(amax, &e2);
-      const int sh = amax > 0.f ? min(15 - e2, 126) : 0;
+      // biased exponent E of amax: amax in [2^(E-127), 2^(E-126)) for E > 0,
+      // so s = 15 - (E - 126); E = 0 (zero or below 2^-126) takes the cap
+      const int E = static_cast<int>(__float_as_uint(amax) >> 23);
+      const int sh = amax > 0.f ? min(141 - E, 126) : 0;
+      const float up = __uint_as_float(static_cast<uint32_t>(sh + 127) << 23);  // 2^s, exact
       __half* dst = reinterpret_cast<__half*>(hc) + static_cast<int64_t>(prefix + i) * ldc;
       uint4* d4 = reinterpret_cast<uint4*>(dst);
       for (int v = lane; v < nvec; v += 32) {
@@ -142,17 +144,17 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
           const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[j]));
-          const __half2 h2 = __floats2half2_rn(ldexpf(f.x, sh), ldexpf(f.y, sh));
+          const __half2 h2 = __floats2half2_rn(f.x * up, f.y * up);
           o[j] = *reinterpret_cast<const uint32_t*>(&h2);
         }
         d4[v] = make_uint4(o[0], o[1], o[2], o[3]);
       }
-      for (int e = nvec * 8 + lane; e < d; e += 32) dst[e] = __float2half_rn(ldexpf(__bfloat162float(src[e]), sh));
-      if (lane == 0) tok_scale[prefix + i] = amax > 0.f ? ldexpf(1.f, -sh) : 0.f;
+      for (int e = nvec * 8 + lane; e < d; e += 32) dst[e] = __float2half_rn(__bfloat162float(src[e]) * up);
+      if (lane == 0) tok_scale[prefix + i] = amax > 0.f ? __uint_as_float(static_cast<uint32_t>(127 - sh) << 23) : 0.f;
     }
     return;
   }
-  if (row_format == ROWS_E4M3) {
+  if constexpr (FMT == ROWS_E4M3) {
     // 3'. W8A8: quantise the chunk's live rows to E4M3 with one scale per row,
     // one warp per row: a = max |h|, inv = 448 / a, code = e4m3(h * inv) (round
     // to nearest even, saturating), scale = a / 448; an all-zero row gets codes
@@ -223,10 +225,12 @@ cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_fla
   if (row_format != ROWS_BF16 && (tok_scale == nullptr || hc == nullptr)) return cudaErrorInvalidValue;
   const int chunk = prep_chunk(P, sm_count);
   const int grid = (P + chunk - 1) / chunk;
-  prep_rows_kernel<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
-                                                  static_cast<const __nv_bfloat16*>(hidden), ld, d,
-                                                  static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows,
-                                                  tok_scale, row_format);
+  auto* kern = row_format == ROWS_F16_POW2 ? prep_rows_kernel<ROWS_F16_POW2>
+               : row_format == ROWS_E4M3  ? prep_rows_kernel<ROWS_E4M3>
+                                          : prep_rows_kernel<ROWS_BF16>;
+  kern<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
+                                      static_cast<const __nv_bfloat16*>(hidden), ld, d,
+                                      static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows, tok_scale);
   return cudaGetLastError();
 }
 
