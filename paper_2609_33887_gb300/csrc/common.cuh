@@ -22,6 +22,13 @@ constexpr uint64_t WAIT_LIMIT_NS = 1000000000ull;  // 1 s
 constexpr uint64_t DRAIN_LIMIT_NS = 100000000ull;  // 0.1 s
 
 constexpr float LOG2E = 1.4426950408889634f;
+// The epilogues form the exponent of exp(l - m) as fmaf(l, log2 e, -mc) with
+// mc = fl32(m log2 e): one instruction, but every exponent then carries mc's
+// rounding error (up to half an ulp of m log2 e), which at the maximum itself
+// should be 0. Below this magnitude of mc that error stays under 2^-13
+// (relative error 1e-4 in the sum); states with a larger running max (logits
+// beyond ~1400) form (l - m) log2 e instead, exact at l = m.
+constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 
 // -------------------------------------------------------------------------
 // Work plan of the LM-head kernels.

@@ -706,12 +706,14 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             }
             if (m[c] != -INFINITY) {
               const float mc = m[c] * k2[c];
+              const bool wide = !(fabsf(mc) < FUSED_SHIFT_LIMIT);  // take x - m first (see common.cuh)
               if constexpr (VERIFY) {
                 // -inf logits give u = -inf, e = 0; clamping u keeps e * u at 0
                 float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
                 for (int r = 0; r < 32; r += 2) {
-                  const float u0 = fmaf(x[r], LOG2E, -mc), u1 = fmaf(x[r + 1], LOG2E, -mc);
+                  const float u0 = wide ? (x[r] - m[c]) * k2[c] : fmaf(x[r], k2[c], -mc);
+                  const float u1 = wide ? (x[r + 1] - m[c]) * k2[c] : fmaf(x[r + 1], k2[c], -mc);
                   const float e0 = ex2_approx(u0), e1 = ex2_approx(u1);
                   s0 += e0;
                   s1 += e1;
@@ -722,10 +724,18 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
                 t[c] += t0 + t1;
               } else {
                 float s0 = 0.f, s1 = 0.f;
+                if (!wide) {
 #pragma unroll
-                for (int r = 0; r < 32; r += 2) {
-                  s0 += ex2_approx(fmaf(x[r], k2[c], -mc));
-                  s1 += ex2_approx(fmaf(x[r + 1], k2[c], -mc));
+                  for (int r = 0; r < 32; r += 2) {
+                    s0 += ex2_approx(fmaf(x[r], k2[c], -mc));
+                    s1 += ex2_approx(fmaf(x[r + 1], k2[c], -mc));
+                  }
+                } else {
+#pragma unroll
+                  for (int r = 0; r < 32; r += 2) {
+                    s0 += ex2_approx((x[r] - m[c]) * k2[c]);
+                    s1 += ex2_approx((x[r + 1] - m[c]) * k2[c]);
+                  }
                 }
                 s[c] += s0 + s1;
               }

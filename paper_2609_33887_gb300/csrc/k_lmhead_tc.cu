@@ -258,11 +258,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
           }
           if (m != -INFINITY) {
             const float mc = m * LOG2E;
+            const bool wide = !(fabsf(mc) < FUSED_SHIFT_LIMIT);  // take v - m first (see common.cuh)
             if constexpr (VERIFY) {
               float s0 = 0.f, s1 = 0.f, t0 = 0.f, t1 = 0.f;
 #pragma unroll
               for (int j = 0; j < 32; j += 2) {
-                const float u0 = fmaf(v[j], LOG2E, -mc), u1 = fmaf(v[j + 1], LOG2E, -mc);
+                const float u0 = wide ? (v[j] - m) * LOG2E : fmaf(v[j], LOG2E, -mc);
+                const float u1 = wide ? (v[j + 1] - m) * LOG2E : fmaf(v[j + 1], LOG2E, -mc);
                 const float e0 = ex2_approx(u0), e1 = ex2_approx(u1);
                 s0 += e0;
                 s1 += e1;
@@ -273,10 +275,18 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
               t += t0 + t1;
             } else {
               float s0 = 0.f, s1 = 0.f;
+              if (!wide) {
 #pragma unroll
-              for (int j = 0; j < 32; j += 2) {
-                s0 += ex2_approx(fmaf(v[j], LOG2E, -mc));
-                s1 += ex2_approx(fmaf(v[j + 1], LOG2E, -mc));
+                for (int j = 0; j < 32; j += 2) {
+                  s0 += ex2_approx(fmaf(v[j], LOG2E, -mc));
+                  s1 += ex2_approx(fmaf(v[j + 1], LOG2E, -mc));
+                }
+              } else {
+#pragma unroll
+                for (int j = 0; j < 32; j += 2) {
+                  s0 += ex2_approx((v[j] - m) * LOG2E);
+                  s1 += ex2_approx((v[j + 1] - m) * LOG2E);
+                }
               }
               s += s0 + s1;
             }

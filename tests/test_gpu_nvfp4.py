@@ -1,11 +1,14 @@
 """NVFP4 heads (the 4-bit weight lever) on the GPU against the float64 oracle.
 
-The library decodes every E2M1 x E4M3 product exactly to bf16 and applies the
-per-row scale to the fp32 logit, so the bf16 path's tolerances apply (tokens
-and commit bits exact away from near-ties, confidence within 2e-3). The CTA-pair
-kernel decodes the codes itself when code and block-scale rows start on
-16-byte boundaries (BD_FUSED_DECODE, default on), and otherwise from a bf16
-copy decoded beforehand; both are checked.
+The library decodes every E2M1 x E4M3 product exactly (to f16 inside the
+commit step's LM head, to bf16 elsewhere) and applies the per-row scale to the
+fp32 logit, so the bf16 path's tolerances apply (tokens and commit bits exact
+away from near-ties, confidence within 2e-3). The CTA-pair kernel decodes the
+codes itself when code and block-scale rows start on 16-byte boundaries
+(BD_FUSED_DECODE, default on), and otherwise from a bf16 copy decoded
+beforehand; both are checked. In the first case the token rows travel as f16
+scaled by a power of two per row, so rows spanning the bf16 exponent range
+are checked too.
 """
 
 import numpy as np
@@ -122,3 +125,18 @@ def test_verify_with_nvfp4_head():
     assert np.all((g["tokens"] == ref["tokens"]) | near)
     assert np.max(np.abs(g["p_draft"] - ref["p_draft"])) <= 2e-3
     assert np.max(np.abs(g["entropy"] - ref["entropy"])) <= 1e-2
+
+
+def scale_rows_by_powers_of_two(wl, exps=(-90, -40, -12, 0, 12, 40, 90)):
+    """Hidden rows multiplied by 2^k (exact in bf16), k cycling over exps."""
+    k = torch.tensor(exps, dtype=torch.float64)[torch.arange(wl.hidden.shape[0]) % len(exps)]
+    wl.hidden = (wl.hidden.double() * torch.exp2(k)[:, None]).to(wl.hidden.dtype)
+    return wl
+
+
+@pytest.mark.parametrize("fused", [True, False])
+def test_row_magnitudes_across_the_bf16_range(fused, monkeypatch):
+    if not fused:
+        monkeypatch.setenv("BD_FUSED_DECODE", "0")
+    rep = check(scale_rows_by_powers_of_two(generate(SMALL["r294_d320"])), variant=3)
+    assert rep.n_live > 0

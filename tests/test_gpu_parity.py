@@ -110,6 +110,16 @@ def test_e4m3_pair_fused_and_decoded(name, fused, monkeypatch):
     check(generate(SMALL[name]), variant=3)
 
 
+def test_e4m3_pair_fused_row_magnitudes():
+    # the fused E4M3 path packs the token rows as f16 scaled by a power of two
+    # per row: rows spanning the bf16 exponent range
+    wl = generate(SMALL["e4m3_ktail"])
+    exps = (-90, -40, -12, 0, 12, 40, 90)
+    k = torch.tensor(exps, dtype=torch.float64)[torch.arange(wl.hidden.shape[0]) % len(exps)]
+    wl.hidden = (wl.hidden.double() * torch.exp2(k)[:, None]).to(wl.hidden.dtype)
+    check(wl, variant=3)
+
+
 @pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "e4m3"])
 def test_small_simt_variant(name):
     wl = generate(SMALL[name])

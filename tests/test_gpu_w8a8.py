@@ -128,3 +128,13 @@ def test_w8a8_full_window_and_deviation():
     print(f"W8A8 vs exact: token agreement {agree:.4f}, max |dconf| {dconf:.4f}, live {int(live.sum())}")
     assert agree >= 0.97
     assert dconf <= 0.1
+
+
+def test_w8a8_row_magnitudes_across_the_bf16_range():
+    """Per-row scales from 2^-90 to 2^90 times the generated rows (exact in bf16)."""
+    wl = generate(SMALL["e4m3_g294_ktail"])
+    exps = (-90, -40, -12, 0, 12, 40, 90)
+    k = torch.tensor(exps, dtype=torch.float64)[torch.arange(wl.hidden.shape[0]) % len(exps)]
+    wl.hidden = (wl.hidden.double() * torch.exp2(k)[:, None]).to(wl.hidden.dtype)
+    _, rep = check(wl)
+    assert rep.n_live > 0
