@@ -31,9 +31,9 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from workloads import CONFIGS, by_name, generate  # noqa: E402
+from workloads import B8X2X32_BF16, by_name, generate  # noqa: E402
 
-DEFAULT_CONFIG = CONFIGS[1].name
+DEFAULT_CONFIG = B8X2X32_BF16.name
 METRIC = "masked positions/s through fused LM-head+confidence+commit"
 UNIT = "positions/s"
 # the LM-head kernel the automatic choice runs on the 8x2x32 window (the CTA-pair kernel)
@@ -303,9 +303,9 @@ def verify_timing(dev, stream) -> dict:
 
     import paper_2609_33887_gb300 as bdc
     from paper_2609_33887_gb300 import bdcommit as B
-    from workloads.verify_inputs import VERIFY_CONFIGS, generate_verify
+    from workloads.verify_inputs import generate_verify, SPEC_LLAMA8B
 
-    cfg = VERIFY_CONFIGS[0]
+    cfg = SPEC_LLAMA8B
     wl = generate_verify(cfg).to(dev)
     R = cfg.rows
     ws = torch.empty(bdc.bd_verify_workspace_size(wl.hidden, wl.weight, None, wl.draft, cfg.n_req, cfg.n_draft,

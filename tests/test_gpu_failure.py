@@ -10,7 +10,7 @@ import torch
 
 from tests.helpers import oracle_on_workload
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B8X2X32_BF16, generate, scaled
 
 pytestmark = pytest.mark.gpu
 
@@ -39,7 +39,7 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     assert 0.9 < waited < 10.0, waited
     assert B.bd_get_device_status() == 0  # read once, then cleared
     # the context still runs the commit step correctly
-    wl = generate(scaled(CONFIGS[1], n_seq=2, n_slots=2, d=256, V=1000))
+    wl = generate(scaled(B8X2X32_BF16, n_seq=2, n_slots=2, d=256, V=1000))
     g = wl.to("cuda")
     tokens, conf, commit, _ = bdc.commit_step(g.hidden, g.weight, g.pos_masked, g.block_flags, 2, 2, 32, wl.tau)
     torch.cuda.synchronize()

@@ -6,7 +6,7 @@ import numpy as np
 import pytest
 import torch
 
-from workloads import CONFIGS, generate, scaled
+from workloads import B8X2X32_BF16, generate, scaled
 
 pytestmark = pytest.mark.gpu
 
@@ -26,7 +26,7 @@ def _lib():
 
 
 def test_graph_replay_matches_eager_and_times_the_lmhead():
-    cfg = scaled(CONFIGS[1], n_seq=4, n_slots=2, d=512, V=5000)
+    cfg = scaled(B8X2X32_BF16, n_seq=4, n_slots=2, d=512, V=5000)
     wl = generate(cfg).to("cuda")
     P = cfg.P
     args = (wl.hidden, wl.weight, None, wl.pos_masked, wl.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, -1,

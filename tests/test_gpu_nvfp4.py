@@ -17,7 +17,7 @@ import torch
 
 from tests.helpers import oracle_on_workload
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B8X2X32_BF16, generate, scaled
 from workloads.configs import by_name
 
 pytestmark = pytest.mark.gpu
@@ -66,10 +66,10 @@ def check(wl, variant=0, blocks=None, pad_scales=False):
 
 
 SMALL = {
-    "r128_d256": scaled(CONFIGS[1], n_seq=2, n_slots=2, d=256, V=1000, weight_dtype="nvfp4"),
+    "r128_d256": scaled(B8X2X32_BF16, n_seq=2, n_slots=2, d=256, V=1000, weight_dtype="nvfp4"),
     # ragged width: a K tail, an odd number of 16-element blocks, padded code rows
-    "r1024_d200": scaled(CONFIGS[1], n_seq=8, n_slots=4, d=200, V=3000, weight_dtype="nvfp4"),
-    "r294_d320": scaled(CONFIGS[1], d=320, V=2600, mask_frac=0.6, weight_dtype="nvfp4"),
+    "r1024_d200": scaled(B8X2X32_BF16, n_seq=8, n_slots=4, d=200, V=3000, weight_dtype="nvfp4"),
+    "r294_d320": scaled(B8X2X32_BF16, d=320, V=2600, mask_frac=0.6, weight_dtype="nvfp4"),
 }
 
 
@@ -93,7 +93,7 @@ def test_pair_fused_and_decoded(name, fused, monkeypatch):
 
 def test_pair_fused_mask_token_in_last_tile():
     """The in-kernel decode with a suppressed mask token inside the partial last v-tile."""
-    cfg = scaled(CONFIGS[1], n_seq=4, n_slots=2, d=256, V=2900, weight_dtype="nvfp4", mask_token_id=2899)
+    cfg = scaled(B8X2X32_BF16, n_seq=4, n_slots=2, d=256, V=2900, weight_dtype="nvfp4", mask_token_id=2899)
     rep = check(generate(cfg), variant=3, pad_scales=True)
     assert rep.n_live > 0
 
@@ -109,9 +109,9 @@ def test_verify_with_nvfp4_head():
     from oracle import verify_oracle as VO
     from workloads.generate import quantize_nvfp4
     from workloads.rawio import dtype_tag, raw_numpy
-    from workloads.verify_inputs import VERIFY_CONFIGS, generate_verify, verify_scaled
+    from workloads.verify_inputs import generate_verify, SPEC_LLAMA8B, verify_scaled
 
-    cfg = verify_scaled(VERIFY_CONFIGS[0], n_req=12, n_draft=4, d=256, V=2000, weight_dtype="f32", seed=8)
+    cfg = verify_scaled(SPEC_LLAMA8B, n_req=12, n_draft=4, d=256, V=2000, weight_dtype="f32", seed=8)
     wl = generate_verify(cfg)
     codes, bs, rs = quantize_nvfp4(wl.weight)
     ref = VO.verify_step(raw_numpy(wl.hidden), dtype_tag(wl.hidden), (codes.numpy(), bs.numpy()), "nvfp4",

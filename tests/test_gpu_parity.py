@@ -15,7 +15,7 @@ import torch
 
 from tests.helpers import oracle_on_workload
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B256X8X64_E4M3, B32X4X32_TIED, B64X4X64_BF16, B8X2X32_BF16, CONFIGS, generate, scaled, TINY_F32
 
 pytestmark = pytest.mark.gpu
 
@@ -63,24 +63,24 @@ def check(wl, variant=0, blocks=None, ref=None):
 
 SMALL = {
     # one m-tile, four v-tiles with a ragged last one
-    "bf16_1mt": scaled(CONFIGS[1], n_seq=2, n_slots=2, d=256, V=1000),
+    "bf16_1mt": scaled(B8X2X32_BF16, n_seq=2, n_slots=2, d=256, V=1000),
     # five m-tiles (ragged), ragged width (K tail of 8), twelve v-tiles
-    "bf16_5mt_ktail": scaled(CONFIGS[1], n_seq=8, n_slots=4, d=200, V=3000),
+    "bf16_5mt_ktail": scaled(B8X2X32_BF16, n_seq=8, n_slots=4, d=200, V=3000),
     # sixteen m-tiles: two bands of the plan
-    "bf16_2bands": scaled(CONFIGS[2], n_seq=32, n_slots=4, d=128, V=2148),
+    "bf16_2bands": scaled(B32X4X32_TIED, n_seq=32, n_slots=4, d=128, V=2148),
     # block_len 64, 16 thresholds
-    "bf16_L64": scaled(CONFIGS[3], n_seq=4, n_slots=4, d=192, V=4000),
+    "bf16_L64": scaled(B64X4X64_BF16, n_seq=4, n_slots=4, d=192, V=4000),
     # 257..320 rows: two token groups of the CTA-pair kernel
-    "bf16_g294": scaled(CONFIGS[1], d=256, V=3000, mask_frac=0.6),
-    "bf16_g271_mask": scaled(CONFIGS[1], d=320, V=2600, mask_frac=0.53, mask_token_id=2599),
+    "bf16_g294": scaled(B8X2X32_BF16, d=256, V=3000, mask_frac=0.6),
+    "bf16_g271_mask": scaled(B8X2X32_BF16, d=320, V=2600, mask_frac=0.53, mask_token_id=2599),
     # FP8 head with per-row scales
-    "e4m3": scaled(CONFIGS[4], n_seq=4, n_slots=4, d=512, V=5000),
-    "e4m3_ktail": scaled(CONFIGS[4], n_seq=3, n_slots=2, d=80, V=700),
+    "e4m3": scaled(B256X8X64_E4M3, n_seq=4, n_slots=4, d=512, V=5000),
+    "e4m3_ktail": scaled(B256X8X64_E4M3, n_seq=3, n_slots=2, d=80, V=700),
 }
 
 
 def test_tiny_f32_full():
-    wl = generate(CONFIGS[0])
+    wl = generate(TINY_F32)
     _, _, rep = check(wl)
     assert rep.n_live == 32
     assert rep.max_dconf < 1e-4  # exact fp32 path
@@ -220,7 +220,7 @@ def _sample_blocks(cfg, n, seed=99):
 
 
 def test_full_size_b8_all_positions():
-    wl = generate(CONFIGS[1])
+    wl = generate(B8X2X32_BF16)
     _, _, rep = check(wl)
     assert rep.n_live > 250
 

@@ -15,7 +15,7 @@ import torch
 from oracle import redline_oracle as RO
 from tests.helpers import oracle_on_workload
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B8X2X32_BF16, generate, scaled
 from workloads.redline_inputs import outcome_matrix
 
 pytestmark = pytest.mark.gpu
@@ -40,7 +40,7 @@ def test_tpf_from_commit_counts_feeds_redline():
     taus = (0.5, 0.7, 0.8, 0.9, 0.95, 0.99)
     gpu_steps, ref_steps, exempt = [], [], 0
     for step in range(4):
-        cfg = scaled(CONFIGS[1], n_seq=8, n_slots=4, d=200, V=3000, tau=taus, seed=100 + step)
+        cfg = scaled(B8X2X32_BF16, n_seq=8, n_slots=4, d=200, V=3000, tau=taus, seed=100 + step)
         wl = generate(cfg)
         g = wl.to("cuda")
         tokens, conf, commit, counts = bdc.commit_step(

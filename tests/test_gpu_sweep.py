@@ -12,7 +12,7 @@ import torch
 from oracle import sweep_oracle as SO
 from tests.helpers import oracle_on_workload
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B8X2X32_BF16, generate, scaled
 from workloads.sweep_inputs import random_step, random_window
 
 pytestmark = pytest.mark.gpu
@@ -120,7 +120,7 @@ def test_decode_loop_commit_step_then_sweep():
     may legitimately part: the sequences concerned are left out of that step's
     comparison and the loop ends there."""
     # 8-position blocks so that blocks complete within a few forwards
-    cfg = scaled(CONFIGS[1], n_seq=8, n_slots=4, block_len=8, d=200, V=3000, tau=(0.5, 0.7, 0.9, 0.95))
+    cfg = scaled(B8X2X32_BF16, n_seq=8, n_slots=4, block_len=8, d=200, V=3000, tau=(0.5, 0.7, 0.9, 0.95))
     wl0 = generate(cfg)
     n_seq, B, L = cfg.n_seq, cfg.n_slots, cfg.block_len
     k = 1  # deploy tau = 0.7

@@ -23,7 +23,7 @@ import torch
 
 from oracle import verify_oracle as VO
 from workloads.rawio import dtype_tag, raw_numpy
-from workloads.verify_inputs import VERIFY_CONFIGS, generate_verify, verify_scaled
+from workloads.verify_inputs import generate_verify, SPEC_LLAMA8B, verify_scaled
 
 pytestmark = pytest.mark.gpu
 
@@ -98,7 +98,7 @@ def check(wl, gpu, ref):
                 assert gpu["accepted"][q, k] == ref["accepted"][q, k], (q, k)
 
 
-BASE = VERIFY_CONFIGS[0]
+BASE = SPEC_LLAMA8B
 SMALL = {
     # one token group of the pair kernel, ragged last vocabulary tile
     "bf16_r40": verify_scaled(BASE, n_req=8, n_draft=4, d=256, V=3000, seed=1),
@@ -132,7 +132,7 @@ def test_full_size_llama_sampled():
     row of three sampled requests against the oracle; the lossless tokens per
     forward sit near 1 + sum a^i = 4.14 (a = 0.905, four drafts; the standard
     error over 64 requests is about 0.15)."""
-    cfg = VERIFY_CONFIGS[0]
+    cfg = SPEC_LLAMA8B
     wl = generate_verify(cfg)
     gpu = run_gpu(wl)
     keep = [0, 17, 63]

@@ -18,7 +18,7 @@ import torch
 
 from tests.helpers import oracle_on_workload, raw_numpy
 from tests.parity import compare
-from workloads import CONFIGS, generate, scaled
+from workloads import B256X8X64_E4M3, B8X2X32_BF16, generate, scaled
 from workloads.configs import by_name
 
 pytestmark = pytest.mark.gpu
@@ -75,11 +75,11 @@ def check(wl, out=None, blocks=None):
 
 SMALL = {
     # one token group, ragged last vocabulary tile
-    "e4m3_g64": scaled(CONFIGS[4], n_seq=4, n_slots=4, block_len=8, d=512, V=5000),
+    "e4m3_g64": scaled(B256X8X64_E4M3, n_seq=4, n_slots=4, block_len=8, d=512, V=5000),
     # two token groups (257..320 rows), width with a K tail of 80 columns
-    "e4m3_g294_ktail": scaled(CONFIGS[1], weight_dtype="e4m3", d=336, V=3000, mask_frac=0.6),
+    "e4m3_g294_ktail": scaled(B8X2X32_BF16, weight_dtype="e4m3", d=336, V=3000, mask_frac=0.6),
     # narrow rows (one partial 128-column stage), mask token in the last tile
-    "e4m3_d48_mask": scaled(CONFIGS[4], n_seq=3, n_slots=2, block_len=16, d=48, V=700, mask_token_id=699),
+    "e4m3_d48_mask": scaled(B256X8X64_E4M3, n_seq=3, n_slots=2, block_len=16, d=48, V=700, mask_token_id=699),
 }
 
 
@@ -101,7 +101,7 @@ def test_w8a8_zero_rows():
 
 
 def test_w8a8_needs_e4m3_pair_head():
-    wl = generate(scaled(CONFIGS[1], d=256, V=1000))  # bf16 head
+    wl = generate(scaled(B8X2X32_BF16, d=256, V=1000))  # bf16 head
     g = wl.to("cuda")
     c = wl.cfg
     with pytest.raises(bdc.BdError):

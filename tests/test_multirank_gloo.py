@@ -40,10 +40,10 @@ def _vocab_parallel_worker(rank, world, port, q):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
         import oracle
-        from workloads import CONFIGS, generate, scaled
+        from workloads import B8X2X32_BF16, generate, scaled
         from workloads.rawio import raw_numpy
 
-        cfg = scaled(CONFIGS[1], n_seq=1, n_slots=2, d=64, V=1001, mask_token_id=500)
+        cfg = scaled(B8X2X32_BF16, n_seq=1, n_slots=2, d=64, V=1001, mask_token_id=500)
         wl = generate(cfg)
         h = oracle.commit_oracle.hidden_f64(raw_numpy(wl.hidden), "bf16")
         w_raw = raw_numpy(wl.weight)

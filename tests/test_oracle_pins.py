@@ -149,10 +149,10 @@ def test_brute_force_50_digits_on_small_integer_problems():
 
 def test_logsumexp_cross_check_on_tiny_workload():
     sp = pytest.importorskip("scipy.special")
-    from workloads import CONFIGS, generate
+    from workloads import generate, TINY_F32
     from tests.helpers import raw_numpy
 
-    wl = generate(CONFIGS[0])
+    wl = generate(TINY_F32)
     h = hidden_f64(raw_numpy(wl.hidden), "f32")
     w = raw_numpy(wl.weight).astype(np.float64)
     for p in range(wl.P):

@@ -22,7 +22,7 @@ import pytest
 
 from oracle import verify_oracle as VO
 from workloads.rawio import dtype_tag, raw_numpy
-from workloads.verify_inputs import VERIFY_CONFIGS, generate_verify, verify_scaled
+from workloads.verify_inputs import generate_verify, SPEC_LLAMA8B, verify_scaled
 
 mpmath = pytest.importorskip("mpmath")
 
@@ -90,7 +90,7 @@ def test_brute_force_50_digits():
 
 @pytest.fixture(scope="module")
 def small():
-    cfg = verify_scaled(VERIFY_CONFIGS[0], n_req=40, n_draft=6, d=96, V=3000, boost_lo=2.0, boost_hi=14.0,
+    cfg = verify_scaled(SPEC_LLAMA8B, n_req=40, n_draft=6, d=96, V=3000, boost_lo=2.0, boost_hi=14.0,
                         agree=0.7, seed=5)
     wl = generate_verify(cfg)
     return wl, run(wl)
@@ -137,7 +137,7 @@ def test_paper_lossless_figures_from_agreement():
     assert round(1 + sum(0.905**i for i in range(1, 5)), 2) == 4.14
     assert round(1 + sum(0.887**i for i in range(1, 5)), 2) == 3.99
     for a in (0.905, 0.887):
-        cfg = verify_scaled(VERIFY_CONFIGS[0], n_req=3000, n_draft=4, d=64, V=256, boost_lo=10.0, boost_hi=18.0,
+        cfg = verify_scaled(SPEC_LLAMA8B, n_req=3000, n_draft=4, d=64, V=256, boost_lo=10.0, boost_hi=18.0,
                             agree=a, eps=(0.1,), hidden_dtype="f32", weight_dtype="f32", seed=21)
         wl = generate_verify(cfg)
         r = run(wl)

@@ -4,7 +4,8 @@ import numpy as np
 import pytest
 import torch
 
-from workloads import ACTIVE, CONFIGS, FALLBACK_ELIGIBLE, generate, scaled
+from workloads import (ACTIVE, B256X8X64_E4M3, B32X4X32_TIED, B64X4X64_BF16, B8X2X32_BF16, CONFIGS,
+    FALLBACK_ELIGIBLE, generate, scaled, TINY_F32)
 
 
 def test_five_workloads_have_the_stated_shapes():
@@ -16,16 +17,16 @@ def test_five_workloads_have_the_stated_shapes():
         (64, 4, 64, 4096, 151936, 16),
         (256, 8, 64, 5120, 157184, 16),
     ]
-    assert CONFIGS[1].tau == (0.7, 0.8, 0.9, 0.95)
-    for c in CONFIGS[2:]:
+    assert B8X2X32_BF16.tau == (0.7, 0.8, 0.9, 0.95)
+    for c in (B32X4X32_TIED, B64X4X64_BF16, B256X8X64_E4M3):
         assert 0.95 in c.tau and list(c.tau) == sorted(c.tau)
-    assert CONFIGS[2].tau[0] == 0.5 and CONFIGS[2].tau[-1] == pytest.approx(0.98)
-    assert CONFIGS[3].tau[0] == pytest.approx(0.3) and CONFIGS[3].tau[-1] == pytest.approx(0.99)
+    assert B32X4X32_TIED.tau[0] == 0.5 and B32X4X32_TIED.tau[-1] == pytest.approx(0.98)
+    assert B64X4X64_BF16.tau[0] == pytest.approx(0.3) and B64X4X64_BF16.tau[-1] == pytest.approx(0.99)
 
 
 def test_tiny_is_seeded_and_reproducible():
-    a = generate(CONFIGS[0])
-    b = generate(CONFIGS[0])
+    a = generate(TINY_F32)
+    b = generate(TINY_F32)
     assert torch.equal(a.hidden, b.hidden) and torch.equal(a.weight, b.weight)
     assert a.hidden.dtype == torch.float32 and a.weight.shape == (4096, 256)
     assert int(a.pos_masked.sum()) == 32
@@ -33,7 +34,7 @@ def test_tiny_is_seeded_and_reproducible():
 
 
 def test_tiny_plants_plus_eight_on_half_the_positions():
-    wl = generate(CONFIGS[0])
+    wl = generate(TINY_F32)
     h = wl.hidden.double()
     w = wl.weight.double()
     logits = h @ w.T
@@ -46,7 +47,7 @@ def test_tiny_plants_plus_eight_on_half_the_positions():
 
 
 def test_scaled_bf16_and_e4m3_variants():
-    c = scaled(CONFIGS[4], n_seq=2, n_slots=2, d=128, V=1000)
+    c = scaled(B256X8X64_E4M3, n_seq=2, n_slots=2, d=128, V=1000)
     wl = generate(c)
     assert wl.weight.dtype == torch.float8_e4m3fn and wl.weight_scale.shape == (1000,)
     deq = wl.weight.float() * wl.weight_scale[:, None]
@@ -60,7 +61,7 @@ def test_scaled_bf16_and_e4m3_variants():
 
 
 def test_mask_fraction_is_close_to_the_stated_rate():
-    c = scaled(CONFIGS[1], d=8, V=64)
+    c = scaled(B8X2X32_BF16, d=8, V=64)
     wl = generate(c)
     frac = wl.pos_masked.float().mean().item()
     assert abs(frac - 0.6) < 0.07

@@ -15,7 +15,7 @@ import numpy as np
 import pytest
 import torch
 
-from workloads import CONFIGS, generate, scaled
+from workloads import B256X8X64_E4M3, B64X4X64_BF16, B8X2X32_BF16, generate, scaled, TINY_F32
 
 pytestmark = pytest.mark.gpu
 
@@ -53,7 +53,7 @@ def _run(wl, static):
     return tok.cpu().numpy(), conf.cpu().numpy(), com.cpu().numpy().view(np.uint32)
 
 
-@pytest.mark.parametrize("cfg", [CONFIGS[1], CONFIGS[0], scaled(CONFIGS[4], n_seq=4, n_slots=4, d=512, V=5000)],
+@pytest.mark.parametrize("cfg", [B8X2X32_BF16, TINY_F32, scaled(B256X8X64_E4M3, n_seq=4, n_slots=4, d=512, V=5000)],
                          ids=["b8x2x32_bf16", "tiny_f32", "e4m3_small"])
 def test_static_matches_the_allocating_entry_point_twice(cfg):
     wl = generate(cfg)
@@ -69,7 +69,7 @@ def test_static_matches_the_allocating_entry_point_twice(cfg):
 def test_static_rejects_windows_beyond_its_array():
     # the 64 x 4 x 64, d = 4096 window needs far more than 32 MiB of workspace;
     # the call is refused before anything is queued
-    cfg = scaled(CONFIGS[3], V=1024, name="too_large")
+    cfg = scaled(B64X4X64_BF16, V=1024, name="too_large")
     P = cfg.P
     dev = torch.device("cuda")
     h = torch.zeros((P, cfg.d), dtype=torch.bfloat16, device=dev)

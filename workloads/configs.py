@@ -68,51 +68,56 @@ class WorkloadConfig:
         return self.n_seq * self.n_slots
 
 
-CONFIGS = (
-    WorkloadConfig(
-        name="tiny_f32_d256_v4096",
-        n_seq=1, n_slots=1, block_len=32, mask_frac=1.0,
-        d=256, V=4096, hidden_dtype="f32", weight_dtype="f32",
-        boost="fixed_half", boost_frac=0.5, boost_lo=8.0, boost_hi=8.0,
-        tau=(0.9,), seed=0,
-    ),
-    WorkloadConfig(
-        name="b8x2x32_d2048_v151936_bf16",
-        n_seq=8, n_slots=2, block_len=32, mask_frac=0.6,
-        d=2048, V=151936, hidden_dtype="bf16", weight_dtype="bf16",
-        boost="single", boost_frac=0.4, boost_lo=2.0, boost_hi=10.0,
-        tau=(0.7, 0.8, 0.9, 0.95), seed=1,
-    ),
-    WorkloadConfig(
-        name="b32x4x32_d2048_v157184_bf16_tied",
-        n_seq=32, n_slots=4, block_len=32, mask_frac=0.5,
-        d=2048, V=157184, hidden_dtype="bf16", weight_dtype="bf16",
-        boost="tied_mix", boost_frac=0.6, boost_lo=2.0, boost_hi=10.0,
-        tau=_grid(0.5, 0.98, 8), seed=2,
-    ),
-    WorkloadConfig(
-        name="b64x4x64_d4096_v151936_bf16",
-        n_seq=64, n_slots=4, block_len=64, mask_frac=0.5,
-        d=4096, V=151936, hidden_dtype="bf16", weight_dtype="bf16",
-        boost="single", boost_frac=0.5, boost_lo=0.0, boost_hi=12.0,
-        tau=_grid(0.3, 0.99, 16), seed=3,
-    ),
-    WorkloadConfig(
-        name="b256x8x64_d5120_v157184_e4m3",
-        n_seq=256, n_slots=8, block_len=64, mask_frac=0.4,
-        d=5120, V=157184, hidden_dtype="bf16", weight_dtype="e4m3",
-        boost="single", boost_frac=0.5, boost_lo=0.0, boost_hi=12.0,
-        tau=_grid(0.5, 0.99, 16), seed=4,
-    ),
+# the small case the oracle runs in full (exact fp32 path)
+TINY_F32 = WorkloadConfig(
+    name="tiny_f32_d256_v4096",
+    n_seq=1, n_slots=1, block_len=32, mask_frac=1.0,
+    d=256, V=4096, hidden_dtype="f32", weight_dtype="f32",
+    boost="fixed_half", boost_frac=0.5, boost_lo=8.0, boost_hi=8.0,
+    tau=(0.9,), seed=0,
 )
+# the bench window: 8 sequences x 2 slots x 32 positions
+B8X2X32_BF16 = WorkloadConfig(
+    name="b8x2x32_d2048_v151936_bf16",
+    n_seq=8, n_slots=2, block_len=32, mask_frac=0.6,
+    d=2048, V=151936, hidden_dtype="bf16", weight_dtype="bf16",
+    boost="single", boost_frac=0.4, boost_lo=2.0, boost_hi=10.0,
+    tau=(0.7, 0.8, 0.9, 0.95), seed=1,
+)
+# 32 x 4 x 32 with tied top logits
+B32X4X32_TIED = WorkloadConfig(
+    name="b32x4x32_d2048_v157184_bf16_tied",
+    n_seq=32, n_slots=4, block_len=32, mask_frac=0.5,
+    d=2048, V=157184, hidden_dtype="bf16", weight_dtype="bf16",
+    boost="tied_mix", boost_frac=0.6, boost_lo=2.0, boost_hi=10.0,
+    tau=_grid(0.5, 0.98, 8), seed=2,
+)
+# 64 x 4 x 64, d = 4096
+B64X4X64_BF16 = WorkloadConfig(
+    name="b64x4x64_d4096_v151936_bf16",
+    n_seq=64, n_slots=4, block_len=64, mask_frac=0.5,
+    d=4096, V=151936, hidden_dtype="bf16", weight_dtype="bf16",
+    boost="single", boost_frac=0.5, boost_lo=0.0, boost_hi=12.0,
+    tau=_grid(0.3, 0.99, 16), seed=3,
+)
+# 256 x 8 x 64 with an FP8 head, d = 5120
+B256X8X64_E4M3 = WorkloadConfig(
+    name="b256x8x64_d5120_v157184_e4m3",
+    n_seq=256, n_slots=8, block_len=64, mask_frac=0.4,
+    d=5120, V=157184, hidden_dtype="bf16", weight_dtype="e4m3",
+    boost="single", boost_frac=0.5, boost_lo=0.0, boost_hi=12.0,
+    tau=_grid(0.5, 0.99, 16), seed=4,
+)
+
+CONFIGS = (TINY_F32, B8X2X32_BF16, B32X4X32_TIED, B64X4X64_BF16, B256X8X64_E4M3)
 
 
 # The precision levers on the bench window (not among the five workloads):
 # the b8x2x32 window and head shape with an NVFP4 or an E4M3 head.
 EXTRA_CONFIGS = (
-    dataclasses.replace(CONFIGS[1], name="b8x2x32_d2048_v151936_nvfp4", weight_dtype="nvfp4"),
+    dataclasses.replace(B8X2X32_BF16, name="b8x2x32_d2048_v151936_nvfp4", weight_dtype="nvfp4"),
     # the 8-bit levers on the same window: an E4M3 head (W8A16 and W8A8)
-    dataclasses.replace(CONFIGS[1], name="b8x2x32_d2048_v151936_e4m3", weight_dtype="e4m3"),
+    dataclasses.replace(B8X2X32_BF16, name="b8x2x32_d2048_v151936_e4m3", weight_dtype="e4m3"),
 )
 
 

@@ -54,14 +54,18 @@ class VerifyConfig:
         return self.n_req * (self.n_draft + 1)
 
 
-VERIFY_CONFIGS = (
-    VerifyConfig(name="spec_llama8b_r64x5_d4096_v128256_bf16", n_req=64, n_draft=4, d=4096, V=128256,
-                 hidden_dtype="bf16", weight_dtype="bf16", boost_lo=8.0, boost_hi=18.0, agree=0.905,
-                 eps=EPS_GRID, seed=11),
-    VerifyConfig(name="spec_qwen7b_r64x5_d3584_v152064_bf16", n_req=64, n_draft=4, d=3584, V=152064,
-                 hidden_dtype="bf16", weight_dtype="bf16", boost_lo=8.0, boost_hi=18.0, agree=0.887,
-                 eps=EPS_GRID, seed=12),
+# Llama-3.1-8B's LM-head shape, 64 requests x (4 drafts + 1)
+SPEC_LLAMA8B = VerifyConfig(
+    name="spec_llama8b_r64x5_d4096_v128256_bf16", n_req=64, n_draft=4, d=4096, V=128256,
+    hidden_dtype="bf16", weight_dtype="bf16", boost_lo=8.0, boost_hi=18.0, agree=0.905, eps=EPS_GRID, seed=11,
 )
+# Qwen2.5-7B's LM-head shape, 64 requests x (4 drafts + 1)
+SPEC_QWEN7B = VerifyConfig(
+    name="spec_qwen7b_r64x5_d3584_v152064_bf16", n_req=64, n_draft=4, d=3584, V=152064,
+    hidden_dtype="bf16", weight_dtype="bf16", boost_lo=8.0, boost_hi=18.0, agree=0.887, eps=EPS_GRID, seed=12,
+)
+
+VERIFY_CONFIGS = (SPEC_LLAMA8B, SPEC_QWEN7B)
 
 
 def verify_by_name(name: str) -> VerifyConfig:
