@@ -157,7 +157,7 @@ typedef struct {
  *   lmhead_event_begin / lmhead_event_end : optional cudaEvent_t recorded on
  *                     the stream right before and after the LM-head kernel,
  *                     for timing it alone.
- *   variant         : 0 = automatic (for BF16 / E4M3 heads the CTA-pair
+ *   variant         : 0 = automatic (for BF16 / E4M3 / NVFP4 heads the CTA-pair
  *                     tensor-core kernel up to 8192 window positions and the
  *                     one-CTA kernel above; the fp32 SIMT kernel for F32
  *                     heads); 1 = force
@@ -206,8 +206,11 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight,
                       const bd_exec* exec);
 
 /* Bytes of device workspace a call with these arguments needs (0 if the
- * arguments are invalid). Depends on sizes, dtypes and the current device's
- * SM count only, not on the data. */
+ * arguments are invalid), for bd_exec.variant 0 (automatic) with flags 0 or
+ * BD_EXEC_FP8_ACTIVATIONS. Depends on sizes, dtypes and the current device's
+ * SM count only, not on the data. A forced variant 1 or 2 can need more (more
+ * partial slots; a decoded copy of a quantised head); such a call with a
+ * smaller caller workspace returns BD_ERR_WORKSPACE without launching. */
 size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
                          const bd_mask_state* mask_state, const bd_tau_grid* tau_grid);
 
