@@ -369,6 +369,29 @@ LEVERS = {
 }
 
 
+def fp8_gemm_tflops(dev, stream, n=8192, reps=30):
+    """Dense E4M3 x E4M3 -> bf16 GEMM throughput of the vendor library
+    (torch._scaled_mm, n x n x n, random codes) on this GPU, for the W8A8
+    roofline's FP8 peak; None (with the reason) where the call is unavailable."""
+    try:
+        g = torch.Generator(device="cpu").manual_seed(5)
+        a = torch.randn(n, n, generator=g).to(dev).to(torch.float8_e4m3fn)
+        b = torch.randn(n, n, generator=g).to(dev).to(torch.float8_e4m3fn).t()  # column-major operand
+        one = torch.ones((), device=dev)
+        with torch.cuda.stream(stream):
+            for _ in range(5):
+                torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+            (e0, e1), = timing_events(1, stream)
+            e0.record(stream)
+            for _ in range(reps):
+                torch._scaled_mm(a, b, scale_a=one, scale_b=one, out_dtype=torch.bfloat16)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        return 2.0 * n ** 3 * reps / (e0.elapsed_time(e1) * 1e-3) / 1e12, None
+    except Exception as exc:  # noqa: BLE001 - reported, not raised
+        return None, f"{type(exc).__name__}: {exc}"[:200]
+
+
 def lever_timing(dev, stream, lever: str) -> dict:
     """The bench window (8 x 2 x 32, d = 2048, V = 151936) with a quantised
     head (the precision levers): device time per commit step (CUDA events
@@ -425,13 +448,21 @@ def lever_timing(dev, stream, lever: str) -> dict:
     flops = 2.0 * n_masked * cfg.d * cfg.V
     hbm_gbs, tc_tflops, _, src = peaks()
     tc_peak = 2.0 * tc_tflops if lever == "w8a8" else tc_tflops
-    return {"workload": cfg.name, "ms_per_step": ms, "positions_per_s": n_masked / (ms / 1e3),
-            "lmhead_us": lm_us, "algorithmic_bytes": abytes, "algorithmic_flops": flops,
-            "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs,
-            "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_peak,
-            "tensor_peak_tflops": tc_peak,
-            "path": path,
-            "peak_source": src + (" (x2: nominal FP8 : BF16 ratio)" if lever == "w8a8" else "")}
+    out = {"workload": cfg.name, "ms_per_step": ms, "positions_per_s": n_masked / (ms / 1e3),
+           "lmhead_us": lm_us, "algorithmic_bytes": abytes, "algorithmic_flops": flops,
+           "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs,
+           "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_peak,
+           "tensor_peak_tflops": tc_peak,
+           "path": path,
+           "peak_source": src + (" (x2: nominal FP8 : BF16 ratio)" if lever == "w8a8" else "")}
+    if lever == "w8a8":
+        # the library's own FP8 GEMM on this GPU, measured here, beside the nominal-ratio peak
+        fp8, why = fp8_gemm_tflops(dev, stream)
+        out["fp8_gemm_tflops_measured"] = fp8
+        out["lmhead_tensor_frac_of_measured_fp8"] = (flops / (lm_us * 1e-6) / 1e12 / fp8) if fp8 else None
+        if why:
+            out["fp8_gemm_unavailable"] = why
+    return out
 
 
 def run_ours(args):
