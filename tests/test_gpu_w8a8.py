@@ -138,3 +138,25 @@ def test_w8a8_row_magnitudes_across_the_bf16_range():
     wl.hidden = (wl.hidden.double() * torch.exp2(k)[:, None]).to(wl.hidden.dtype)
     _, rep = check(wl)
     assert rep.n_live > 0
+
+
+def test_w8a8_lossless_rows_match_the_exact_step():
+    """Rows the per-row quantiser reproduces exactly (E4M3 values times 2^k,
+    largest magnitude 448 * 2^k): the W8A8 step must match the exact oracle on
+    the bf16 rows themselves."""
+    from oracle import commit_oracle as C
+
+    wl = generate(SMALL["e4m3_g294_ktail"])
+    rng = np.random.default_rng(21)
+    finite = C.decode_e4m3(np.arange(256))
+    finite = finite[np.isfinite(finite)]
+    P, d = wl.hidden.shape
+    h = rng.choice(finite, size=(P, d)) * 2.0 ** -6
+    h[:, 0] = np.where(rng.random(P) < 0.5, 448.0, -448.0) * 2.0 ** -6
+    k = rng.integers(-8, 3, size=P).astype(np.float64)
+    wl.hidden = torch.from_numpy(h * np.exp2(k)[:, None]).to(torch.bfloat16)
+    assert np.array_equal(wl.hidden.double().numpy(), h * np.exp2(k)[:, None])  # exact in bf16
+    out = run_w8a8(wl)
+    rep = compare(out, oracle_on_workload(wl), wl.tau, "e4m3", wl.cfg.block_len, wl.cfg.n_slots)
+    assert rep.ok(), rep.failures
+    assert rep.n_live > 0

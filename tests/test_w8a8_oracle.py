@@ -84,3 +84,41 @@ def test_row_quantiser():
     assert np.all(err <= bound)
     # scale = amax / 448 in float32
     assert np.array_equal(scale[rows], (np.max(np.abs(h[rows]), axis=1) / np.float32(448)).astype(np.float32))
+
+
+def representable_rows(rng, n, d):
+    """Rows that the per-row E4M3 quantiser reproduces exactly: every entry an
+    E4M3 value times 2^k_row, and the row's largest magnitude 448 * 2^k_row
+    (so inv = 2^-k_row exactly and every code is the entry's own)."""
+    finite = C.decode_e4m3(np.arange(256))
+    finite = finite[np.isfinite(finite)]
+    h = rng.choice(finite, size=(n, d))
+    h[:, 0] = np.where(rng.random(n) < 0.5, 448.0, -448.0)
+    k = rng.integers(-20, 4, size=n).astype(np.float64)
+    return (h * np.exp2(k)[:, None]).astype(np.float32)
+
+
+def test_quantiser_is_exact_on_representable_rows():
+    rng = np.random.default_rng(9)
+    h = representable_rows(rng, 40, 96)
+    codes, scale = C.quantize_rows_e4m3(h)
+    assert np.array_equal(C.dequantize_rows_e4m3(codes, scale), h.astype(np.float64))
+
+
+def test_w8a8_step_equals_exact_step_on_representable_rows():
+    """Where quantisation is lossless, the W8A8 oracle (the step on the
+    dequantised rows) is the exact step itself."""
+    rng = np.random.default_rng(10)
+    L, S, B, d, V = 8, 2, 2, 64, 300
+    P = L * S * B
+    h = representable_rows(rng, P, d)
+    w = rng.normal(size=(V, d)).astype(np.float32)
+    pm = (rng.random(P) < 0.7).astype(np.uint8)
+    flags = np.array([3, 1, 1, 3], dtype=np.uint8)
+    taus = [0.3, 0.6, 0.9]
+    exact = C.commit_step(h, "f32", w, "f32", None, pm, flags, B, S, L, -1, taus)
+    codes, scale = C.quantize_rows_e4m3(h)
+    w8 = C.commit_step(C.dequantize_rows_e4m3(codes, scale), "f64", w, "f32", None, pm, flags, B, S, L, -1, taus)
+    for key in ("tokens", "commit", "counts"):
+        assert np.array_equal(exact[key], w8[key])
+    assert np.array_equal(exact["conf"], w8["conf"])
