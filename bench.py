@@ -240,7 +240,7 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
-                   "d": cfg.d, "V": cfg.V, "T": len(cfg.tau)},
+                   "d": cfg.d, "V": cfg.V, "T": len(cfg.tau), "inputs_sha256": wl.digests()},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                          "sample": f"{n_blocks} whole block(s) per step of {cfg.name}; head decoded to float64 "
                                    "once, outside the timed steps"},
@@ -746,7 +746,8 @@ def run_ours(args):
                        "masked_positions_per_rank": n_masked, "d": cfg.d, "V": cfg.V, "T": len(cfg.tau),
                        "parallelism": f"independent windows x{world}", "graph": bool(args.graph),
                        "l2": "inputs larger than L2 (the LM head is %.0f MB, read every step)"
-                             % (cfg.V * cfg.d * {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype] / 1e6)},
+                             % (cfg.V * cfg.d * {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype] / 1e6),
+                       "inputs_sha256": wl_host.digests()},
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,

@@ -13,6 +13,7 @@ the CUDA library read.
 
 from __future__ import annotations
 
+import hashlib
 import math
 from dataclasses import dataclass
 from typing import Optional, Tuple
@@ -42,6 +43,17 @@ class Workload:
     @property
     def P(self) -> int:
         return self.cfg.P
+
+    def digests(self) -> dict:
+        """SHA-256 (first 16 hex digits) of each stored input tensor's bytes, so a
+        run can record exactly which inputs it used."""
+        out = {}
+        for name in ("hidden", "weight", "weight_scale", "weight_block_scale", "pos_masked", "block_flags"):
+            t = getattr(self, name)
+            if t is not None:
+                raw = t.detach().to("cpu").contiguous().view(torch.uint8).numpy().tobytes()
+                out[name] = hashlib.sha256(raw).hexdigest()[:16]
+        return out
 
     def to(self, device) -> "Workload":
         return Workload(
