@@ -261,3 +261,56 @@ def test_sampled_blocks_match_full_evaluation():
     assert ev.sum() == 3 * wl.cfg.block_len
     for key in ("tokens", "conf", "commit"):
         assert np.array_equal(part[key][ev], full[key][ev])
+
+
+# ---------------------------------------------------- the merge operator --
+
+def _partial(l, lo):
+    """(max, sum of exp(l - max), lowest argmax) of one chunk starting at index lo."""
+    m = float(np.max(l))
+    if m == -math.inf:
+        return (-math.inf, 0.0, 1 << 30)
+    return (m, float(np.sum(np.exp(l - m))), lo + int(np.flatnonzero(l == m)[0]))
+
+
+def _combine(x, y):
+    """The merge rule the CUDA kernels apply across CTAs, restated: the larger
+    max wins and the other sum is rescaled to it; equal maxima add their sums
+    and keep the lower index."""
+    (m1, s1, a1), (m2, s2, a2) = x, y
+    if m2 > m1:
+        return (m2, s2 + (s1 * math.exp(m1 - m2) if m1 > -math.inf else 0.0), a2)
+    if m2 == m1:
+        return (m1, s1 + s2 if m1 > -math.inf else 0.0, min(a1, a2))
+    return (m1, s1 + (s2 * math.exp(m2 - m1) if m2 > -math.inf else 0.0), a1)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_chunked_merge_equals_the_single_pass(seed):
+    """Splitting the vocabulary into any number of chunks (uneven, some holding
+    only the suppressed entry) and merging their partials in any order and
+    grouping gives the oracle's single-pass token and confidence: the merge is
+    associative and commutative and keeps the lowest index on equal maxima.
+    Small integer logits make ties across chunks frequent."""
+    rng = np.random.default_rng(seed)
+    for _ in range(40):
+        V = int(rng.integers(2, 60))
+        l = rng.integers(-3, 4, size=V).astype(np.float64)
+        mask = int(rng.integers(-1, V))
+        token, conf, _ = oracle.commit_oracle.row_confidence(l, mask)
+        lm = l.copy()
+        if mask >= 0:
+            lm[mask] = -np.inf
+        k = int(rng.integers(1, V + 1))
+        cuts = np.sort(rng.choice(np.arange(1, V), size=min(k - 1, V - 1), replace=False)) if V > 1 else []
+        bounds = [0, *[int(c) for c in cuts], V]
+        parts = [_partial(lm[a:b], a) for a, b in zip(bounds[:-1], bounds[1:])]
+        order = rng.permutation(len(parts))
+        # a random binary tree over the shuffled partials
+        pool = [parts[i] for i in order]
+        while len(pool) > 1:
+            i = int(rng.integers(0, len(pool) - 1))
+            pool[i:i + 2] = [_combine(pool[i], pool[i + 1])]
+        m, s, a = pool[0]
+        assert a == token
+        assert abs(1.0 / s - conf) < 1e-12
