@@ -546,6 +546,7 @@ def run_ours(args):
         pg.barrier()
     torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push(f"timed region: {K} steps")  # trace range (no-op without a tracer)
     t_start.record(stream)
     if graph is None:
         for i in range(K):
@@ -553,6 +554,7 @@ def run_ours(args):
     else:
         graph.replay()
     t_end.record(stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
@@ -732,9 +734,12 @@ def run_ours(args):
                "sample": f"{passes} pass(es) over {len(blocks)} whole blocks of {cfg.name} ({tot_n} masked "
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
-    redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
-    verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
-    levers = {k: lever_timing(dev, stream, k) for k in LEVERS} if rank == 0 and not args.no_verify else {}
+    with torch.cuda.nvtx.range("redline"):
+        redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
+    with torch.cuda.nvtx.range("verify"):
+        verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
+    with torch.cuda.nvtx.range("precision levers"):
+        levers = {k: lever_timing(dev, stream, k) for k in LEVERS} if rank == 0 and not args.no_verify else {}
 
     if rank == 0:
         line = {

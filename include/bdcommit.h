@@ -50,7 +50,9 @@ typedef enum {
   BD_ERR_CUDA = -7,      /* a CUDA runtime call or kernel launch failed */
   BD_ERR_TIMEOUT = -8,   /* a bounded device-side wait gave up (see bd_get_device_status) */
   BD_ERR_DEVICE = -9,    /* the current device cannot run this library (needs sm_103) */
-  BD_ERR_ARG = -10       /* other invalid argument (mask_token_id, variant, flags) */
+  BD_ERR_ARG = -10,      /* other invalid argument (mask_token_id, variant, flags) */
+  BD_ERR_BOUNDS = -11    /* a device-side index check failed: only the bounds-checked build
+                            (libbdcommit_checks.so, -DBD_CHECKS) checks indices */
 } bd_status;
 
 /* ----------------------------------------------------------------- dtypes */

@@ -17,7 +17,9 @@ from typing import Optional, Sequence
 import torch
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libbdcommit.so")
+# BD_LIBRARY selects another build of the library (e.g. the bounds-checked
+# libbdcommit_checks.so); by default the in-tree libbdcommit.so
+LIB_PATH = os.environ.get("BD_LIBRARY") or os.path.join(_PKG, "libbdcommit.so")
 
 # status codes (bd_status)
 BD_OK = 0
@@ -31,6 +33,7 @@ BD_ERR_CUDA = -7
 BD_ERR_TIMEOUT = -8
 BD_ERR_DEVICE = -9
 BD_ERR_ARG = -10
+BD_ERR_BOUNDS = -11
 
 # dtypes (bd_dtype)
 BD_F32 = 0

@@ -22,6 +22,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libbdcommit.so")
+LIB_CHECKS = os.path.join(PKG, "libbdcommit_checks.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
@@ -54,19 +55,25 @@ def _stamp(nvcc: str, extra) -> str:
     return h.hexdigest()
 
 
-def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
-    """Compile every source and link libbdcommit.so; returns its path."""
+def build(verbose: bool = False, force: bool = False, extra_flags=(), checks: bool = False) -> str:
+    """Compile every source and link libbdcommit.so; returns its path.
+
+    checks=True builds the bounds-checked variant instead (-DBD_CHECKS:
+    device-side index checks that set a status bit rather than access out of
+    range) as libbdcommit_checks.so, in its own build directory."""
     nvcc = _nvcc()
-    os.makedirs(BUILD, exist_ok=True)
-    stamp_file = os.path.join(BUILD, "libbdcommit.stamp")
+    build_dir, lib = (BUILD + "_checks", LIB_CHECKS) if checks else (BUILD, LIB)
+    extra_flags = list(extra_flags) + (["-DBD_CHECKS"] if checks else [])
+    os.makedirs(build_dir, exist_ok=True)
+    stamp_file = os.path.join(build_dir, "libbdcommit.stamp")
     stamp = _stamp(nvcc, extra_flags)
-    if not force and os.path.exists(LIB) and os.path.exists(stamp_file):
+    if not force and os.path.exists(lib) and os.path.exists(stamp_file):
         with open(stamp_file) as f:
             if f.read().strip() == stamp:
-                return LIB
+                return lib
 
     def compile_one(src):
-        obj = os.path.join(BUILD, os.path.splitext(os.path.basename(src))[0] + ".o")
+        obj = os.path.join(build_dir, os.path.splitext(os.path.basename(src))[0] + ".o")
         cmd = [nvcc] + NVCC_FLAGS + list(extra_flags) + ["-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
@@ -78,19 +85,19 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
     srcs = _sources()
     with ThreadPoolExecutor(max_workers=min(8, len(srcs))) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB + ".tmp"
-    exports = os.path.join(BUILD, "exports.map")
+    tmp = lib + ".tmp"
+    exports = os.path.join(build_dir, "exports.map")
     with open(exports, "w") as f:
         f.write("{ global: bd_*; local: *; };\n")  # only the C ABI is visible
     cmd = [nvcc] + ARCH + ["-shared", "-cudart", "static", "-Xlinker", "--version-script=" + exports,
-                           "-o", tmp] + objs
+                           "-o", tmp] + objs + ["-ldl"]  # libdl: the NVTX trace ranges load a tracer on demand
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    os.replace(tmp, lib)
     with open(stamp_file, "w") as f:
         f.write(stamp)
-    return LIB
+    return lib
 
 
 if __name__ == "__main__":

@@ -9,7 +9,9 @@
 #include <mutex>
 
 #include "bdcommit.h"
+#include "checks.h"
 #include "kernels.h"
+#include "trace.h"
 
 namespace {
 
@@ -427,7 +429,7 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   const int64_t ld_rows = c.fp8_act ? ld_fp8_rows(c) : c.ldc;
   int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
                                             c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
-                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc, row_format));
+                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc, row_format, status));
   if (rc != BD_OK) return rc;
 
   rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, ld_rows, ws + lay.wq, idx, n_rows, nullptr,
@@ -455,6 +457,7 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   ca.out_conf = out_conf;
   ca.out_commit = out_commit;
   ca.out_counts = out_counts;
+  ca.status = status;
   return cuda_status(bd::launch_merge_commit(ca, st));
 }
 }  // namespace
@@ -476,6 +479,7 @@ const char* bd_status_string(int status) {
     case BD_ERR_TIMEOUT: return "a bounded device-side wait gave up";
     case BD_ERR_DEVICE: return "the current device cannot run this library (needs sm_103)";
     case BD_ERR_ARG: return "invalid argument";
+    case BD_ERR_BOUNDS: return "a device-side index check failed (bounds-checked build)";
     default: return "unknown status";
   }
 }
@@ -492,6 +496,7 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const
 int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
                       const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                       const bd_exec* exec) {
+  bd::TraceRange trace("bd_commit_step");
   const int variant = exec ? exec->variant : 0;
   const int flags = exec ? exec->flags : 0;
   if (flags & ~BD_EXEC_FP8_ACTIVATIONS) return BD_ERR_ARG;
@@ -554,6 +559,7 @@ int bd_get_device_status(void* stream) {
   if (word != 0 && cudaMemset(ctx->status, 0, sizeof(word)) != cudaSuccess) return BD_ERR_CUDA;
   if (word & bd::DEV_TIMEOUT) return BD_ERR_TIMEOUT;
   if (word & bd::DEV_BAD_LAUNCH) return BD_ERR_CUDA;
+  if (word & bd::DEV_BOUNDS) return BD_ERR_BOUNDS;
   return BD_OK;
 }
 
@@ -652,6 +658,7 @@ int static_ctx(StaticCtx** out) {
 extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
                                      const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
                                      int32_t* out_tokens, float* out_conf, uint32_t* out_commit, void* stream) {
+  bd::TraceRange trace("bd_commit_step_static");
   Call c;
   int rc = check_args(hidden, weight, mask_state, tau_grid, 0, &c);
   if (rc != BD_OK) return rc;
@@ -808,6 +815,7 @@ size_t bd_verify_workspace_size(const bd_hidden* hidden, const bd_weight* weight
 int bd_verify_step(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft, const bd_eps_grid* eps,
                    int32_t* out_tokens, float* out_p_draft, float* out_entropy, uint32_t* out_accept,
                    int32_t* out_accepted, const bd_exec* exec) {
+  bd::TraceRange trace("bd_verify_step");
   const int variant = exec ? exec->variant : 0;
   if (exec && (exec->flags != 0 || exec->out_counts != nullptr)) return BD_ERR_ARG;
   VerifyCall vc;

@@ -9,6 +9,7 @@
 //                     no position cleared tau_k, and p is the masked position of
 //                     highest confidence (lowest position on ties)         (App. B.2)
 // with one warp ballot per tau (two for blocks longer than 32).
+#include "checks.h"
 #include "kernels.h"
 
 namespace bd {
@@ -39,8 +40,10 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
     const int g = threadIdx.x / Lp;
     float m = -INFINITY, s = 0.f;
     int arg = 0x7fffffff;
-    const int r = jj < L ? a.rowpos[base + jj] : -1;
-    if (r >= 0) {
+    // partial slots the workspace holds (index checks of the bounds-checked build)
+    const int64_t part_n = static_cast<int64_t>(a.plan.cpu) * (a.plan.G < a.plan.n_vt ? a.plan.G : a.plan.n_vt) * a.P;
+    const int r = jj < L && index_ok(base + jj, a.P, a.status) ? a.rowpos[base + jj] : -1;
+    if (r >= 0 && index_ok(r, a.P, a.status)) {
       const int ns = slots_of_row(a.plan, n_rows, r);
       int slot = g;
       for (; slot + 3 * groups < ns; slot += 4 * groups) {
@@ -49,16 +52,17 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           const int64_t o = static_cast<int64_t>(slot + u * groups) * a.P + r;
-          pm[u] = a.part_m[o];
-          ps[u] = a.part_s[o];
-          pa[u] = a.part_a[o];
+          const bool in = index_ok(o, part_n, a.status);
+          pm[u] = in ? a.part_m[o] : -INFINITY;
+          ps[u] = in ? a.part_s[o] : 0.f;
+          pa[u] = in ? a.part_a[o] : 0x7fffffff;
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) softmax_combine(m, s, arg, pm[u], ps[u], pa[u]);
       }
       for (; slot < ns; slot += groups) {
         const int64_t o = static_cast<int64_t>(slot) * a.P + r;
-        softmax_combine(m, s, arg, a.part_m[o], a.part_s[o], a.part_a[o]);
+        if (index_ok(o, part_n, a.status)) softmax_combine(m, s, arg, a.part_m[o], a.part_s[o], a.part_a[o]);
       }
     }
     if (jj < L) {

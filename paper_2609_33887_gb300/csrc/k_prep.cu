@@ -1,6 +1,7 @@
 // Preparation kernels of the commit step: compaction of the still-masked
 // positions of active blocks, packing of their hidden rows, and the FP8 e4m3
 // and NVFP4 -> bf16 weight decodes of the precision levers.
+#include "checks.h"
 #include "kernels.h"
 
 namespace bd {
@@ -47,7 +48,8 @@ template <int FMT>  // the packed row format (ROWS_*); one instantiation per for
 __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags, int P, int block_len, int chunk,
     const __nv_bfloat16* __restrict__ hidden, int64_t ld, int d, __nv_bfloat16* __restrict__ hc, int64_t ldc,
-    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale) {
+    int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale,
+    uint32_t* __restrict__ status) {
   __shared__ int red[PREP_THREADS / 32];
   __shared__ int warp_excl[PREP_THREADS / 32];
   __shared__ int rows_s[2048];
@@ -93,7 +95,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     const int p = q0 + i;
     if (p < p1) {
       if (live_at(pos_masked, block_flags, p, block_len)) {
-        idx[r] = p;
+        if (index_ok(r, P, status)) idx[r] = p;
         rowpos[p] = r;
         if (r - prefix < 2048) rows_s[r - prefix] = p;
         ++r;
@@ -114,6 +116,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // after scaling is exact in f16), s at most 126 so 2^-s stays a normal
     // float; tok_scale = 2^-s, 0 for an all-zero row.
     for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+      if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
@@ -161,6 +164,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // 0 and scale 0. Each float32 step is one correctly rounded operation.
     uint8_t* hq = reinterpret_cast<uint8_t*>(hc);  // ldc counts bytes here
     for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+      if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
@@ -201,6 +205,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
 
   // 3. copy the chunk's live rows, one warp per row, 16-byte vectors
   for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+    if (!index_ok(prefix + i, P, status)) continue;
     const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
     const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
     __nv_bfloat16* dst = hc + static_cast<int64_t>(prefix + i) * ldc;
@@ -221,7 +226,8 @@ int prep_chunk(int P, int sm_count) {
 
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale, int row_format) {
+                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale, int row_format,
+                             uint32_t* status) {
   if (row_format != ROWS_BF16 && (tok_scale == nullptr || hc == nullptr)) return cudaErrorInvalidValue;
   const int chunk = prep_chunk(P, sm_count);
   const int grid = (P + chunk - 1) / chunk;
@@ -230,7 +236,7 @@ cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_fla
                                           : prep_rows_kernel<ROWS_BF16>;
   kern<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
                                       static_cast<const __nv_bfloat16*>(hidden), ld, d,
-                                      static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows, tok_scale);
+                                      static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows, tok_scale, status);
   return cudaGetLastError();
 }
 

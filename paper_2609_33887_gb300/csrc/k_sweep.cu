@@ -12,6 +12,7 @@
 
 #include "bdcommit.h"
 #include "common.cuh"
+#include "trace.h"
 
 namespace {
 
@@ -130,6 +131,7 @@ int check_device() {
 extern "C" int bd_commit_sweep(const bd_window* window, const int32_t* step_tokens, const uint32_t* step_commit,
                                int32_t tau_index, uint32_t options, int32_t* out_cache_tokens,
                                int32_t* out_n_committed, int32_t* out_n_resolved, void* stream) {
+  bd::TraceRange trace("bd_commit_sweep");
   if (window == nullptr) return BD_ERR_NULL;
   const bd_window& w = *window;
   if (w.n_seq < 0 || w.n_slots < 1 || w.n_slots > MAX_SLOTS || w.block_len < 1 || w.block_len > 64)

@@ -29,7 +29,7 @@ enum : int { ROWS_BF16 = 0, ROWS_E4M3 = 1, ROWS_F16_POW2 = 2 };
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
                              int* n_rows, int sm_count, cudaStream_t st, float* tok_scale = nullptr,
-                             int row_format = ROWS_BF16);
+                             int row_format = ROWS_BF16, uint32_t* status = nullptr);
 
 // Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
@@ -138,6 +138,7 @@ struct CommitArgs {
   float* out_conf;
   uint32_t* out_commit;
   int32_t* out_counts;
+  uint32_t* status = nullptr;  // device status word (index checks of the bounds-checked build)
 };
 cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st);
 

@@ -60,8 +60,24 @@ def test_library_exports_nothing_else(lib):
     assert names == declared_functions()
 
 
+def test_bounds_checked_build_exports_the_same_abi():
+    """The bounds-checked variant (-DBD_CHECKS, libbdcommit_checks.so) builds
+    and exports exactly the declared C ABI."""
+    if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+        pytest.skip("no CUDA toolkit")
+    from paper_2609_33887_gb300 import build as bld
+
+    path = bld.build(checks=True)
+    assert os.path.basename(path) == "libbdcommit_checks.so"
+    nm = shutil.which("nm")
+    if nm is None:
+        pytest.skip("no nm")
+    out = subprocess.run([nm, "-D", "--defined-only", path], capture_output=True, text=True).stdout
+    assert sorted(l.split()[-1] for l in out.splitlines() if " T " in l) == declared_functions()
+
+
 def test_status_strings_and_version(lib):
-    for code in range(-10, 1):
+    for code in range(-11, 1):
         s = B.bd_status_string(code)
         assert s and s != "unknown status"
     assert B.bd_status_string(-99) == "unknown status"
