@@ -17,6 +17,7 @@ host cores, one bounded sample of whole blocks per step.
 from __future__ import annotations
 
 import argparse
+import contextlib
 import hashlib
 import json
 import os
@@ -369,6 +370,22 @@ LEVERS = {
 }
 
 
+@contextlib.contextmanager
+def trace(name: str):
+    """An NVTX range around a region (a no-op without a tracer, or where the
+    torch build has no NVTX)."""
+    try:
+        torch.cuda.nvtx.range_push(name)
+        pushed = True
+    except Exception:  # noqa: BLE001 - tracing is optional
+        pushed = False
+    try:
+        yield
+    finally:
+        if pushed:
+            torch.cuda.nvtx.range_pop()
+
+
 def fp8_gemm_tflops(dev, stream, n=8192, reps=30):
     """Dense E4M3 x E4M3 -> bf16 GEMM throughput of the vendor library
     (torch._scaled_mm, n x n x n, random codes) on this GPU, for the W8A8
@@ -546,15 +563,14 @@ def run_ours(args):
         pg.barrier()
     torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    torch.cuda.nvtx.range_push(f"timed region: {K} steps")  # trace range (no-op without a tracer)
-    t_start.record(stream)
-    if graph is None:
-        for i in range(K):
-            step(ev=evs[i])
-    else:
-        graph.replay()
-    t_end.record(stream)
-    torch.cuda.nvtx.range_pop()
+    with trace(f"timed region: {K} steps"):
+        t_start.record(stream)
+        if graph is None:
+            for i in range(K):
+                step(ev=evs[i])
+        else:
+            graph.replay()
+        t_end.record(stream)
     torch.cuda.synchronize()
     if pg:
         pg.barrier()
@@ -734,11 +750,11 @@ def run_ours(args):
                "sample": f"{passes} pass(es) over {len(blocks)} whole blocks of {cfg.name} ({tot_n} masked "
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
-    with torch.cuda.nvtx.range("redline"):
+    with trace("redline"):
         redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
-    with torch.cuda.nvtx.range("verify"):
+    with trace("verify"):
         verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
-    with torch.cuda.nvtx.range("precision levers"):
+    with trace("precision levers"):
         levers = {k: lever_timing(dev, stream, k) for k in LEVERS} if rank == 0 and not args.no_verify else {}
 
     if rank == 0:
