@@ -2,13 +2,20 @@
 confidence + multi-threshold commit) on GB300, as masked positions per second.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--config NAME] [--no-graph]
+                    [--config NAME] [--no-graph] [--no-configs]
 
 One step = one bd_commit_step over one window of the workload (compaction,
 packing, LM head with the online softmax epilogue, merge and commit for the
-whole threshold grid). With N > 1 (torchrun, one rank per GPU) every rank
-runs its own independent window: the step shards by sequence with no data
-exchange, so scaling is weak. Rank 0 prints one JSON line.
+whole threshold grid). The headline workload is the largest that fits one
+GPU: 256 sequences x 8 slots x 64 positions, d = 5120, V = 157184, an E4M3
+head with per-row scales and bf16 hidden states (W8A16). The line's
+`configs` object reports each of the other four workloads the same way (its
+own positions/s, LM-head time and roofline fractions), and `sustained` runs
+two of them back to back for seconds, in the power-capped steady state.
+
+With N > 1 (torchrun, one rank per GPU) every rank runs its own independent
+window: the step shards by sequence with no data exchange, so scaling is
+weak. Rank 0 prints one JSON line.
 
 The reference arm (--impl reference) times the float64 CPU oracle on the
 host cores, one bounded sample of whole blocks per step.
@@ -32,14 +39,19 @@ import torch
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from workloads import B8X2X32_BF16, by_name, generate  # noqa: E402
+from workloads import B256X8X64_E4M3, B64X4X64_BF16, B8X2X32_BF16, CONFIGS, by_name, generate  # noqa: E402
 
-DEFAULT_CONFIG = B8X2X32_BF16.name
+DEFAULT_CONFIG = B256X8X64_E4M3.name
 METRIC = "masked positions/s through fused LM-head+confidence+commit"
 UNIT = "positions/s"
-# the LM-head kernel the automatic choice runs on the 8x2x32 window (the CTA-pair kernel)
-KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_pair.cu", "paper_2609_33887_gb300/csrc/common.cuh"]
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_pair_traffic.txt")
+# the arithmetic type the path computes in, per head format
+DTYPE_OF = {"f32": "f32", "bf16": "bf16", "e4m3": "e4m3xbf16", "nvfp4": "nvfp4xbf16"}
+# workloads also run back to back for seconds (power-capped steady state)
+SUSTAINED = (B8X2X32_BF16.name, B64X4X64_BF16.name)
+# sources of the LM-head kernels (the traffic records name the hash of these)
+KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_pair.cu", "paper_2609_33887_gb300/csrc/k_lmhead_tc.cu",
+                  "paper_2609_33887_gb300/csrc/common.cuh"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_traffic.txt")
 
 
 def parse_args():
@@ -55,6 +67,8 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-verify", action="store_true",
                     help="skip the speculative-verification and precision-lever (NVFP4, E4M3, W8A8) measurements")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the other workloads and the sustained legs")
     return ap.parse_args()
 
 
@@ -106,22 +120,31 @@ def kernel_hash():
 
 
 def recorded_traffic(config_name):
-    """DRAM bytes per LM-head launch from a committed ncu summary, if it was
-    taken on the current kernel source for this workload; else None."""
+    """DRAM bytes per LM-head launch from a committed ncu summary (records of
+    `key: value` lines separated by blank lines), if one was taken on the
+    current kernel sources for this workload; else None."""
     if not os.path.exists(TRAFFIC_FILE):
         return None
-    rec = {}
+    recs, rec = [], {}
     with open(TRAFFIC_FILE) as f:
         for line in f:
-            if ":" in line and not line.startswith("#"):
+            if not line.strip():
+                if rec:
+                    recs.append(rec)
+                rec = {}
+            elif ":" in line and not line.startswith("#"):
                 k, v = line.split(":", 1)
                 rec[k.strip()] = v.strip()
-    if rec.get("kernel_sha256_16") != kernel_hash() or rec.get("workload") != config_name:
-        return None
-    try:
-        return float(rec["dram_bytes_per_launch"])
-    except (KeyError, ValueError):
-        return None
+    if rec:
+        recs.append(rec)
+    h = kernel_hash()
+    for rec in recs:
+        if rec.get("kernel_sha256_16") == h and rec.get("workload") == config_name:
+            try:
+                return float(rec["dram_bytes_per_launch"])
+            except (KeyError, ValueError):
+                return None
+    return None
 
 
 class ClockSampler:
@@ -240,8 +263,7 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / max(1, args.steps),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
-                   "d": cfg.d, "V": cfg.V, "T": len(cfg.tau), "inputs_sha256": wl.digests()},
+        "config": config_object(cfg, wl, masked_count(wl), world),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                          "sample": f"{n_blocks} whole block(s) per step of {cfg.name}; head decoded to float64 "
                                    "once, outside the timed steps"},
@@ -363,7 +385,9 @@ LEVERS = {
               "codes streamed by TMA and decoded exactly to f16 inside the LM-head kernel (f16 MMA, token rows "
               "scaled by a power of two per row); bound: the converter warps"),
     "e4m3": ("b8x2x32_d2048_v151936_e4m3",
-             "W8A16: E4M3 codes streamed by TMA and decoded exactly to f16 inside the LM-head kernel (f16 MMA)"),
+             "W8A16 on the 8-bit tensor path: E4M3 codes read by TMA straight into the MMA operand; each bf16 row "
+             "packed as two E4M3 terms (exact above 2^-10 of the row's largest), both multiplied by the head "
+             "(tcgen05.mma kind::f8f6f4) into one fp32 accumulator"),
     "w8a8": ("b8x2x32_d2048_v151936_e4m3",
              "W8A8: packed rows quantised to E4M3 per row by the compaction kernel, E4M3 x E4M3 on the "
              "8-bit tensor path (tcgen05.mma kind::f8f6f4), both scales applied to the fp32 logits"),
@@ -482,9 +506,302 @@ def lever_timing(dev, stream, lever: str) -> dict:
     return out
 
 
+def config_object(cfg, wl_host, n_masked, world):
+    """The workload description both arms print (identical keys and values)."""
+    wbytes = {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype]
+    return {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
+            "masked_positions_per_rank": int(n_masked), "d": cfg.d, "V": cfg.V, "T": len(cfg.tau),
+            "head_dtype": cfg.weight_dtype, "hidden_dtype": cfg.hidden_dtype,
+            "parallelism": f"independent windows x{world}",
+            "l2": ("inputs larger than L2 (the LM head is %.0f MB, read every step)" if cfg.V * cfg.d * wbytes > 129e6
+                   else "no flush: the %.0f MB head stays in L2 between steps (a launch-latency-bound workload)")
+                  % (cfg.V * cfg.d * wbytes / 1e6),
+            "inputs_sha256": wl_host.digests()}
+
+
+def masked_count(wl_host):
+    cfg = wl_host.cfg
+    return int(((wl_host.pos_masked != 0) &
+                (torch.repeat_interleave(wl_host.block_flags & 1, cfg.block_len) != 0)).sum())
+
+
+def launches_per_step(cfg):
+    """Library kernels per commit step: compaction + row packing, LM head, merge +
+    commit, plus the decode of an NVFP4 head where the LM-head kernel reads a
+    bf16 copy (the automatic choice decodes it inside the kernel for windows of
+    at most 8192 positions; E4M3 heads are read as they are at every size).
+    The counts reset is a runtime memset, not a kernel of the library."""
+    decoded = cfg.weight_dtype == "nvfp4" and cfg.P > 8192
+    return 3 + (1 if decoded else 0)
+
+
+class StepRunner:
+    """One workload resident on the device with its workspace and outputs."""
+
+    def __init__(self, cfg, wl_host, dev):
+        import paper_2609_33887_gb300 as bdc
+
+        self.B = bdc.bdcommit
+        self.cfg = cfg
+        self.wl_host = wl_host
+        self.wl = wl_host.to(dev)
+        self.dev = dev
+        wl, P, T = self.wl, cfg.P, len(cfg.tau)
+        ws_bytes = bdc.bd_workspace_size(wl.hidden, wl.weight, wl.weight_scale, wl.pos_masked, wl.block_flags,
+                                         cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau)
+        self.workspace = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+        self.tokens = torch.empty(P, dtype=torch.int32, device=dev)
+        self.conf = torch.empty(P, dtype=torch.float32, device=dev)
+        self.commit = torch.empty(P, dtype=torch.int32, device=dev)
+        self.counts = torch.empty((cfg.n_seq, T), dtype=torch.int32, device=dev)
+        self.n_masked = masked_count(wl_host)
+
+    def step(self, ev=None, hidden=None, pm=None, bf=None, outs=None):
+        cfg, wl = self.cfg, self.wl
+        o = outs or (self.tokens, self.conf, self.commit, self.counts)
+        rc = self.B.bd_commit_step_ex(wl.hidden if hidden is None else hidden, wl.weight, wl.weight_scale,
+                                      wl.pos_masked if pm is None else pm, wl.block_flags if bf is None else bf,
+                                      cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau,
+                                      o[0], o[1], o[2], stream=torch.cuda.current_stream(),
+                                      workspace=self.workspace, out_counts=o[3], lmhead_events=ev)
+        if rc != 0:
+            raise self.B.BdError(rc)
+
+    def check_status(self, where):
+        st = self.B.bd_get_device_status(torch.cuda.current_stream())
+        if st != 0:
+            raise self.B.BdError(st, where)
+
+    def capture(self, n):
+        """n steps as one CUDA graph (the serving engine also replays captured graphs)."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for _ in range(n):
+                self.step()
+        torch.cuda.synchronize()
+        return g
+
+    def lmhead_ms(self, n=24):
+        """The LM-head kernel's own duration, CUDA events on the launching stream
+        around each of n eager steps (outside any graph: an event node between two
+        kernels would cancel their programmatic launch overlap in the graph)."""
+        stream = torch.cuda.current_stream()
+        evs = timing_events(n, stream)
+        for ev in evs:
+            self.step(ev=ev)
+        torch.cuda.synchronize()
+        self.check_status("LM-head timing")
+        return [a.elapsed_time(b) for a, b in evs]
+
+
+def roofline_of(cfg, n_masked, lm_ms, traffic=None):
+    """Roofline of the LM-head kernel: the algorithmic FLOPs (2 N d V) or bytes
+    per launch over its mean CUDA-event duration, against the measured peak."""
+    hbm_gbs, tc_tflops, tc_sus, peak_src = peaks()
+    flops, abytes = algorithmic(cfg, n_masked)
+    lm_s = statistics.mean(lm_ms) / 1e3
+    t_tc = flops / (tc_tflops * 1e12)
+    t_hbm = abytes / (hbm_gbs * 1e9)
+    if t_tc >= t_hbm:
+        achieved = flops / lm_s / 1e12
+        roof = {"bound": "tensor", "achieved": achieved, "peak": tc_tflops, "unit": "TFLOP/s",
+                "frac": achieved / tc_tflops, "traffic": traffic,
+                "peak_source": f"bf16_tflops (burst) of {peak_src}",
+                "frac_of_sustained": (achieved / tc_sus) if tc_sus else None}
+    else:
+        achieved = abytes / lm_s / 1e9
+        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
+                "frac": achieved / hbm_gbs, "traffic": traffic, "peak_source": f"hbm_gbs of {peak_src}"}
+    roof["lmhead_ms_avg"] = statistics.mean(lm_ms)
+    roof["lmhead_ms_median"] = statistics.median(lm_ms)
+    roof["lmhead_launches_timed"] = len(lm_ms)
+    roof["hbm_view"] = {"algorithmic_bytes": abytes, "achieved_gbs": abytes / lm_s / 1e9,
+                        "frac": abytes / lm_s / 1e9 / hbm_gbs,
+                        # against the nominal HBM3e figure, for context (the measured copy is the peak)
+                        "frac_of_nominal_7900": abytes / lm_s / 1e9 / 7900.0}
+    roof["tensor_view"] = {"algorithmic_flops": flops, "achieved_tflops": flops / lm_s / 1e12,
+                           "frac": flops / lm_s / 1e12 / tc_tflops,
+                           "frac_of_sustained": (flops / lm_s / 1e12 / tc_sus) if tc_sus else None}
+    roof["traffic_over_algorithmic"] = (traffic / abytes) if traffic else None
+    roof["kernel_sha256_16"] = kernel_hash()
+    return roof
+
+
+def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
+    """One of the other workloads: positions/s over a graph-replayed timed region
+    of at least `steps` steps and ~min_s seconds, and the LM-head roofline from
+    24 event-timed launches."""
+    wl_host = generate(cfg)
+    r = StepRunner(cfg, wl_host, dev)
+    for _ in range(warmup):
+        r.step()
+    torch.cuda.synchronize()
+    r.check_status("warm-up")
+    t0 = time.perf_counter()
+    for _ in range(3):
+        r.step()
+    torch.cuda.synchronize()
+    est = (time.perf_counter() - t0) / 3
+    k = int(min(2000, max(steps, min_s / max(est, 1e-6))))
+    g = r.capture(k)
+    g.replay()  # warm replay
+    torch.cuda.synchronize()
+    stream = torch.cuda.current_stream()
+    (e0, e1), = timing_events(1, stream)
+    e0.record(stream)
+    g.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    r.check_status("timed region")
+    ms = e0.elapsed_time(e1) / k
+    lm = r.lmhead_ms()
+    roof = roofline_of(cfg, r.n_masked, lm, recorded_traffic(cfg.name))
+    out = {"positions_per_s": r.n_masked / (ms / 1e3), "ms_per_step": ms, "steps": k,
+           "masked_positions": r.n_masked, "lmhead_us": roof["lmhead_ms_avg"] * 1e3,
+           "tensor_frac": roof["tensor_view"]["frac"], "hbm_frac": roof["hbm_view"]["frac"],
+           "traffic_over_algorithmic": roof["traffic_over_algorithmic"], "roofline": roof,
+           "gpu_launches_per_step": launches_per_step(cfg)}
+    del g, r
+    torch.cuda.empty_cache()
+    return out
+
+
+def sustained_leg(cfg, dev, gpu_index, seconds=3.0):
+    """Back-to-back commit steps for >= `seconds` (the power-capped steady
+    state a serving loop sees), with the clocks sampled meanwhile; the step's
+    tensor rate against the measured sustained bf16 peak."""
+    wl_host = generate(cfg)
+    r = StepRunner(cfg, wl_host, dev)
+    for _ in range(5):
+        r.step()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(3):
+        r.step()
+    torch.cuda.synchronize()
+    est = (time.perf_counter() - t0) / 3
+    per_graph = int(min(500, max(1, 0.25 / max(est, 1e-6))))
+    g = r.capture(per_graph)
+    stream = torch.cuda.current_stream()
+    sampler = ClockSampler(gpu_index)
+    sampler.start()
+    (e0, e1), = timing_events(1, stream)
+    e0.record(stream)
+    n_rep, t_start = 0, time.perf_counter()
+    while time.perf_counter() - t_start < seconds or n_rep < 2:
+        g.replay()
+        n_rep += 1
+        if n_rep % 4 == 0:
+            torch.cuda.synchronize()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    r.check_status("sustained leg")
+    steps = n_rep * per_graph
+    ms = e0.elapsed_time(e1) / steps
+    _, tc_tflops, tc_sus, src = peaks()
+    flops, abytes = algorithmic(cfg, r.n_masked)
+    out = {"workload": cfg.name, "seconds": e0.elapsed_time(e1) / 1e3, "steps": steps, "ms_per_step": ms,
+           "positions_per_s": r.n_masked / (ms / 1e3),
+           "step_tflops": flops / (ms / 1e3) / 1e12,
+           "step_frac_of_sustained_bf16": (flops / (ms / 1e3) / 1e12 / tc_sus) if tc_sus else None,
+           "step_frac_of_burst_bf16": flops / (ms / 1e3) / 1e12 / tc_tflops,
+           "step_hbm_gbs": abytes / (ms / 1e3) / 1e9, "peak_source": src, "clocks": clocks}
+    del g, r
+    torch.cuda.empty_cache()
+    return out
+
+
+def e2e_leg(r, K, W, pg, dev):
+    """The metric end to end through the public call with host buffers: every
+    step copies its inputs (hidden states and mask state) in from pinned host
+    memory and its outputs (tokens, conf, commit, counts) out to pinned host
+    memory. The copies are double-buffered on two copy streams, ordered by
+    events, so the input copy of step i + 1 and the output copy of step i - 1
+    overlap the kernels of step i, as a serving loop would run them."""
+    cfg, wl_host, P, T = r.cfg, r.wl_host, r.cfg.P, len(r.cfg.tau)
+    h_host = wl_host.hidden.pin_memory()
+    pm_host = wl_host.pos_masked.pin_memory()
+    bf_host = wl_host.block_flags.pin_memory()
+    bufs = []
+    for _ in range(2):
+        bufs.append({
+            "h": torch.empty_like(r.wl.hidden), "pm": torch.empty_like(r.wl.pos_masked),
+            "bf": torch.empty_like(r.wl.block_flags),
+            "out": [torch.empty(P, dtype=torch.int32, device=dev), torch.empty(P, dtype=torch.float32, device=dev),
+                    torch.empty(P, dtype=torch.int32, device=dev),
+                    torch.empty((cfg.n_seq, T), dtype=torch.int32, device=dev)],
+            "host": [torch.empty(P, dtype=torch.int32).pin_memory(),
+                     torch.empty(P, dtype=torch.float32).pin_memory(),
+                     torch.empty(P, dtype=torch.int32).pin_memory(),
+                     torch.empty((cfg.n_seq, T), dtype=torch.int32).pin_memory()],
+        })
+    c_in, c_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
+    evs = [torch.cuda.Event() for _ in range(6)]
+
+    def e2e_steps(n):
+        # the stream current at call time: inside a graph capture, the capture stream
+        stream = torch.cuda.current_stream()
+        comp, outd, inr = evs[0:2], evs[2:4], evs[4:6]
+        fork = torch.cuda.Event()
+        fork.record(stream)
+        c_in.wait_event(fork)
+        c_out.wait_event(fork)
+        for i in range(n):
+            b = i & 1
+            u = bufs[b]
+            with torch.cuda.stream(c_in):
+                if i >= 2:
+                    c_in.wait_event(comp[b])  # step i - 2 no longer reads these inputs
+                u["h"].copy_(h_host, non_blocking=True)
+                u["pm"].copy_(pm_host, non_blocking=True)
+                u["bf"].copy_(bf_host, non_blocking=True)
+                inr[b].record(c_in)
+            stream.wait_event(inr[b])
+            if i >= 2:
+                stream.wait_event(outd[b])  # the outputs of step i - 2 have been copied out
+            r.step(hidden=u["h"], pm=u["pm"], bf=u["bf"], outs=u["out"])
+            comp[b].record(stream)
+            with torch.cuda.stream(c_out):
+                c_out.wait_event(comp[b])
+                for hst, d_ in zip(u["host"], u["out"]):
+                    hst.copy_(d_, non_blocking=True)
+                outd[b].record(c_out)
+        stream.wait_stream(c_in)
+        stream.wait_stream(c_out)
+
+    e2e_steps(W)
+    torch.cuda.synchronize()
+    egraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(egraph):
+        e2e_steps(K)
+    torch.cuda.synchronize()
+    if pg:
+        pg.barrier()
+    stream = torch.cuda.current_stream()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    egraph.replay()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    r.check_status("e2e")
+    e_ms, total = aggregate_over_ranks(e0.elapsed_time(e1), r.n_masked, pg, dev)
+    h2d = h_host.numel() * h_host.element_size() + pm_host.numel() + bf_host.numel()
+    d2h = sum(o.numel() * o.element_size() for o in bufs[0]["host"])
+    # the results of the last step really arrived in host memory
+    last = bufs[(K - 1) & 1]
+    assert torch.equal(last["host"][0], last["out"][0].cpu())
+    out = {"value": total * K / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+           "d2h_bytes_per_step": int(d2h),
+           "note": "pinned host hidden states + mask state in, tokens/conf/commit/counts out, every step; "
+                   "double-buffered on two copy streams so copies overlap the neighbouring steps' kernels; "
+                   "LM-head weights stay resident in HBM; the K steps replayed as one CUDA graph"}
+    del egraph, bufs
+    return out
+
+
 def run_ours(args):
     import paper_2609_33887_gb300 as bdc
-    from paper_2609_33887_gb300 import bdcommit as B
 
     rank, world, local = dist_env()
     if not torch.cuda.is_available():
@@ -498,76 +815,35 @@ def run_ours(args):
         dist.init_process_group("nccl", device_id=dev)
         pg = dist
     bdc.load_library()
+    vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x]
+    gpu_index = vis[local] if local < len(vis) else str(local)
 
     cfg = by_name(args.config)
     # each rank serves its own window (independent sequences): weak scaling
     from dataclasses import replace
 
     wl_host = generate(replace(cfg, seed=cfg.seed + 1000 * rank) if rank else cfg)
-    wl = wl_host.to(dev)
-    P, T = cfg.P, len(cfg.tau)
-    n_masked = int(((wl_host.pos_masked != 0) &
-                    (torch.repeat_interleave(wl_host.block_flags & 1, cfg.block_len) != 0)).sum())
-    stream = torch.cuda.current_stream()
-    ws_bytes = bdc.bd_workspace_size(wl.hidden, wl.weight, wl.weight_scale, wl.pos_masked, wl.block_flags,
-                                     cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau)
-    workspace = torch.empty(ws_bytes, dtype=torch.uint8, device=dev)
-    tokens = torch.empty(P, dtype=torch.int32, device=dev)
-    conf = torch.empty(P, dtype=torch.float32, device=dev)
-    commit = torch.empty(P, dtype=torch.int32, device=dev)
-    counts = torch.empty((cfg.n_seq, T), dtype=torch.int32, device=dev)
-
-    def step(h=None, ev=None):
-        rc = B.bd_commit_step_ex(wl.hidden if h is None else h, wl.weight, wl.weight_scale, wl.pos_masked,
-                                 wl.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
-                                 cfg.tau, tokens, conf, commit, stream=torch.cuda.current_stream(),
-                                 workspace=workspace, out_counts=counts, lmhead_events=ev)
-        if rc != 0:
-            raise B.BdError(rc)
-
-    # library kernels per step: compaction + row packing, LM head, merge + commit
-    # (+ the e4m3 decode); the counts reset is a runtime memset, not one of ours
-    launches_per_step = 3 + (1 if cfg.weight_dtype == "e4m3" else 0)
+    r = StepRunner(cfg, wl_host, dev)
     K, W = args.steps, args.warmup
     for _ in range(W):
-        step()
+        r.step()
     torch.cuda.synchronize()
-    st = B.bd_get_device_status(stream)
-    if st != 0:
-        raise B.BdError(st, "warm-up")
+    r.check_status("warm-up")
+    graph = r.capture(K) if args.graph else None
 
-    # LM-head events on every EVENT_STRIDE-th step of the timed region (on the
-    # launching stream): an event node between two kernels turns their
-    # programmatic (overlapped) launch back into full serialisation, so timing
-    # every step would slow every step down
-    EVENT_STRIDE = 10
-    ev_steps = list(range(0, K, EVENT_STRIDE))
-    evs_list = timing_events(len(ev_steps), stream)
-    evs = [None] * K
-    for j, i in enumerate(ev_steps):
-        evs[i] = evs_list[j]
-    graph = None
-    if args.graph:
-        # the K timed steps as one CUDA graph (the serving engine also replays captured graphs)
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            for i in range(K):
-                step(ev=evs[i])
-        torch.cuda.synchronize()
-
-    # ---- device-resident timed region
-    vis = [x for x in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if x]
-    sampler = ClockSampler(vis[local] if local < len(vis) else str(local))
+    # ---- device-resident timed region: exactly K steps
+    sampler = ClockSampler(gpu_index)
     sampler.start()
     if pg:
         pg.barrier()
+    stream = torch.cuda.current_stream()
     torch.cuda.synchronize()
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with trace(f"timed region: {K} steps"):
         t_start.record(stream)
         if graph is None:
-            for i in range(K):
-                step(ev=evs[i])
+            for _ in range(K):
+                r.step()
         else:
             graph.replay()
         t_end.record(stream)
@@ -576,182 +852,58 @@ def run_ours(args):
         pg.barrier()
     clocks = sampler.stop()
     elapsed_ms = t_start.elapsed_time(t_end)
-    lm_ms = [a.elapsed_time(b) for a, b in evs_list]
-    st = B.bd_get_device_status(stream)
-    if st != 0:
-        raise B.BdError(st, "timed region")
-    elapsed_ms, total_masked = aggregate_over_ranks(elapsed_ms, n_masked, pg, dev)
+    r.check_status("timed region")
+    elapsed_ms, total_masked = aggregate_over_ranks(elapsed_ms, r.n_masked, pg, dev)
     ms_per_step = elapsed_ms / K
     value = total_masked * K / (elapsed_ms / 1e3)
+    del graph
+
+    # ---- the LM head's own duration (roofline), outside the timed region
+    with trace("LM-head events"):
+        lm = r.lmhead_ms(max(24, min(K, 200)))
+    roof = roofline_of(cfg, r.n_masked, lm, recorded_traffic(cfg.name))
 
     # ---- end to end through the public call with host buffers
     e2e = None
     if not args.no_e2e:
-        # Every step copies its inputs (hidden states and mask state) in from
-        # pinned host memory and its outputs out to pinned host memory. The
-        # copies are double-buffered on two copy streams, ordered by events, so
-        # the input copy of step i + 1 and the output copy of step i - 1 overlap
-        # the kernels of step i, as a serving loop would run them.
-        h_host = wl_host.hidden.pin_memory()
-        pm_host = wl_host.pos_masked.pin_memory()
-        bf_host = wl_host.block_flags.pin_memory()
-        bufs = []
-        for _ in range(2):
-            bufs.append({
-                "h": torch.empty_like(wl.hidden), "pm": torch.empty_like(wl.pos_masked),
-                "bf": torch.empty_like(wl.block_flags),
-                "out": [torch.empty(P, dtype=torch.int32, device=dev), torch.empty(P, dtype=torch.float32, device=dev),
-                        torch.empty(P, dtype=torch.int32, device=dev),
-                        torch.empty((cfg.n_seq, T), dtype=torch.int32, device=dev)],
-                "host": [torch.empty(P, dtype=torch.int32).pin_memory(),
-                         torch.empty(P, dtype=torch.float32).pin_memory(),
-                         torch.empty(P, dtype=torch.int32).pin_memory(),
-                         torch.empty((cfg.n_seq, T), dtype=torch.int32).pin_memory()],
-            })
-        c_in, c_out = torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev)
-        n_events = 3 * 2
-        evs = [torch.cuda.Event() for _ in range(n_events)]
-
-        def e2e_steps(n):
-            # the stream current at call time: inside a graph capture, the capture stream
-            stream = torch.cuda.current_stream()
-            comp, outd, inr = evs[0:2], evs[2:4], evs[4:6]
-            fork = torch.cuda.Event()
-            fork.record(stream)
-            c_in.wait_event(fork)
-            c_out.wait_event(fork)
-            for i in range(n):
-                b = i & 1
-                u = bufs[b]
-                with torch.cuda.stream(c_in):
-                    if i >= 2:
-                        c_in.wait_event(comp[b])  # step i - 2 no longer reads these inputs
-                    u["h"].copy_(h_host, non_blocking=True)
-                    u["pm"].copy_(pm_host, non_blocking=True)
-                    u["bf"].copy_(bf_host, non_blocking=True)
-                    inr[b].record(c_in)
-                stream.wait_event(inr[b])
-                if i >= 2:
-                    stream.wait_event(outd[b])  # the outputs of step i - 2 have been copied out
-                o = u["out"]
-                rc = B.bd_commit_step_ex(u["h"], wl.weight, wl.weight_scale, u["pm"], u["bf"], cfg.n_seq,
-                                         cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau, o[0], o[1], o[2],
-                                         stream=stream, workspace=workspace, out_counts=o[3])
-                if rc != 0:
-                    raise B.BdError(rc, "e2e step")
-                comp[b].record(stream)
-                with torch.cuda.stream(c_out):
-                    c_out.wait_event(comp[b])
-                    for hst, d_ in zip(u["host"], o):
-                        hst.copy_(d_, non_blocking=True)
-                    outd[b].record(c_out)
-            stream.wait_stream(c_in)
-            stream.wait_stream(c_out)
-
-        e2e_steps(W)
-        torch.cuda.synchronize()
-        egraph = None
-        if args.graph:
-            egraph = torch.cuda.CUDAGraph()
-            with torch.cuda.graph(egraph):
-                e2e_steps(K)
-            torch.cuda.synchronize()
-        if pg:
-            pg.barrier()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        if egraph is None:
-            e2e_steps(K)
-        else:
-            egraph.replay()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        e_ms, _ = aggregate_over_ranks(e0.elapsed_time(e1), 0, pg, dev)
-        h2d = h_host.numel() * h_host.element_size() + pm_host.numel() + bf_host.numel()
-        d2h = sum(o.numel() * o.element_size() for o in bufs[0]["host"])
-        # the results of the last step really arrived: compare with a device-side step on the same inputs
-        last = bufs[(K - 1) & 1]
-        assert torch.equal(last["host"][0], last["out"][0].cpu())
-        e2e = {"value": total_masked * K / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": int(h2d),
-               "d2h_bytes_per_step": int(d2h),
-               "note": "pinned host hidden states + mask state in, tokens/conf/commit/counts out, every step; "
-                       "double-buffered on two copy streams so copies overlap the neighbouring steps' kernels; "
-                       "LM-head weights stay resident in HBM"
-                       + ("; the K steps replayed as one CUDA graph" if args.graph else "")}
-
-    # ---- the commit sweep that follows the step in a decode loop (on a copy of
-    # the window: it updates the window in place)
-    sweep = None
-    if rank == 0:
-        tok_w = torch.full((P,), -1, dtype=torch.int32, device=dev)
-        pm_w, fl_w = wl.pos_masked.clone(), wl.block_flags.clone()
-        cache_w = torch.empty(P, dtype=torch.int32, device=dev)
-        ncom_w = torch.empty(cfg.n_seq, dtype=torch.int32, device=dev)
-
-        def sweep_once():
-            rc = B.bd_commit_sweep(tok_w, pm_w, fl_w, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
-                                   tokens, commit, len(cfg.tau) - 1, B.BD_SWEEP_ADMIT | B.BD_SWEEP_ELIGIBLE_OLDEST,
-                                   cache_w, ncom_w, None, stream=stream)
-            if rc != 0:
-                raise B.BdError(rc, "bd_commit_sweep")
-
-        for _ in range(10):
-            sweep_once()
-        n_sw = 500
-        (e0, e1), = timing_events(1, stream)
-        e0.record(stream)
-        for _ in range(n_sw):
-            sweep_once()
-        e1.record(stream)
-        torch.cuda.synchronize()
-        sweep = {"us_per_launch": e0.elapsed_time(e1) * 1e3 / n_sw, "launches_timed": n_sw,
-                 "window_positions": P, "ctas": cfg.n_seq, "bound": "latency (one CTA per sequence)",
-                 "note": "bd_commit_sweep on the bench window after the timed steps, back to back on one stream"}
-
-    # ---- roofline of the dominant kernel (LM head)
-    hbm_gbs, tc_tflops, tc_sus, peak_src = peaks()
-    flops, abytes = algorithmic(cfg, n_masked)
-    lm_avg_s = statistics.mean(lm_ms) / 1e3
-    t_tc = flops / (tc_tflops * 1e12)
-    t_hbm = abytes / (hbm_gbs * 1e9)
-    traffic = recorded_traffic(cfg.name)
-    if t_tc >= t_hbm:
-        achieved = flops / lm_avg_s / 1e12
-        roof = {"bound": "tensor", "achieved": achieved, "peak": tc_tflops, "unit": "TFLOP/s",
-                "frac": achieved / tc_tflops, "traffic": traffic,
-                "peak_source": f"bf16_tflops (burst) of {peak_src}",
-                "frac_of_sustained": (achieved / tc_sus) if tc_sus else None}
-    else:
-        achieved = abytes / lm_avg_s / 1e9
-        roof = {"bound": "hbm", "achieved": achieved, "peak": hbm_gbs, "unit": "GB/s",
-                "frac": achieved / hbm_gbs, "traffic": traffic, "peak_source": f"hbm_gbs of {peak_src}"}
-    roof["lmhead_ms_avg"] = lmhead_ms = statistics.mean(lm_ms)
-    roof["lmhead_launches_timed"] = len(lm_ms)
-    roof["hbm_view"] = {"algorithmic_bytes": abytes, "achieved_gbs": abytes / lm_avg_s / 1e9,
-                        "frac": abytes / lm_avg_s / 1e9 / hbm_gbs,
-                        # against the nominal HBM3e figure, for context (the measured copy is the peak)
-                        "frac_of_nominal_7900": abytes / lm_avg_s / 1e9 / 7900.0}
-    roof["algorithmic_flops"] = flops
-    roof["kernel_sha256_16"] = kernel_hash()
+        with trace("e2e"):
+            e2e = e2e_leg(r, K, W, pg, dev)
 
     # ---- CPU baseline: the oracle on a bounded sample, rank 0 at N = 1 only
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        dt, n, blocks, w64 = oracle_sample_time(wl_host, 2)
+        dt, n, blocks, w64 = oracle_sample_time(wl_host, 1)
         target = 12.0  # seconds of oracle work
-        nb = max(1, min(cfg.n_blocks, int(2 * target / max(dt, 1e-3))))
+        nb = max(1, min(cfg.n_blocks, int(target / 4 / max(dt, 1e-3))))
         tot_t, tot_n, passes = 0.0, 0, 0
         while tot_t < target and passes < 1000:
             dt, n, blocks, _ = oracle_sample_time(wl_host, nb, seed=11 + passes, w64=w64)
             tot_t += dt
             tot_n += n
             passes += 1
+        del w64
         cpu = {"value": tot_n / tot_t, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                "sample": f"{passes} pass(es) over {len(blocks)} whole blocks of {cfg.name} ({tot_n} masked "
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
+    conf_obj = config_object(cfg, wl_host, r.n_masked, world)
+    del r
+    torch.cuda.empty_cache()
+
+    # ---- every other workload, the sustained legs and the side measurements (rank 0)
+    configs, sustained = {}, {}
+    if rank == 0 and not args.no_configs:
+        for other in CONFIGS:
+            if other.name != cfg.name:
+                with trace(f"workload {other.name}"):
+                    configs[other.name] = side_config(other, dev)
+        for name in SUSTAINED:
+            with trace(f"sustained {name}"):
+                sustained[name] = sustained_leg(by_name(name), dev, gpu_index)
     with trace("redline"):
         redline = redline_timing(with_oracle=cpu is not None) if rank == 0 else None
+    with trace("sweep"):
+        sweep = sweep_timing(dev) if rank == 0 and not args.no_verify else None
     with trace("verify"):
         verify = verify_timing(dev, stream) if rank == 0 and not args.no_verify else None
     with trace("precision levers"):
@@ -761,19 +913,19 @@ def run_ours(args):
         line = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": W,
             "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "bf16" if cfg.weight_dtype == "bf16" else ("e4m3xbf16" if cfg.weight_dtype == "e4m3" else "f32"),
-            "data": "synthetic",
-            "config": {"workload": cfg.name, "n_seq": cfg.n_seq, "n_slots": cfg.n_slots, "block_len": cfg.block_len,
-                       "masked_positions_per_rank": n_masked, "d": cfg.d, "V": cfg.V, "T": len(cfg.tau),
-                       "parallelism": f"independent windows x{world}", "graph": bool(args.graph),
-                       "l2": "inputs larger than L2 (the LM head is %.0f MB, read every step)"
-                             % (cfg.V * cfg.d * {"f32": 4, "bf16": 2, "e4m3": 1}[cfg.weight_dtype] / 1e6),
-                       "inputs_sha256": wl_host.digests()},
+            "dtype": DTYPE_OF[cfg.weight_dtype], "data": "synthetic",
+            "config": conf_obj,
+            "timing": {"graph": bool(args.graph),
+                       "region": f"{K} steps" + (" replayed as one CUDA graph" if args.graph else " launched eagerly"),
+                       "lmhead": f"{len(lm)} eager launches with CUDA events around the LM-head kernel, "
+                                 "after the timed region"},
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches_per_step * K,
+            "gpu_launches": launches_per_step(cfg) * K,
             "clocks": clocks,
+            "configs": configs or None,
+            "sustained": sustained or None,
             "redline": redline,
             "sweep": sweep,
             "verify": verify,
@@ -785,6 +937,44 @@ def run_ours(args):
     if pg:
         pg.destroy_process_group()
     return 0
+
+
+def sweep_timing(dev):
+    """bd_commit_sweep (the block-buffer update that follows the step in a
+    decode loop) on the 8 x 2 x 32 window, back to back on one stream."""
+    import paper_2609_33887_gb300 as bdc
+
+    B = bdc.bdcommit
+    cfg = B8X2X32_BF16
+    r = StepRunner(cfg, generate(cfg), dev)
+    r.step()
+    torch.cuda.synchronize()
+    P = cfg.P
+    stream = torch.cuda.current_stream()
+    tok_w = torch.full((P,), -1, dtype=torch.int32, device=dev)
+    pm_w, fl_w = r.wl.pos_masked.clone(), r.wl.block_flags.clone()
+    cache_w = torch.empty(P, dtype=torch.int32, device=dev)
+    ncom_w = torch.empty(cfg.n_seq, dtype=torch.int32, device=dev)
+
+    def sweep_once():
+        rc = B.bd_commit_sweep(tok_w, pm_w, fl_w, cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id,
+                               r.tokens, r.commit, len(cfg.tau) - 1, B.BD_SWEEP_ADMIT | B.BD_SWEEP_ELIGIBLE_OLDEST,
+                               cache_w, ncom_w, None, stream=stream)
+        if rc != 0:
+            raise B.BdError(rc, "bd_commit_sweep")
+
+    for _ in range(10):
+        sweep_once()
+    n_sw = 500
+    (e0, e1), = timing_events(1, stream)
+    e0.record(stream)
+    for _ in range(n_sw):
+        sweep_once()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return {"workload": cfg.name, "us_per_launch": e0.elapsed_time(e1) * 1e3 / n_sw, "launches_timed": n_sw,
+            "window_positions": P, "ctas": cfg.n_seq, "bound": "latency (one CTA per sequence)",
+            "note": "bd_commit_sweep after one commit step, back to back on one stream"}
 
 
 def main():

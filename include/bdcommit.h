@@ -159,19 +159,34 @@ typedef struct {
  *   lmhead_event_begin / lmhead_event_end : optional cudaEvent_t recorded on
  *                     the stream right before and after the LM-head kernel,
  *                     for timing it alone.
- *   variant         : 0 = automatic (for BF16 / E4M3 / NVFP4 heads the CTA-pair
- *                     tensor-core kernel up to 8192 window positions and the
- *                     one-CTA kernel above; the fp32 SIMT kernel for F32
- *                     heads); 1 = force
- *                     the fp32-FMA SIMT LM-head kernel; 2 = force the one-CTA
- *                     tensor-core kernel (tokens on the MMA M side); 3 = force the
- *                     CTA-pair tensor-core kernel (vocabulary on the M side).
- *                     2 and 3 need BF16 hidden states.
+ *   variant         : 0 = automatic: the CTA-pair tensor-core kernel for BF16
+ *                     heads at every window size and for E4M3 heads with
+ *                     16-byte aligned rows (see below); NVFP4 heads (and E4M3
+ *                     heads the 8-bit path cannot read) on the CTA-pair kernel
+ *                     up to 8192 window positions and the one-CTA kernel on a
+ *                     decoded bf16 copy above; the fp32 SIMT kernel for F32
+ *                     heads. 1 = force the fp32-FMA SIMT LM-head kernel; 2 =
+ *                     force the one-CTA tensor-core kernel (tokens on the MMA M
+ *                     side); 3 = force the CTA-pair tensor-core kernel
+ *                     (vocabulary on the M side). 2 and 3 need BF16 hidden
+ *                     states.
+ *                     E4M3 heads on the CTA-pair kernel (variant 0 or 3, code
+ *                     rows 16-byte aligned, dim >= 16) run on the 8-bit tensor
+ *                     path with the BF16 hidden states unchanged in value: each
+ *                     packed row is scaled by a power of two 2^s so that its
+ *                     largest magnitude lies in [128, 256) and written as two
+ *                     E4M3 terms hi = e4m3(h 2^s), lo = e4m3(h 2^s - hi); the
+ *                     head's codes multiply both terms (tcgen05.mma
+ *                     kind::f8f6f4, exact products, fp32 accumulation) and the
+ *                     logits are scaled by 2^-s and the head's row scale.
+ *                     hi + lo equals h 2^s exactly for every element of at
+ *                     least 2^-10 of its row's largest; a smaller one is off
+ *                     by at most 2^-17 of the row's largest.
  *   flags           : 0, or BD_EXEC_FP8_ACTIVATIONS (commit step only): the
  *                     W8A8 variant of the precision lever. Needs a BD_E4M3 head
  *                     (16-byte aligned, ld a multiple of 16, dim >= 16), BF16
- *                     hidden states and the CTA-pair kernel (variant 0 or 3,
- *                     windows up to 8192 positions); else BD_ERR_ARG / ALIGN.
+ *                     hidden states and the CTA-pair kernel (variant 0 or 3);
+ *                     else BD_ERR_ARG / ALIGN.
  *                     Each packed hidden row is quantised to E4M3 with one
  *                     scale per row (a = max |h|, code = e4m3(h * fl32(448 /
  *                     a)) rounding to nearest even and saturating, scale =
@@ -216,6 +231,50 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight,
 size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
                          const bd_mask_state* mask_state, const bd_tau_grid* tau_grid);
 
+/* ------------------------------------------------ vocabulary-parallel split --
+ * The head split by vocabulary rows over G ranks (or G calls on one device):
+ * rank g holds rows [offset_g, offset_g + V_g) of W. The only exchange is
+ * 12 bytes per position and rank: each rank's (max m, sum of exp(l - m),
+ * lowest argmax a) over its rows, which combine exactly as the kernels'
+ * vocabulary parts do: (m, s, a) + (m', s', a') = (M, s e^(m - M) + s' e^(m' - M),
+ * the lowest id among the maxima), with M = max(m, m'); conf = 1 / s, token = a
+ * (App. B.1: the mask-suppressed softmax over the whole vocabulary).
+ *
+ * Per-position partials, device arrays of P = n_seq * n_slots * block_len
+ * entries each (or [n_parts, P] when gathered, part g at g * P):
+ *   m : float32 max logit, -inf where the position has no prediction
+ *   s : float32 sum of exp(l - m) over the shard's rows (0 there)
+ *   a : int32 global vocabulary id of the lowest argmax (-1 there) */
+typedef struct {
+  float* m;
+  float* s;
+  int32_t* a;
+} bd_partials;
+
+/* Part 1: the LM head and its softmax statistics over one head shard. `shard`
+ * holds vocabulary rows [vocab_offset, vocab_offset + shard->vocab) of the
+ * head (any dtype bd_commit_step accepts; an E4M3 shard's scale covers its own
+ * rows); mask_state->mask_token_id is a GLOBAL id (-1 = none), suppressed by
+ * the shard that holds it. Writes `out` for every window position: the
+ * partial of the masked positions of active blocks, (-inf, 0, -1) elsewhere.
+ * exec: stream, workspace (bd_workspace_size with the shard as the head and
+ * mask_token_id -1), variant; flags, out_counts and events must be 0 / NULL.
+ * Errors as bd_commit_step_ex, plus BD_ERR_ARG for a negative offset or an
+ * offset + vocab beyond 2^30; a shard whose only row is the mask token has
+ * nothing to predict (BD_ERR_SHAPE): leave it out of the split. */
+int bd_lmhead_partials(const bd_hidden* hidden, const bd_weight* shard, int64_t vocab_offset,
+                       const bd_mask_state* mask_state, const bd_partials* out, const bd_exec* exec);
+
+/* Part 2: merges the n_parts (1..4096) shards' partials of every position,
+ * gathered as [n_parts, P] arrays (e.g. by an all-gather), and applies the
+ * commit rule of bd_commit_step for the whole threshold grid; outputs as
+ * bd_commit_step (tokens are global ids). Equal maxima in two shards go to
+ * the lower id, as in one pass. exec: stream and out_counts; workspace,
+ * flags and events must be NULL / 0. Needs no workspace. */
+int bd_merge_commit(const bd_partials* gathered, int32_t n_parts, const bd_mask_state* mask_state,
+                    const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+                    const bd_exec* exec);
+
 /* Synchronises `stream` (a cudaStream_t, NULL = legacy default), then returns
  * and clears the device-side status of the current device: BD_OK, or
  * BD_ERR_TIMEOUT if a kernel's bounded wait gave up since the last call (its
@@ -234,8 +293,10 @@ int bd_selftest_timeout(void* stream);
 /* Static English text for a status code. Never NULL. */
 const char* bd_status_string(int status);
 
-/* Frees the library-owned workspaces and status words of every device.
- * No call may be in flight. */
+/* Frees the library-owned workspaces and status words of every device, and
+ * forgets the cached device address of bd_commit_step_static's array (the
+ * next such call looks it up again, so the library stays usable after a
+ * cudaDeviceReset that follows this call). No call may be in flight. */
 int bd_shutdown(void);
 
 /* Size of the device scratch array that bd_commit_step_static works in. */
@@ -260,15 +321,32 @@ int bd_shutdown(void);
  *     cudaGetSymbolAddress (the device must be current) and caches it; make
  *     that first call before any stream capture.
  *   - Sharing: every call on a device uses the same array, which keeps the
- *     previous call's contents (the call clears the one word that must start
- *     at zero). Calls that can overlap on the GPU (different streams, or
+ *     previous call's contents (everything a call reads there it writes
+ *     first). Calls that can overlap on the GPU (different streams, or
  *     different host threads) race on the array: serialise them.
- *   - A bounded device-side wait that gives up is recorded in the array, not
- *     in the word bd_get_device_status reads. */
+ *   - Failures on the device: a bounded device-side wait that gives up is
+ *     recorded in a status word inside the array (not in the word
+ *     bd_get_device_status reads) and stays recorded, across later calls,
+ *     until bd_static_device_status reads and clears it. */
 int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* weight,
                           const bd_mask_state* mask_state, const bd_tau_grid* tau_grid,
                           int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                           void* stream);
+
+/* The device status of bd_commit_step_static on the current device (no paper
+ * counterpart; allocates nothing either). Synchronises `stream`, then returns
+ * and clears the status word in the array: BD_OK, BD_ERR_TIMEOUT if a bounded
+ * wait of any static call gave up since the last read (that call's outputs
+ * are invalid), BD_ERR_BOUNDS (bounds-checked build), or BD_ERR_CUDA.
+ * Read it after the static calls whose outputs you use. */
+int bd_static_device_status(void* stream);
+
+/* The failure-detection self-test of bd_selftest_timeout aimed at the status
+ * word of bd_commit_step_static's array (no paper counterpart): one small
+ * kernel on `stream` waits about 1 s on a barrier nothing completes and
+ * records the timeout there; the next bd_static_device_status returns
+ * BD_ERR_TIMEOUT. No fault, trap or hang is involved. */
+int bd_static_selftest_timeout(void* stream);
 
 /* ---------------------------------------------- speculative verification --
  * The same LM head and fused softmax serve the verification step of

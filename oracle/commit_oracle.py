@@ -178,7 +178,13 @@ def weights_f64(raw, dtype: str, scale: Optional[np.ndarray] = None, d: Optional
     if dtype == "e4m3":
         if scale is None:
             raise ValueError("e4m3 weights need a per-row scale")
-        return decode_e4m3(raw) * np.asarray(scale, dtype=np.float32).astype(np.float64)[:, None]
+        # decode_e4m3 of each of the 256 codes, looked up per element: the same
+        # values as decoding the matrix element by element, without its
+        # full-size temporaries (a 157184 x 5120 head would need ~40 GB)
+        table = decode_e4m3(np.arange(256, dtype=np.uint8))
+        w = table[np.asarray(raw, dtype=np.uint8)]
+        w *= np.asarray(scale, dtype=np.float32).astype(np.float64)[:, None]
+        return w
     raise ValueError(dtype)
 
 

@@ -19,6 +19,8 @@ from .bdcommit import (
     bd_commit_step_ex,
     bd_commit_sweep,
     bd_get_device_status,
+    bd_lmhead_partials,
+    bd_merge_commit,
     bd_shutdown,
     bd_status_string,
     bd_verify_step,
@@ -27,7 +29,9 @@ from .bdcommit import (
     bd_workspace_size,
     commit_step,
     commit_sweep,
+    lmhead_partials,
     load_library,
+    merge_commit,
     verify_step,
 )
 
@@ -43,6 +47,8 @@ __all__ = [
     "bd_commit_step_ex",
     "bd_commit_sweep",
     "bd_get_device_status",
+    "bd_lmhead_partials",
+    "bd_merge_commit",
     "bd_shutdown",
     "bd_status_string",
     "bd_verify_step",
@@ -52,7 +58,9 @@ __all__ = [
     "bdcommit",
     "commit_step",
     "commit_sweep",
+    "lmhead_partials",
     "load_library",
+    "merge_commit",
     "redline",
     "verify_step",
 ]

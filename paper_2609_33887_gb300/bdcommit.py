@@ -80,6 +80,10 @@ class bd_exec(ctypes.Structure):
                 ("variant", c_int32), ("flags", c_int32)]
 
 
+class bd_partials(ctypes.Structure):
+    _fields_ = [("m", c_void_p), ("s", c_void_p), ("a", c_void_p)]
+
+
 class bd_draft(ctypes.Structure):
     _fields_ = [("n_req", c_int32), ("n_draft", c_int32), ("draft", c_void_p)]
 
@@ -130,8 +134,14 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
                                                 POINTER(bd_eps_grid)]),
         "bd_commit_sweep": (c_int, [POINTER(bd_window), c_void_p, c_void_p, c_int32, ctypes.c_uint32, c_void_p,
                                     c_void_p, c_void_p, c_void_p]),
+        "bd_lmhead_partials": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), ctypes.c_int64,
+                                       POINTER(bd_mask_state), POINTER(bd_partials), POINTER(bd_exec)]),
+        "bd_merge_commit": (c_int, [POINTER(bd_partials), ctypes.c_int32, POINTER(bd_mask_state),
+                                    POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, POINTER(bd_exec)]),
         "bd_get_device_status": (c_int, [c_void_p]),
         "bd_selftest_timeout": (c_int, [c_void_p]),
+        "bd_static_device_status": (c_int, [c_void_p]),
+        "bd_static_selftest_timeout": (c_int, [c_void_p]),
         "bd_status_string": (ctypes.c_char_p, [c_int]),
         "bd_shutdown": (c_int, []),
         "bd_version": (c_int, []),
@@ -290,6 +300,89 @@ def bd_commit_step_static(hidden, weight, weight_scale, pos_masked, block_flags,
     return int(load_library().bd_commit_step_static(
         ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
         _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit), _stream_handle(stream)))
+
+
+def bd_lmhead_partials(hidden, shard, shard_scale, vocab_offset, pos_masked, block_flags, n_seq, n_slots,
+                       block_len, mask_token_id, out_m, out_s, out_a, *, stream=None, workspace=None,
+                       variant=VARIANT_AUTO) -> int:
+    """Queue part 1 of the vocabulary-parallel step: the LM head over head rows
+    [vocab_offset, vocab_offset + shard rows) and one (max, sum of exp, global
+    argmax) partial per window position into out_m / out_s / out_a (device
+    float32 / float32 / int32 [P]). mask_token_id is a global id. Returns the status."""
+    h = make_hidden(hidden)
+    w = make_weight(shard, shard_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    out = bd_partials(_ptr(out_m), _ptr(out_s), _ptr(out_a))
+    ex = bd_exec()
+    ex.stream = _stream_handle(stream)
+    if workspace is not None:
+        ex.workspace = workspace.data_ptr()
+        ex.workspace_bytes = workspace.numel() * workspace.element_size()
+    ex.variant = variant
+    return int(load_library().bd_lmhead_partials(ctypes.byref(h), ctypes.byref(w), int(vocab_offset),
+                                                 ctypes.byref(ms), ctypes.byref(out), ctypes.byref(ex)))
+
+
+def bd_merge_commit(parts_m, parts_s, parts_a, n_parts, pos_masked, block_flags, n_seq, n_slots, block_len, tau,
+                    out_tokens, out_conf, out_commit, *, stream=None, out_counts=None) -> int:
+    """Queue part 2: merge the gathered partials ([n_parts, P] device arrays)
+    of every position and apply the commit rule for the threshold grid.
+    Returns the status."""
+    g = bd_partials(_ptr(parts_m), _ptr(parts_s), _ptr(parts_a))
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, -1)
+    tg, _keep = make_tau_grid(tau)
+    ex = bd_exec()
+    ex.stream = _stream_handle(stream)
+    ex.out_counts = _ptr(out_counts)
+    return int(load_library().bd_merge_commit(ctypes.byref(g), int(n_parts), ctypes.byref(ms), ctypes.byref(tg),
+                                              _ptr(out_tokens), _ptr(out_conf), _ptr(out_commit),
+                                              ctypes.byref(ex)))
+
+
+def lmhead_partials(hidden, shard, vocab_offset, pos_masked, block_flags, n_seq, n_slots, block_len, *,
+                    shard_scale=None, mask_token_id=-1, stream=None, workspace=None, variant=VARIANT_AUTO):
+    """Allocate the per-position partials on the hidden states' device, queue
+    part 1, raise on error. Returns (m float32 [P], s float32 [P], a int32 [P])."""
+    P = n_seq * n_slots * block_len
+    dev = hidden.device
+    m = torch.empty(P, dtype=torch.float32, device=dev)
+    s_ = torch.empty(P, dtype=torch.float32, device=dev)
+    a = torch.empty(P, dtype=torch.int32, device=dev)
+    rc = bd_lmhead_partials(hidden, shard, shard_scale, vocab_offset, pos_masked, block_flags, n_seq, n_slots,
+                            block_len, mask_token_id, m, s_, a, stream=stream, workspace=workspace, variant=variant)
+    if rc != BD_OK:
+        raise BdError(rc, "bd_lmhead_partials")
+    return m, s_, a
+
+
+def merge_commit(parts_m, parts_s, parts_a, pos_masked, block_flags, n_seq, n_slots, block_len, tau, *,
+                 stream=None, counts=False):
+    """Allocate the outputs, queue part 2 on [n_parts, P] gathered partials,
+    raise on error. Returns (tokens, conf, commit, counts or None) as commit_step."""
+    P = n_seq * n_slots * block_len
+    n_parts = parts_m.numel() // max(1, P)
+    dev = parts_m.device
+    tokens = torch.empty(P, dtype=torch.int32, device=dev)
+    conf = torch.empty(P, dtype=torch.float32, device=dev)
+    commit = torch.empty(P, dtype=torch.int32, device=dev)
+    cnt = torch.empty((n_seq, len(tau)), dtype=torch.int32, device=dev) if counts else None
+    rc = bd_merge_commit(parts_m, parts_s, parts_a, n_parts, pos_masked, block_flags, n_seq, n_slots, block_len, tau,
+                         tokens, conf, commit, stream=stream, out_counts=cnt)
+    if rc != BD_OK:
+        raise BdError(rc, "bd_merge_commit")
+    return tokens, conf, commit, cnt
+
+
+def bd_static_device_status(stream=None) -> int:
+    """Synchronise `stream`, then read and clear the status word of
+    bd_commit_step_static's array (BD_OK, or BD_ERR_TIMEOUT after a bounded
+    wait of a static call gave up)."""
+    return int(load_library().bd_static_device_status(_stream_handle(stream)))
+
+
+def bd_static_selftest_timeout(stream=None) -> int:
+    """Queue the failure-detection self-test against the static array's status word."""
+    return int(load_library().bd_static_selftest_timeout(_stream_handle(stream)))
 
 
 def commit_step(hidden, weight, pos_masked, block_flags, n_seq, n_slots, block_len, tau, *,

@@ -3,6 +3,7 @@
 // step on the caller's stream.
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
@@ -82,6 +83,7 @@ struct Call {
   int64_t ldq;      // decoded e4m3 head (bf16), elements
   bool fused;       // pair kernel decodes an E4M3 / NVFP4 head itself (no bf16 copy)
   bool fp8_act = false;  // W8A8: token rows quantised to E4M3, kind::f8f6f4 MMAs on the E4M3 head
+  bool split = false;    // W8A16 on the 8-bit path: bf16 rows as two E4M3 terms times the E4M3 head
 };
 
 bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
@@ -89,7 +91,7 @@ bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) %
 int esize(int dt) { return dt == BD_F32 ? 4 : dt == BD_BF16 ? 2 : 1; }  // NVFP4: ld counts bytes
 
 bool decoded_head(const Call& c) {
-  return c.tc && !c.fused && !c.fp8_act && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4);
+  return c.tc && !c.fused && !c.fp8_act && !c.split && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4);
 }
 
 // Decodes an FP8 or NVFP4 head into the bf16 workspace copy the tensor-core
@@ -143,10 +145,13 @@ int check_head(const bd_hidden* h, const bd_weight* w, int64_t rows, int variant
   c->wdt = wdt;
   c->tc = tc;
   // automatic choice: the CTA-pair kernel (vocabulary on M, token dimension
-  // padded only to a multiple of 32) wins while the window is small; at large
-  // windows both kernels saturate the tensor pipe under the power cap and the
-  // one-CTA kernel runs slightly faster
-  c->pair = tc && (variant == 3 || (variant == 0 && rows <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30)));
+  // padded only to a multiple of 32, 256 x 256 tiles per pair at large
+  // windows) for bf16 heads at every size; heads decoded in the kernel by its
+  // converter warps only while the window is small (at large windows the
+  // one-CTA kernel on a decoded bf16 copy keeps the tensor pipe busier)
+  const bool quant_head = wdt == BD_E4M3 || wdt == BD_NVFP4;
+  c->pair = tc && (variant == 3 ||
+                   (variant == 0 && (!quant_head || rows <= env_int("BD_PAIR_MAX_P", 8192, 0, 1 << 30))));
   c->ldh = h->ld;
   c->ldw = w->ld;
   c->ldc = round_up(c->d, 8);
@@ -177,6 +182,15 @@ int check_args(const bd_hidden* h, const bd_weight* w, const bd_mask_state* ms, 
   if (ms->mask_token_id < -1 || ms->mask_token_id >= w->vocab) return BD_ERR_ARG;
   if (ms->mask_token_id >= 0 && w->vocab < 2) return BD_ERR_SHAPE;  // nothing left to predict
   if (P > 0 && (!ms->pos_masked || !ms->block_flags)) return BD_ERR_NULL;
+  // An E4M3 head on the commit step: the pair kernel multiplies its codes
+  // directly on the 8-bit tensor path, with the bf16 rows packed as two E4M3
+  // terms (needs 16-byte aligned code rows), at every window size.
+  if (c->tc && w->dtype == BD_E4M3 && (variant == 0 || variant == 3) && env_int("BD_E4M3_SPLIT", 1, 0, 1) != 0 &&
+      aligned(w->data, 16) && w->ld % 16 == 0 && w->dim >= 16) {
+    c->pair = true;
+    c->split = true;
+    c->fused = false;
+  }
   c->P = P;
   c->n_seq = ms->n_seq;
   c->n_slots = ms->n_slots;
@@ -195,27 +209,39 @@ int env_int(const char* name, int dflt, int lo, int hi) {
   return v < lo ? lo : v > hi ? hi : v;
 }
 
+// Bytes of one row of the LM head's token operand (the packed rows, or the
+// caller's rows for the SIMT kernel).
+int64_t row_operand_bytes(const Call& c) {
+  if (!c.tc) return c.d * esize(c.hdt);
+  if (c.fp8_act) return round_up(c.d, 16);
+  if (c.split) return 2 * round_up(c.d, 16);
+  return 2 * c.ldc;
+}
+
 BandPlan make_plan(const Call& c, int sm_count, int pairs) {
   BandPlan p;
   if (c.pair) {
     p.BM = 0;  // token groups derived from N on the device
     p.BN = 256;
     p.G = pairs;
-    p.GM = env_int("BD_PAIR_GM", 4, 1, pairs);
     p.cpu = 2;
   } else if (c.tc) {
     p.BM = bd::TC_BM;
     p.BN = bd::TC_BN;
     p.G = sm_count;
-    p.GM = env_int("BD_TC_GM", 8, 1, sm_count);
     p.cpu = 1;
   } else {
     p.BM = bd::SIMT_BM;
     p.BN = bd::SIMT_BN;
     p.G = 2 * sm_count;
-    p.GM = 8;
     p.cpu = 1;
   }
+  // bands: as many m-tiles as keep their rows within the L2 budget (they are
+  // re-read for every v-tile while the head streams through once per band)
+  p.GM = env_int("BD_PLAN_GM", 0, 0, 1 << 20);
+  const int64_t budget = int64_t(env_int("BD_L2_ROWS_MB", 64, 1, 1 << 16)) << 20;
+  const int64_t rows = budget / std::max<int64_t>(1, row_operand_bytes(c));
+  p.rows_l2 = static_cast<int>(std::min<int64_t>(rows, int64_t(1) << 30));
   p.n_vt = static_cast<int>((c.V + p.BN - 1) / p.BN);
   return p;
 }
@@ -241,7 +267,9 @@ Layout make_layout(const Call& c, const BandPlan& p) {
   l.pm = take(4 * slots * P, 256);
   l.ps = take(4 * slots * P, 256);
   l.pa = take(4 * slots * P, 256);
-  l.hc = c.tc ? take(2 * static_cast<size_t>(c.ldc) * P, 1024) : 0;  // bf16 rows, or E4M3 rows (W8A8)
+  // bf16 rows, E4M3 rows (W8A8) or the two E4M3 terms of each row (W8A16 on the 8-bit path)
+  const size_t hc_row = std::max<size_t>(2 * static_cast<size_t>(c.ldc), 2 * static_cast<size_t>(round_up(c.d, 16)));
+  l.hc = c.tc ? take(hc_row * P, 1024) : 0;
   l.tsc = take(4 * P, 256);                                             // W8A8: per-row token scales
   l.wq = decoded_head(c) ? take(2 * static_cast<size_t>(c.ldq) * static_cast<size_t>(c.V), 1024) : 0;
   l.total = (off + 255) / 256 * 256;
@@ -319,7 +347,13 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
   bd::PairQuantMaps tmQ;
   std::memset(&tmB, 0, sizeof(tmB));
   std::memset(&tmQ, 0, sizeof(tmQ));
-  const int hf = c.fp8_act ? bd::HF_W8A8 : !c.fused ? bd::HF_BF16 : c.wdt == BD_NVFP4 ? bd::HF_NVFP4 : bd::HF_E4M3;
+  const int hf = c.fp8_act ? bd::HF_W8A8
+                 : c.split ? bd::HF_E4M3X2
+                 : !c.fused ? bd::HF_BF16
+                 : c.wdt == BD_NVFP4 ? bd::HF_NVFP4
+                                     : bd::HF_E4M3;
+  bd::PairTokenMaps tmLo;
+  std::memset(&tmLo, 0, sizeof(tmLo));
   if (c.fused) {
     // codes: 128 bytes of a row per box (128 NVFP4 / E4M3 ... columns of d: 256 / 128)
     const int64_t code_bytes = c.wdt == BD_NVFP4 ? (c.d + 1) / 2 : c.d;
@@ -335,10 +369,15 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
       const int rc = decode_head(c, weight, wq, sm_count, st, &wsrc, &wld);
       if (rc != BD_OK) return rc;
     }
-    if (c.pair && c.fp8_act) {
-      // W8A8: E4M3 token rows and head rows, 128-byte (128-column) boxes
-      for (int i = 0; i < 8; ++i)
+    if (c.pair && (c.fp8_act || c.split)) {
+      // W8A8 / two-term rows: E4M3 token rows and head rows, 128-byte
+      // (128-column) boxes; the lo terms follow the hi terms' P rows
+      for (int i = 0; i < 8; ++i) {
         if (!encode_u8_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 128, 16 * (i + 1), true)) return BD_ERR_CUDA;
+        if (c.split && !encode_u8_2d(&tmLo.m[i], static_cast<const uint8_t*>(rows) + c.P * ld_rows, c.d, c.P,
+                                     ld_rows, 128, 16 * (i + 1), true))
+          return BD_ERR_CUDA;
+      }
       if (!encode_u8_2d(&tmB, weight->data, c.d, c.V, c.ldw, 128, 128, true)) return BD_ERR_CUDA;
     } else if (c.pair) {
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
@@ -369,7 +408,8 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
     a.part_t = part.t;
     a.part_x = part.x;
     a.tok_scale = tok_scale;
-    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, c.fused ? &tmQ : nullptr, hf, a, st))
+    rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, c.fused ? &tmQ : nullptr, c.split ? &tmLo : nullptr,
+                                                     hf, a, st))
                 : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));
   } else {
     bd::SimtArgs a;
@@ -402,12 +442,22 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
   return BD_OK;
 }
 
+// Per-position partials of one vocabulary shard (bd_lmhead_partials).
+struct EmitTarget {
+  float* m;
+  float* s;
+  int32_t* a;
+  int offset;  // global id of the shard's first vocabulary entry
+};
+
 // The launch sequence of one commit step (a0..a4) on `st`, working in `ws`
-// laid out by `lay`; kernel timeouts are reported in `status`.
+// laid out by `lay`; kernel timeouts are reported in `status`. With `emit`,
+// the step ends after a3 with one merged partial per position (a head shard
+// of a vocabulary-parallel split) instead of the commit.
 int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws, uint32_t* status, int sm_count,
              const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
              const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
-             int32_t* out_counts, void* ev_begin, void* ev_end, cudaStream_t st) {
+             int32_t* out_counts, void* ev_begin, void* ev_end, cudaStream_t st, const EmitTarget* emit = nullptr) {
   int* n_rows = reinterpret_cast<int*>(ws + lay.hdr);
   int* idx = reinterpret_cast<int*>(ws + lay.idx);
   int* rowpos = reinterpret_cast<int*>(ws + lay.rowpos);
@@ -416,7 +466,7 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   int* pa = reinterpret_cast<int*>(ws + lay.pa);
   const int P = static_cast<int>(c.P), d = static_cast<int>(c.d);
 
-  if (out_counts) {
+  if (out_counts && !emit) {
     if (cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(c.n_seq) * c.T, st) != cudaSuccess)
       return BD_ERR_CUDA;
   }
@@ -424,12 +474,16 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   // a0: compaction of the masked positions of active blocks (+ packing of their rows)
   // W8A8: the packed rows are quantised to E4M3 with one scale per row; a
   // head decoded inside the LM head: f16 rows scaled by a power of two per row
-  const int row_format = c.fp8_act ? bd::ROWS_E4M3 : c.fused ? bd::ROWS_F16_POW2 : bd::ROWS_BF16;
+  const int row_format = c.fp8_act ? bd::ROWS_E4M3
+                         : c.split ? bd::ROWS_E4M3X2
+                         : c.fused ? bd::ROWS_F16_POW2
+                                   : bd::ROWS_BF16;
   float* tsc = row_format != bd::ROWS_BF16 ? reinterpret_cast<float*>(ws + lay.tsc) : nullptr;
-  const int64_t ld_rows = c.fp8_act ? ld_fp8_rows(c) : c.ldc;
+  const int64_t ld_rows = (c.fp8_act || c.split) ? ld_fp8_rows(c) : c.ldc;
   int rc = cuda_status(bd::launch_prep_rows(mask_state->pos_masked, mask_state->block_flags, P, c.L,
                                             c.tc ? hidden->data : nullptr, c.ldh, d, c.tc ? ws + lay.hc : nullptr,
-                                            ld_rows, idx, rowpos, n_rows, sm_count, st, tsc, row_format, status));
+                                            ld_rows, idx, rowpos, n_rows, sm_count, st, plan, tsc, row_format,
+                                            status));
   if (rc != BD_OK) return rc;
 
   rc = launch_lmhead(c, plan, hidden, weight, ws + lay.hc, ld_rows, ws + lay.wq, idx, n_rows, nullptr,
@@ -458,8 +512,19 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   ca.out_commit = out_commit;
   ca.out_counts = out_counts;
   ca.status = status;
+  if (emit) {
+    ca.emit_m = emit->m;
+    ca.emit_s = emit->s;
+    ca.emit_a = emit->a;
+    ca.vocab_offset = emit->offset;
+    ca.out_counts = nullptr;
+    return cuda_status(bd::launch_merge_commit(ca, st, bd::MERGE_EMIT));
+  }
   return cuda_status(bd::launch_merge_commit(ca, st));
 }
+// Drops the cached device addresses of the allocation-free entry point's
+// array (defined with it, below); the caller holds g_mu.
+void forget_static_devices();
 }  // namespace
 
 extern "C" {
@@ -509,6 +574,7 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd
     if (!aligned(weight->data, 16) || weight->ld % 16 != 0 || c.d < 16) return BD_ERR_ALIGN;
     c.fp8_act = true;
     c.fused = false;
+    c.split = false;
   }
   if (c.P == 0) return BD_OK;
   if (!out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
@@ -549,6 +615,111 @@ int bd_commit_step(const bd_hidden* hidden, const bd_weight* weight, const bd_ma
   return bd_commit_step_ex(hidden, weight, mask_state, tau_grid, out_tokens, out_conf, out_commit, nullptr);
 }
 
+int bd_lmhead_partials(const bd_hidden* hidden, const bd_weight* shard, int64_t vocab_offset,
+                       const bd_mask_state* mask_state, const bd_partials* out, const bd_exec* exec) {
+  bd::TraceRange trace("bd_lmhead_partials");
+  if (!hidden || !shard || !mask_state || !out) return BD_ERR_NULL;
+  if (vocab_offset < 0 || vocab_offset + shard->vocab > MAX_VOCAB) return BD_ERR_ARG;
+  if (mask_state->mask_token_id < -1) return BD_ERR_ARG;
+  if (exec && (exec->flags != 0 || exec->out_counts || exec->lmhead_event_begin || exec->lmhead_event_end))
+    return BD_ERR_ARG;
+  // the mask token, a global id, is suppressed by the shard that holds it
+  bd_mask_state local = *mask_state;
+  const int64_t mid = mask_state->mask_token_id;
+  local.mask_token_id = (mid >= vocab_offset && mid < vocab_offset + shard->vocab)
+                            ? static_cast<int32_t>(mid - vocab_offset) : -1;
+  const float tau1 = 0.5f;  // the shared checks want a grid; the shard step commits nothing
+  const bd_tau_grid tg{&tau1, 1};
+  Call c;
+  int rc = check_args(hidden, shard, &local, &tg, exec ? exec->variant : 0, &c);
+  if (rc != BD_OK) return rc;
+  if (c.P == 0) return BD_OK;
+  if (!out->m || !out->s || !out->a) return BD_ERR_NULL;
+  if (!aligned(out->m, 4) || !aligned(out->s, 4) || !aligned(out->a, 4)) return BD_ERR_ALIGN;
+  if (exec && exec->workspace && !aligned(exec->workspace, 256)) return BD_ERR_ALIGN;
+  DevCtx* ctx = nullptr;
+  rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs);
+  const Layout lay = make_layout(c, plan);
+  uint8_t* ws = nullptr;
+  if (exec && exec->workspace) {
+    if (exec->workspace_bytes < lay.total) return BD_ERR_WORKSPACE;
+    ws = static_cast<uint8_t*>(exec->workspace);
+  } else {
+    std::lock_guard<std::mutex> lk(g_mu);
+    if (ctx->ws_bytes < lay.total) {
+      if (ctx->ws) cudaFree(ctx->ws);  // synchronises the device: no call can still use it
+      ctx->ws = nullptr;
+      ctx->ws_bytes = 0;
+      if (cudaMalloc(&ctx->ws, lay.total) != cudaSuccess) return BD_ERR_CUDA;
+      ctx->ws_bytes = lay.total;
+    }
+    ws = static_cast<uint8_t*>(ctx->ws);
+  }
+  const EmitTarget emit{out->m, out->s, out->a, static_cast<int>(vocab_offset)};
+  cudaStream_t st = static_cast<cudaStream_t>(exec ? exec->stream : nullptr);
+  return run_step(c, plan, lay, ws, ctx->status, ctx->sm_count, hidden, shard, &local, &tg, nullptr, nullptr,
+                  nullptr, nullptr, nullptr, nullptr, st, &emit);
+}
+
+int bd_merge_commit(const bd_partials* gathered, int32_t n_parts, const bd_mask_state* mask_state,
+                    const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
+                    const bd_exec* exec) {
+  bd::TraceRange trace("bd_merge_commit");
+  if (!gathered || !mask_state || !tau_grid) return BD_ERR_NULL;
+  if (n_parts < 1 || n_parts > 4096) return BD_ERR_ARG;
+  if (!tau_grid->tau) return BD_ERR_TAU;
+  if (tau_grid->T < 1 || tau_grid->T > 32) return BD_ERR_TAU;
+  for (int k = 0; k < tau_grid->T; ++k)
+    if (std::isnan(tau_grid->tau[k])) return BD_ERR_TAU;
+  if (exec && (exec->flags != 0 || exec->workspace || exec->lmhead_event_begin || exec->lmhead_event_end))
+    return BD_ERR_ARG;
+  const bd_mask_state* ms = mask_state;
+  if (ms->n_seq < 0 || ms->n_slots < 1 || ms->block_len < 1 || ms->block_len > 64) return BD_ERR_SHAPE;
+  const int64_t n_blocks = int64_t(ms->n_seq) * ms->n_slots;
+  const int64_t P = n_blocks * ms->block_len;
+  if (P > MAX_POSITIONS || P * n_parts > (int64_t(1) << 31)) return BD_ERR_SHAPE;
+  if (P == 0) return BD_OK;
+  if (!ms->pos_masked || !ms->block_flags) return BD_ERR_NULL;
+  if (!gathered->m || !gathered->s || !gathered->a || !out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
+  if (!aligned(gathered->m, 4) || !aligned(gathered->s, 4) || !aligned(gathered->a, 4) || !aligned(out_tokens, 4) ||
+      !aligned(out_conf, 4) || !aligned(out_commit, 4))
+    return BD_ERR_ALIGN;
+  if (exec && exec->out_counts && !aligned(exec->out_counts, 4)) return BD_ERR_ALIGN;
+  DevCtx* ctx = nullptr;
+  const int rc = device_ctx(&ctx);
+  if (rc != BD_OK) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(exec ? exec->stream : nullptr);
+  int32_t* out_counts = exec ? exec->out_counts : nullptr;
+  if (out_counts &&
+      cudaMemsetAsync(out_counts, 0, sizeof(int32_t) * size_t(ms->n_seq) * tau_grid->T, st) != cudaSuccess)
+    return BD_ERR_CUDA;
+  bd::CommitArgs ca;
+  std::memset(&ca.plan, 0, sizeof(ca.plan));
+  ca.pos_masked = ms->pos_masked;
+  ca.block_flags = ms->block_flags;
+  ca.rowpos = nullptr;
+  ca.n_rows = nullptr;
+  ca.P = static_cast<int>(P);
+  ca.part_m = gathered->m;
+  ca.part_s = gathered->s;
+  ca.part_a = gathered->a;
+  ca.n_blocks = static_cast<int>(n_blocks);
+  ca.n_slots = ms->n_slots;
+  ca.block_len = ms->block_len;
+  std::memset(&ca.taus, 0, sizeof(ca.taus));
+  for (int k = 0; k < tau_grid->T; ++k) ca.taus.tau[k] = tau_grid->tau[k];
+  ca.taus.T = tau_grid->T;
+  ca.out_tokens = out_tokens;
+  ca.out_conf = out_conf;
+  ca.out_commit = out_commit;
+  ca.out_counts = out_counts;
+  ca.status = ctx->status;
+  ca.n_parts = n_parts;
+  return cuda_status(bd::launch_merge_commit(ca, st, bd::MERGE_GATHERED));
+}
+
 int bd_get_device_status(void* stream) {
   DevCtx* ctx = nullptr;
   int rc = device_ctx(&ctx);
@@ -587,6 +758,7 @@ int bd_shutdown(void) {
     c = DevCtx();
   }
   cudaSetDevice(cur);
+  forget_static_devices();
   return rc;
 }
 
@@ -612,6 +784,12 @@ struct StaticCtx {
   uint8_t* scratch = nullptr;  // device address of g_static_scratch on this device
 };
 StaticCtx g_static[MAX_DEVICES];
+
+// After bd_shutdown (and possibly a device reset) the module may be loaded
+// again at another address: the next call resolves it anew.
+void forget_static_devices() {
+  for (int dev = 0; dev < MAX_DEVICES; ++dev) g_static[dev] = StaticCtx();
+}
 
 // Once per device, with that device current: checks the device, fetches the
 // tensor-map encoder and resolves the device address of g_static_scratch.
@@ -645,6 +823,8 @@ int static_ctx(StaticCtx** out) {
     const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
     if (e != cudaSuccess || p == nullptr) return e == cudaSuccess ? BD_ERR_CUDA : cuda_status(e);
     s.scratch = static_cast<uint8_t*>(p);
+    // the status word starts clear; afterwards only bd_static_device_status clears it
+    if (cudaMemset(s.scratch + STATIC_STATUS_OFFSET, 0, sizeof(uint32_t)) != cudaSuccess) return BD_ERR_CUDA;
     s.sm_count = sms;
     s.pairs = pairs;
     s.ready = true;
@@ -675,12 +855,41 @@ extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* w
 
   uint8_t* ws = sctx->scratch;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // The array keeps the previous call's contents: everything the step reads
+  // it writes first, except the status word, which is cleared once at set-up
+  // and then by bd_static_device_status (a failure stays recorded until read).
   uint32_t* status = reinterpret_cast<uint32_t*>(ws + lay.hdr + STATIC_STATUS_OFFSET);
-  // The array keeps the previous call's contents; only the timeout word must
-  // start at zero (everything else is written before it is read).
-  if (cudaMemsetAsync(status, 0, sizeof(uint32_t), st) != cudaSuccess) return BD_ERR_CUDA;
   return run_step(c, plan, lay, ws, status, sctx->sm_count, hidden, weight, mask_state, tau_grid, out_tokens,
                   out_conf, out_commit, nullptr, nullptr, nullptr, st);
+}
+
+namespace {
+int static_status_of(uint32_t word) {
+  if (word & bd::DEV_TIMEOUT) return BD_ERR_TIMEOUT;
+  if (word & bd::DEV_BAD_LAUNCH) return BD_ERR_CUDA;
+  if (word & bd::DEV_BOUNDS) return BD_ERR_BOUNDS;
+  return BD_OK;
+}
+}  // namespace
+
+extern "C" int bd_static_device_status(void* stream) {
+  StaticCtx* sctx = nullptr;
+  const int rc = static_ctx(&sctx);
+  if (rc != BD_OK) return rc;
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return BD_ERR_CUDA;
+  uint32_t word = 0;
+  uint8_t* at = sctx->scratch + STATIC_STATUS_OFFSET;
+  if (cudaMemcpy(&word, at, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess) return BD_ERR_CUDA;
+  if (word != 0 && cudaMemset(at, 0, sizeof(word)) != cudaSuccess) return BD_ERR_CUDA;
+  return static_status_of(word);
+}
+
+extern "C" int bd_static_selftest_timeout(void* stream) {
+  StaticCtx* sctx = nullptr;
+  const int rc = static_ctx(&sctx);
+  if (rc != BD_OK) return rc;
+  return cuda_status(bd::launch_timeout_selftest(reinterpret_cast<uint32_t*>(sctx->scratch + STATIC_STATUS_OFFSET),
+                                                 static_cast<cudaStream_t>(stream)));
 }
 
 // ---------------------------------------------------------------------------
@@ -765,7 +974,7 @@ int run_verify(const VerifyCall& vc, const BandPlan& plan, const VerifyLayout& l
   float* px = reinterpret_cast<float*>(ws + lay.px);
   const int R = static_cast<int>(c.P);
 
-  int rc = cuda_status(bd::launch_prep_verify(draft->draft, vc.n_req, vc.n_draft, idx, draft_row, n_rows, st));
+  int rc = cuda_status(bd::launch_prep_verify(draft->draft, vc.n_req, vc.n_draft, idx, draft_row, n_rows, plan, st));
   if (rc != BD_OK) return rc;
 
   rc = launch_lmhead(c, plan, hidden, weight, hidden->data, c.ldh, ws + lay.wq, idx, n_rows, draft_row,

@@ -33,31 +33,32 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // -------------------------------------------------------------------------
 // Work plan of the LM-head kernels.
 //
-// The N compacted rows are cut into m-tiles of BM rows and the vocabulary
-// into v-tiles of BN entries. m-tiles are taken in bands of at most GM; in a
-// band of gm m-tiles the vocabulary is split into gv = min(G / gm, n_vt)
-// contiguous parts, and CTA c (c < gm * gv) takes m-tile m0 + c % gm over
-// part c / gm. CTAs of one part walk the same v-tiles at the same time, so a
-// weight tile is fetched from HBM about once per band and re-read from L2 by
-// the gm CTAs that share it. Each (row, part) leaves one partial
-// (max, sum of exponentials, argmax) in slot `part` of the partial arrays;
-// the merge kernel combines the gv slots of a row. N is only known on the
-// device, so kernels recompute the plan from it.
+// The N compacted rows are cut into m-tiles of BM rows (token groups of the
+// pair kernel) and the vocabulary into v-tiles of BN entries, split into gv
+// contiguous parts of (nearly) equal length. A unit of work is one (m-tile,
+// part): a runner (a CTA, or a CTA pair) walks the part's v-tiles with the
+// m-tile's rows and leaves one partial (max, sum of exponentials, argmax) per
+// row in slot `part` (times the CTAs per unit) of the partial arrays.
+//
+// Units are numbered band by band: a band holds at most GM consecutive
+// m-tiles, sized so that its rows stay resident in L2, and inside a band the
+// units go part by part (all m-tiles of part 0, then part 1, ...). Runner c
+// takes units c, c + G, c + 2G, ...: the G units in flight at any time are
+// consecutive, i.e. a few parts of one band, so every head tile is fetched
+// from HBM about once per band and re-read from L2 by the m-tiles that share
+// it while the band's rows stay in L2. gv minimises the makespan
+// ceil(units / G) * (ceil(n_vt / gv) + 1/2) (half a v-tile for each unit's
+// start and finish). N is only known on the device, so kernels recompute the
+// plan from it.
 // -------------------------------------------------------------------------
 struct BandPlan {
-  int BM;    // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
-  int BN;    // vocabulary entries per v-tile
-  int GM;    // m-tiles per band (at most)
-  int G;     // units that can run at once (CTAs, or CTA pairs)
-  int n_vt;  // ceil(V / BN)
-  int cpu;   // CTAs per unit: each writes its own partial, so a part has cpu slots
-};
-
-struct Band {
-  int m0;     // first m-tile of the band
-  int gm;     // m-tiles in the band
-  int gv;     // vocabulary parts per m-tile
-  int units;  // gm * gv units busy in this band
+  int BM;       // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
+  int BN;       // vocabulary entries per v-tile
+  int GM;       // m-tiles per band at most; 0 = derived from rows_l2
+  int rows_l2;  // rows a band may hold (GM = 0): the L2 budget over the packed row bytes
+  int G;        // units that can run at once (CTAs, or CTA pairs)
+  int n_vt;     // ceil(V / BN)
+  int cpu;      // CTAs per unit: each writes its own partial, so a part has cpu slots
 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
@@ -74,59 +75,99 @@ __host__ __device__ __forceinline__ int plan_bm(const BandPlan& p, int n_rows) {
   return p.BM > 0 ? p.BM : pair_group_rows(n_rows);
 }
 
-__host__ __device__ __forceinline__ Band band_of(const BandPlan& p, int n_mt, int b) {
-  Band r;
-  r.m0 = b * p.GM;
-  r.gm = n_mt - r.m0 < p.GM ? n_mt - r.m0 : p.GM;
-  int gv = p.G / r.gm;
-  r.gv = gv < p.n_vt ? gv : p.n_vt;
-  if (r.gv < 1) r.gv = 1;
-  r.units = r.gm * r.gv;
-  return r;
+// m-tiles per band (all bands but the last are full)
+__host__ __device__ __forceinline__ int plan_gm(const BandPlan& p, int bm) {
+  if (p.GM > 0) return p.GM;
+  const int g = p.rows_l2 / bm;
+  return g < 1 ? 1 : g;
 }
 
-// Number of partial slots of compacted row `row`.
-__host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int row) {
-  const int bm = plan_bm(p, n_rows);
-  const int n_mt = cdiv(n_rows, bm);
-  const int b = (row / bm) / p.GM;
-  return band_of(p, n_mt, b).gv * p.cpu;
+// The makespan of gv parts, in half v-tiles, packed with gv into one key:
+// the smallest key is the smallest makespan, then the fewest parts.
+__host__ __device__ __forceinline__ uint64_t plan_gv_key(const BandPlan& p, int n_mt, int gv) {
+  const uint64_t rounds = (static_cast<uint64_t>(n_mt) * gv + p.G - 1) / p.G;
+  const uint64_t cost = rounds * (2 * static_cast<uint64_t>(cdiv(p.n_vt, gv)) + 1);
+  return (cost << 10) | static_cast<uint64_t>(gv);  // gv <= G < 2^10
 }
 
-// Iterates the (m-tile, v-tile) sequence of unit-runner `unit` (a CTA, or a
-// CTA pair) under the band plan.
+// vocabulary parts per m-tile: the makespan rule above, over 1..min(G, n_vt)
+__host__ __device__ __forceinline__ int plan_gv(const BandPlan& p, int n_mt) {
+  const int hi = p.G < p.n_vt ? p.G : p.n_vt;
+  uint64_t best = ~uint64_t(0);
+  for (int gv = 1; gv <= hi; ++gv) {
+    const uint64_t k = plan_gv_key(p, n_mt, gv);
+    best = k < best ? k : best;
+  }
+  return static_cast<int>(best & 1023u);
+}
+
+#ifdef __CUDACC__
+// The same choice by a whole warp, 32 candidates at a time. The kernel that
+// learns N (compaction, or the verification rows) evaluates it once and
+// stores gv beside N in the workspace header (plan_hdr[0] = N, plan_hdr[1] =
+// gv), so the LM-head and merge kernels only read it.
+__device__ __forceinline__ int plan_gv_warp(const BandPlan& p, int n_mt) {
+  const int hi = p.G < p.n_vt ? p.G : p.n_vt;
+  uint64_t best = ~uint64_t(0);
+  for (int gv = static_cast<int>(threadIdx.x & 31) + 1; gv <= hi; gv += 32) {
+    const uint64_t k = plan_gv_key(p, n_mt, gv);
+    best = k < best ? k : best;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t other = __shfl_xor_sync(0xffffffffu, best, o);
+    best = other < best ? other : best;
+  }
+  return static_cast<int>(best & 1023u);
+}
+#endif
+
+// Number of partial slots of every compacted row.
+__host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int /*row*/) {
+  const int n_mt = cdiv(n_rows, plan_bm(p, n_rows));
+  return plan_gv(p, n_mt) * p.cpu;
+}
+
+// Iterates the (m-tile, v-tile range) units of unit-runner `runner` (a CTA,
+// or a CTA pair) under the plan.
 struct TileIter {
-  BandPlan p;
-  int unit;
-  int bm, n_mt, n_bands;
-  int b;       // current band
+  int runner, G;
+  int n_mt, gm_full, gv, n_vt;
+  int64_t u, n_units;
   int m_tile;  // current m-tile
   int part;    // vocabulary part of the current unit
   int vt, vt_end;
 
-  __device__ void init(const BandPlan& plan, int n_rows, int unit_index) {
-    p = plan;
-    unit = unit_index;
-    bm = plan_bm(p, n_rows);
-    n_mt = cdiv(n_rows, bm);
-    n_bands = cdiv(n_mt, p.GM);
-    b = -1;
+  // n_rows and parts: the header the compaction kernel wrote (N, gv)
+  __host__ __device__ void init(const BandPlan& plan, int n_rows, int parts, int runner_index) {
+    runner = runner_index;
+    G = plan.G;
+    n_vt = plan.n_vt;
+    const int bm = plan_bm(plan, n_rows);
+    n_mt = n_rows > 0 ? cdiv(n_rows, bm) : 0;
+    gm_full = plan_gm(plan, bm);
+    gv = parts;
+    n_units = static_cast<int64_t>(n_mt) * gv;
+    u = static_cast<int64_t>(runner) - G;
     vt = vt_end = 0;
   }
-  __device__ void init(const BandPlan& plan, int n_rows) { init(plan, n_rows, blockIdx.x); }
+#ifdef __CUDACC__
+  __device__ void init(const BandPlan& plan, int n_rows, int parts) { init(plan, n_rows, parts, blockIdx.x); }
+#endif
   // Advances to the next unit; false when there is no more work.
-  __device__ bool next_unit() {
-    for (++b; b < n_bands; ++b) {
-      Band bd = band_of(p, n_mt, b);
-      const int c = unit;
-      if (c >= bd.units) continue;
-      m_tile = bd.m0 + c % bd.gm;
-      part = c / bd.gm;
-      vt = static_cast<int>(static_cast<int64_t>(part) * p.n_vt / bd.gv);
-      vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * p.n_vt / bd.gv);
-      return true;
-    }
-    return false;
+  __host__ __device__ bool next_unit() {
+    u += G;
+    if (u >= n_units) return false;
+    const int64_t band_units = static_cast<int64_t>(gm_full) * gv;
+    const int b = static_cast<int>(u / band_units);
+    const int i = static_cast<int>(u - b * band_units);
+    const int m0 = b * gm_full;
+    const int gm = n_mt - m0 < gm_full ? n_mt - m0 : gm_full;
+    part = i / gm;
+    m_tile = m0 + i % gm;
+    vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
+    vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
+    return true;
   }
 };
 

@@ -9,6 +9,12 @@
 //                     no position cleared tau_k, and p is the masked position of
 //                     highest confidence (lowest position on ties)         (App. B.2)
 // with one warp ballot per tau (two for blocks longer than 32).
+//
+// Vocabulary-parallel split (one head shard per rank): MERGE_EMIT merges the
+// slots of each position of this shard's LM head into one partial per window
+// position (global token ids: the shard's offset added) instead of
+// committing; MERGE_GATHERED merges the n_parts such per-position partials
+// gathered from every shard ([n_parts, P] arrays) and commits.
 #include "checks.h"
 #include "kernels.h"
 
@@ -20,15 +26,18 @@ constexpr int MAX_L = 64;
 constexpr int MAX_GROUPS = THREADS / 32;
 }  // namespace
 
+template <int MODE>
 __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
   __shared__ float sm_m[MAX_GROUPS][MAX_L], sm_s[MAX_GROUPS][MAX_L];
   __shared__ int sm_a[MAX_GROUPS][MAX_L];
+  __shared__ bool sm_live[MAX_L];  // the position has a compacted row (read once, in the merge stage)
   const int blk = blockIdx.x;
   const int L = a.block_len;
   const int64_t base = static_cast<int64_t>(blk) * L;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   griddep_wait();  // the partials come from the LM-head kernel
-  const int n_rows = *a.n_rows;
+  // partial slots per row: the plan's parts (header word 1) times the CTAs per unit
+  const int slots = MODE == MERGE_GATHERED ? a.n_parts : a.n_rows[1] * a.plan.cpu;
 
   // ---- a3: merge of the partial slots. Thread t takes position t % Lp of the
   // block and every groups-th slot starting at t / Lp; loads are issued four
@@ -41,10 +50,18 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
     float m = -INFINITY, s = 0.f;
     int arg = 0x7fffffff;
     // partial slots the workspace holds (index checks of the bounds-checked build)
-    const int64_t part_n = static_cast<int64_t>(a.plan.cpu) * (a.plan.G < a.plan.n_vt ? a.plan.G : a.plan.n_vt) * a.P;
-    const int r = jj < L && index_ok(base + jj, a.P, a.status) ? a.rowpos[base + jj] : -1;
+    const int64_t part_n = MODE == MERGE_GATHERED
+                               ? static_cast<int64_t>(a.n_parts) * a.P
+                               : static_cast<int64_t>(a.plan.cpu) * (a.plan.G < a.plan.n_vt ? a.plan.G : a.plan.n_vt) * a.P;
+    int r = -1;  // the slot index of this position: its compacted row, or (gathered) the position itself
+    if (jj < L && index_ok(base + jj, a.P, a.status)) {
+      if constexpr (MODE == MERGE_GATHERED)
+        r = (a.pos_masked[base + jj] != 0 && (a.block_flags[blk] & 1u)) ? static_cast<int>(base + jj) : -1;
+      else
+        r = a.rowpos[base + jj];
+    }
     if (r >= 0 && index_ok(r, a.P, a.status)) {
-      const int ns = slots_of_row(a.plan, n_rows, r);
+      const int ns = slots;
       int slot = g;
       for (; slot + 3 * groups < ns; slot += 4 * groups) {
         float pm[4], ps[4];
@@ -69,10 +86,34 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
       sm_m[g][jj] = m;
       sm_s[g][jj] = s;
       sm_a[g][jj] = arg;
+      if (g == 0) sm_live[jj] = r >= 0;
     }
   }
   __syncthreads();
   if (warp != 0) return;
+
+  if constexpr (MODE == MERGE_EMIT) {
+    // one partial per window position, token ids of the whole vocabulary
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int jj = lane + 32 * h;
+      if (jj < L) {
+        float m = -INFINITY, s = 0.f;
+        int arg = -1;
+        if (sm_live[jj]) {
+          m = sm_m[0][jj];
+          s = sm_s[0][jj];
+          arg = sm_a[0][jj];
+          for (int g = 1; g < groups; ++g) softmax_combine(m, s, arg, sm_m[g][jj], sm_s[g][jj], sm_a[g][jj]);
+          arg = m == -INFINITY ? -1 : arg + a.vocab_offset;  // a shard holding only the mask token: nothing
+        }
+        a.emit_m[base + jj] = m;
+        a.emit_s[base + jj] = s;
+        a.emit_a[base + jj] = arg;
+      }
+    }
+    return;
+  }
 
   const uint32_t flags = a.block_flags[blk];
   const bool eligible = (flags & 2u) != 0;
@@ -82,7 +123,7 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
 #pragma unroll
   for (int h = 0; h < 2; ++h) {
     const int jj = lane + 32 * h;
-    live[h] = jj < L && a.rowpos[base + jj] >= 0;
+    live[h] = jj < L && sm_live[jj];
     conf[h] = 0.f;
     tok[h] = -1;
     if (live[h]) {
@@ -153,7 +194,7 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
   }
 }
 
-cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st) {
+cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st, int mode) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(a.n_blocks, 1, 1);
   cfg.blockDim = dim3(THREADS, 1, 1);
@@ -163,7 +204,14 @@ cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st) {
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, merge_commit_kernel, a);
+  switch (mode) {
+    case MERGE_EMIT:
+      return cudaLaunchKernelEx(&cfg, merge_commit_kernel<MERGE_EMIT>, a);
+    case MERGE_GATHERED:
+      return cudaLaunchKernelEx(&cfg, merge_commit_kernel<MERGE_GATHERED>, a);
+    default:
+      return cudaLaunchKernelEx(&cfg, merge_commit_kernel<MERGE_ROWS>, a);
+  }
 }
 
 }  // namespace bd

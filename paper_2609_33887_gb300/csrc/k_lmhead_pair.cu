@@ -42,6 +42,15 @@
 // quarter, alternate 32-column chunks; 320 threads). Each token's scale
 // multiplies its logits through the exponent's factor.
 //
+// W8A16 on the 8-bit path (HF = HF_E4M3X2): an E4M3 head times bf16 token
+// rows, each row packed by the compaction kernel as two E4M3 terms hi + lo of
+// the row scaled by a power of two (exact for every element of at least 2^-10
+// of the row's largest). Per 128-column stage the head atom is staged once
+// and multiplied into the same accumulator by the hi and the lo token atoms:
+// eight K = 32 kind::f8f6f4 MMAs, the tensor time of the bf16 head's stage,
+// at half its head bytes and with no decode of the head at all. The E4M3 x
+// E4M3 products are exact in fp32.
+//
 // Heads decoded in the kernel (HF = HF_E4M3, HF_NVFP4: the precision levers):
 // HBM carries the stored head only. A raw-code producer warp streams this
 // CTA's head codes (and NVFP4 block scales) with TMA into a raw ring, and
@@ -75,6 +84,16 @@ template <int HF>
 __host__ __device__ constexpr bool pair_cluster() {
   return !is_quant<HF>();
 }
+// E4M3 head codes read by TMA straight into the MMA operand (8-bit atoms)
+template <int HF>
+__host__ __device__ constexpr bool is_8bit() {
+  return HF == HF_W8A8 || HF == HF_E4M3X2;
+}
+// token-operand terms per stage: hi and lo for the two-term rows, else one
+template <int HF>
+__host__ __device__ constexpr int b_terms() {
+  return HF == HF_E4M3X2 ? 2 : 1;
+}
 // columns of d per operand stage: two 64-column 16-bit swizzle atoms for bf16
 // heads; one 128-column 8-bit atom for W8A8; one 16-bit atom for heads decoded
 // in the kernel, whose small stages leave room for a deep raw ring
@@ -85,7 +104,7 @@ __host__ __device__ constexpr int stage_k() {
 // columns of one 128-byte swizzle atom
 template <int HF>
 __host__ __device__ constexpr int atom_cols() {
-  return HF == HF_W8A8 ? 128 : 64;
+  return is_8bit<HF>() ? 128 : 64;
 }
 constexpr int MAX_STAGES = 8;
 constexpr uint32_t ATOM_ROWS_BYTES = 128;  // one row of a swizzle atom (64 16-bit or 128 8-bit columns)
@@ -179,7 +198,8 @@ template <int HF>
 __host__ __device__ constexpr uint32_t stage_bytes(int nt) {
   // heads decoded in the kernel: one CTA multiplies its 128 head rows by all NT token rows
   return is_quant<HF>() ? A_BLOCK + static_cast<uint32_t>(nt) * ATOM_ROWS_BYTES
-                        : (stage_k<HF>() / atom_cols<HF>()) * (A_BLOCK + static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES);
+                        : (stage_k<HF>() / atom_cols<HF>()) *
+                              (A_BLOCK + b_terms<HF>() * static_cast<uint32_t>(nt / 2) * ATOM_ROWS_BYTES);
 }
 // Operand stages: as many as fit (at most MAX_STAGES) for bf16 heads; for
 // quantised heads at most QUANT_STAGES next to a raw ring of at least three
@@ -207,6 +227,8 @@ static_assert(stage_count<HF_BF16, false>(256) >= 3 && stage_count<HF_BF16, true
 static_assert(stage_count<HF_BF16, false>(160) == 4, "four stages at NT = 160 on the commit path");
 static_assert(stage_count<HF_W8A8, false>(160) == 7 && stage_count<HF_W8A8, false>(256) >= 5,
               "W8A8: seven 26 KB stages at NT = 160, five 32 KB stages at NT = 256");
+static_assert(stage_count<HF_E4M3X2, false>(160) == 5 && stage_count<HF_E4M3X2, false>(256) == 4,
+              "two-term rows: five 36 KB stages at NT = 160, four 48 KB stages at NT = 256");
 static_assert(stage_count<HF_NVFP4, false>(160) == 4 && stage_count<HF_E4M3, false>(160) == 4 &&
                   stage_count<HF_NVFP4, true>(160) == 4 && stage_count<HF_E4M3, true>(160) == 4,
               "four operand stages at NT = 160 for quantised heads");
@@ -288,15 +310,17 @@ __device__ __forceinline__ void convert_stage(uint32_t raw_base, int h, uint32_t
 template <int HF, bool VERIFY>
 __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     lmhead_pair_kernel(const __grid_constant__ PairTokenMaps tmH, const __grid_constant__ CUtensorMap tmW,
-                       const __grid_constant__ PairQuantMaps tmQ, TcArgs a) {
+                       const __grid_constant__ PairQuantMaps tmQ, const __grid_constant__ PairTokenMaps tmL,
+                       TcArgs a) {
   constexpr bool QUANT = is_quant<HF>();
   constexpr bool W8A8 = HF == HF_W8A8;
-  static_assert(!(W8A8 && VERIFY), "the W8A8 variant serves the commit step");
+  constexpr bool X2 = HF == HF_E4M3X2;
+  static_assert(!((W8A8 || X2) && VERIFY), "the 8-bit instantiations serve the commit step");
   // commit step with a head decoded in the kernel: f16 operands (the decode
   // ends at f16), token rows pre-scaled by a power of two per row
   constexpr bool F16OPS = QUANT && !VERIFY;
   // the packed rows carry a per-row scale that multiplies their logits
-  constexpr bool TOKS = W8A8 || F16OPS;
+  constexpr bool TOKS = W8A8 || X2 || F16OPS;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   constexpr int EW = epi_warps<HF>();
@@ -363,7 +387,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   volatile int* abort_flag = &ctl->abort_flag;
 
   griddep_wait();  // the packed rows and N come from the preceding kernel
-  const int n_rows = *a.n_rows;
+  const int n_rows = a.n_rows[0];
+  const int parts = a.n_rows[1];  // vocabulary parts of the plan (see common.cuh)
   constexpr int BK = stage_k<HF>();
   constexpr int ACOLS = atom_cols<HF>();
   constexpr int NATOM = BK / ACOLS;
@@ -384,6 +409,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   const uint32_t tx_total = QUANT ? static_cast<uint32_t>(NT) * ATOM_ROWS_BYTES : 2u * SB;
   const uint32_t raw_base = smem_base + static_cast<uint32_t>(STAGES) * SB;  // quantised heads' raw ring
   const CUtensorMap* tm_tok = &tmH.m[half / 16 - 1];  // box of exactly `half` rows
+  const CUtensorMap* tm_lo = &tmL.m[half / 16 - 1];   // two-term rows: the lo terms
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer
@@ -395,7 +421,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, pair);
+    it.init(a.plan, n_rows, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       const int tok0 = it.m_tile * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
@@ -422,6 +448,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
                 tma_load_2d_pair(sa + j * A_BLOCK, &tmW, fb, kb * BK + ACOLS * j, vrow, pol_w);
                 tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + ACOLS * j, tok0, pol_h);
               }
+              if constexpr (X2) tma_load_2d_pair(sa + A_BLOCK + B_BLOCK, tm_lo, fb, kb * BK, tok0, pol_h);
             }
           }
           __syncwarp();
@@ -444,13 +471,13 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     // ------------------------------------------------------ MMA issuer (even CTA; every CTA for quantised heads)
     if (rank == 0 || QUANT) {
       const bool leader = elect_one();
-      const uint32_t idesc = W8A8     ? idesc_e4m3_f32(256, NT)
+      const uint32_t idesc = (W8A8 || X2) ? idesc_e4m3_f32(256, NT)
                              : F16OPS ? idesc_f16_f32(128, NT)
                                       : idesc_bf16_f32(QUANT ? 128 : 256, NT);
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
-      it.init(a.plan, n_rows, pair);
+      it.init(a.plan, n_rows, parts, pair);
       bool ok = true;
       while (ok && it.next_unit()) {
         for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -475,12 +502,18 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
 #pragma unroll
                 for (int k = 0; k < 4; ++k) {
                   // +32 bytes along K per MMA (16 bf16 / 32 E4M3 columns) = +2 in the address field
-                  if constexpr (QUANT)
+                  if constexpr (QUANT) {
                     umma_bf16(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
-                  else if constexpr (W8A8)
+                  } else if constexpr (X2) {
+                    // the head atom times the hi terms, then times the lo terms
+                    const uint64_t ldesc = sw128_kmajor_desc(sa + A_BLOCK + B_BLOCK);
+                    umma_f8_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | k) != 0);
+                    umma_f8_pair(d_tmem, adesc + 2u * k, ldesc + 2u * k, idesc, true);
+                  } else if constexpr (W8A8) {
                     umma_f8_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
-                  else
+                  } else {
                     umma_bf16_pair(d_tmem, adesc + 2u * k, bdesc + 2u * k, idesc, (kb | j | k) != 0);
+                  }
                 }
               }
               if constexpr (QUANT)
@@ -526,7 +559,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t r = 0, rph = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, pair);
+    it.init(a.plan, n_rows, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -564,7 +597,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     constexpr int RK = raw_k<HF>();
     uint32_t r = 0, rph = 0, stage = 0, phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, pair);
+    it.init(a.plan, n_rows, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -610,7 +643,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t epi_phase = 0;
     uint32_t acc = 0, acc_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, pair);
+    it.init(a.plan, n_rows, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       float m[MAX_CHUNKS], s[MAX_CHUNKS];
@@ -883,32 +916,43 @@ cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs) {
 
 template <int HF, bool VERIFY>
 static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps& tmQ,
-                               const TcArgs& a, cudaStream_t st) {
+                               const PairTokenMaps& tmL, const TcArgs& a, cudaStream_t st) {
   cudaError_t e = pair_opt_in<HF, VERIFY>();
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
   pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, pair_cluster<HF>());
-  return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, a);
+  return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, a);
 }
 
-cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ, int hf,
-                               const TcArgs& a, cudaStream_t st) {
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ,
+                               const PairTokenMaps* tmLo, int hf, const TcArgs& a, cudaStream_t st) {
   const bool verify = a.part_t != nullptr;
   PairQuantMaps none;
   std::memset(&none, 0, sizeof(none));
   const PairQuantMaps& q = tmQ ? *tmQ : none;
+  static const PairTokenMaps no_lo = [] {
+    PairTokenMaps m;
+    std::memset(&m, 0, sizeof(m));
+    return m;
+  }();
+  const PairTokenMaps& lo = tmLo ? *tmLo : no_lo;
   switch (hf) {
     case HF_W8A8:
       if (verify) return cudaErrorInvalidValue;
-      return launch_pair<HF_W8A8, false>(tmH, tmW, q, a, st);
+      return launch_pair<HF_W8A8, false>(tmH, tmW, q, lo, a, st);
+    case HF_E4M3X2:
+      if (verify || tmLo == nullptr) return cudaErrorInvalidValue;
+      return launch_pair<HF_E4M3X2, false>(tmH, tmW, q, lo, a, st);
     case HF_E4M3:
-      return verify ? launch_pair<HF_E4M3, true>(tmH, tmW, q, a, st) : launch_pair<HF_E4M3, false>(tmH, tmW, q, a, st);
+      return verify ? launch_pair<HF_E4M3, true>(tmH, tmW, q, lo, a, st)
+                    : launch_pair<HF_E4M3, false>(tmH, tmW, q, lo, a, st);
     case HF_NVFP4:
-      return verify ? launch_pair<HF_NVFP4, true>(tmH, tmW, q, a, st)
-                    : launch_pair<HF_NVFP4, false>(tmH, tmW, q, a, st);
+      return verify ? launch_pair<HF_NVFP4, true>(tmH, tmW, q, lo, a, st)
+                    : launch_pair<HF_NVFP4, false>(tmH, tmW, q, lo, a, st);
     default:
-      return verify ? launch_pair<HF_BF16, true>(tmH, tmW, q, a, st) : launch_pair<HF_BF16, false>(tmH, tmW, q, a, st);
+      return verify ? launch_pair<HF_BF16, true>(tmH, tmW, q, lo, a, st)
+                    : launch_pair<HF_BF16, false>(tmH, tmW, q, lo, a, st);
   }
 }
 

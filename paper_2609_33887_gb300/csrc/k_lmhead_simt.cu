@@ -66,10 +66,11 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   __shared__ SimtSmem sm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   griddep_wait();  // idx and N come from the preceding kernel
-  const int n_rows = *a.n_rows;
+  const int n_rows = a.n_rows[0];
+  const int parts = a.n_rows[1];  // vocabulary parts of the plan (see common.cuh)
 
   TileIter it;
-  it.init(a.plan, n_rows);
+  it.init(a.plan, n_rows, parts);
   while (it.next_unit()) {
     const int r0 = it.m_tile * SIMT_BM;
     if (tid < SIMT_BM) {

@@ -44,12 +44,17 @@ __device__ __forceinline__ uint32_t f32x2_to_e4m3x2(float lo, float hi) {
   return r;
 }
 
+// f16x2 bit pattern -> two float32 values (exact).
+__device__ __forceinline__ float2 f16x2_bits_to_float2(uint32_t h2) {
+  return __half22float2(*reinterpret_cast<const __half2*>(&h2));
+}
+
 template <int FMT>  // the packed row format (ROWS_*); one instantiation per format
 __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     const uint8_t* __restrict__ pos_masked, const uint8_t* __restrict__ block_flags, int P, int block_len, int chunk,
     const __nv_bfloat16* __restrict__ hidden, int64_t ld, int d, __nv_bfloat16* __restrict__ hc, int64_t ldc,
     int* __restrict__ idx, int* __restrict__ rowpos, int* __restrict__ n_rows, float* __restrict__ tok_scale,
-    uint32_t* __restrict__ status) {
+    uint32_t* __restrict__ status, BandPlan plan) {
   __shared__ int red[PREP_THREADS / 32];
   __shared__ int warp_excl[PREP_THREADS / 32];
   __shared__ int rows_s[2048];
@@ -104,7 +109,17 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       }
     }
   }
-  if (p1 == P && tid == 0) *n_rows = prefix + local_total;
+  if (p1 == P && warp == 0) {
+    // the CTA holding the last position knows N: it writes N and the plan's
+    // vocabulary parts for it into the header the later kernels read
+    const int N = prefix + local_total;
+    const int n_mt = N > 0 ? cdiv(N, plan_bm(plan, N)) : 1;
+    const int gv = plan_gv_warp(plan, n_mt);
+    if (lane == 0) {
+      n_rows[0] = N;
+      n_rows[1] = gv;
+    }
+  }
   if (hidden == nullptr) return;
   __syncthreads();
 
@@ -153,6 +168,77 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
         d4[v] = make_uint4(o[0], o[1], o[2], o[3]);
       }
       for (int e = nvec * 8 + lane; e < d; e += 32) dst[e] = __float2half_rn(__bfloat162float(src[e]) * up);
+      if (lane == 0) tok_scale[prefix + i] = amax > 0.f ? __uint_as_float(static_cast<uint32_t>(127 - sh) << 23) : 0.f;
+    }
+    return;
+  }
+  if constexpr (FMT == ROWS_E4M3X2) {
+    // 3'''. bf16 rows as two E4M3 terms for an E4M3 head on the 8-bit tensor
+    // path (W8A16): row r is scaled by 2^s so that its largest magnitude lands
+    // in [128, 256) (s = 134 - E for the biased exponent E of max |h|, between
+    // -126 and 126 so 2^s and 2^-s stay normal floats; exact), then
+    // y = h * 2^s becomes hi = e4m3(y) and lo = e4m3(y - hi), both rounded to
+    // nearest even. y has at most 8 significant bits and y - hi (exact in
+    // float32) at most 4 more, so hi + lo == y exactly whenever |y| >= 2^-2,
+    // i.e. for every element of at least 2^-10 times the row's largest; a
+    // smaller element is off by at most 2^-10 (half the smallest E4M3 step),
+    // 2^-17 of the row's largest. hi rows at hc, lo rows at hc + P * ldc (ldc
+    // in bytes); tok_scale = 2^-s (0 for an all-zero row).
+    uint8_t* hq = reinterpret_cast<uint8_t*>(hc);
+    uint8_t* lq = hq + static_cast<int64_t>(P) * ldc;
+    for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+      if (!index_ok(prefix + i, P, status)) continue;
+      const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
+      const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
+      const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      float amax = 0.f;
+      for (int v = lane; v < nvec; v += 32) {
+        const uint4 q = __ldg(s4 + v);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[j]));
+          amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+        }
+      }
+      for (int e = nvec * 8 + lane; e < d; e += 32) amax = fmaxf(amax, fabsf(__bfloat162float(src[e])));
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+      const int E = static_cast<int>(__float_as_uint(amax) >> 23);
+      const int sh = amax > 0.f ? max(min(134 - E, 126), -126) : 0;
+      const float up = __uint_as_float(static_cast<uint32_t>(sh + 127) << 23);  // 2^s, exact
+      uint8_t* dh = hq + static_cast<int64_t>(prefix + i) * ldc;
+      uint8_t* dl = lq + static_cast<int64_t>(prefix + i) * ldc;
+      for (int v = lane; v < nvec; v += 32) {
+        const uint4 q = __ldg(s4 + v);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+        uint32_t oh[2], ol[2];
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+          uint32_t h4 = 0, l4 = 0;
+#pragma unroll
+          for (int u = 0; u < 2; ++u) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[2 * j + u]));
+            const float y0 = f.x * up, y1 = f.y * up;
+            const uint32_t h2 = f32x2_to_e4m3x2(y0, y1);
+            const float2 back = f16x2_bits_to_float2(e4m3x2_to_f16x2(h2));
+            const uint32_t l2 = f32x2_to_e4m3x2(y0 - back.x, y1 - back.y);
+            h4 |= h2 << (16 * u);
+            l4 |= l2 << (16 * u);
+          }
+          oh[j] = h4;
+          ol[j] = l4;
+        }
+        *reinterpret_cast<uint2*>(dh + 8 * v) = make_uint2(oh[0], oh[1]);
+        *reinterpret_cast<uint2*>(dl + 8 * v) = make_uint2(ol[0], ol[1]);
+      }
+      for (int e = nvec * 8 + lane; e < d; e += 32) {
+        const float y = __bfloat162float(src[e]) * up;
+        const uint32_t h2 = f32x2_to_e4m3x2(y, 0.f);
+        const float back = f16x2_bits_to_float2(e4m3x2_to_f16x2(h2)).x;
+        dh[e] = static_cast<uint8_t>(h2 & 0xFFu);
+        dl[e] = static_cast<uint8_t>(f32x2_to_e4m3x2(y - back, 0.f) & 0xFFu);
+      }
       if (lane == 0) tok_scale[prefix + i] = amax > 0.f ? __uint_as_float(static_cast<uint32_t>(127 - sh) << 23) : 0.f;
     }
     return;
@@ -226,17 +312,19 @@ int prep_chunk(int P, int sm_count) {
 
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale, int row_format,
-                             uint32_t* status) {
+                             int* n_rows, int sm_count, cudaStream_t st, const BandPlan& plan, float* tok_scale,
+                             int row_format, uint32_t* status) {
   if (row_format != ROWS_BF16 && (tok_scale == nullptr || hc == nullptr)) return cudaErrorInvalidValue;
   const int chunk = prep_chunk(P, sm_count);
   const int grid = (P + chunk - 1) / chunk;
   auto* kern = row_format == ROWS_F16_POW2 ? prep_rows_kernel<ROWS_F16_POW2>
                : row_format == ROWS_E4M3  ? prep_rows_kernel<ROWS_E4M3>
-                                          : prep_rows_kernel<ROWS_BF16>;
+               : row_format == ROWS_E4M3X2 ? prep_rows_kernel<ROWS_E4M3X2>
+                                           : prep_rows_kernel<ROWS_BF16>;
   kern<<<grid, PREP_THREADS, 0, st>>>(pos_masked, block_flags, P, block_len, chunk,
                                       static_cast<const __nv_bfloat16*>(hidden), ld, d,
-                                      static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows, tok_scale, status);
+                                      static_cast<__nv_bfloat16*>(hc), ldc, idx, rowpos, n_rows, tok_scale, status,
+                                      plan);
   return cudaGetLastError();
 }
 
@@ -247,7 +335,7 @@ cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_fla
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restrict__ draft, int n_req, int n_draft,
                                                           int* __restrict__ idx, int* __restrict__ draft_row,
-                                                          int* __restrict__ n_rows) {
+                                                          int* __restrict__ n_rows, BandPlan plan) {
   griddep_launch_dependents();
   const int R = n_req * (n_draft + 1);
   for (int r = blockIdx.x * blockDim.x + threadIdx.x; r < R; r += gridDim.x * blockDim.x) {
@@ -255,16 +343,22 @@ __global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restr
     idx[r] = r;
     draft_row[r] = i < n_draft ? draft[q * n_draft + i] : -1;
   }
-  if (blockIdx.x == 0 && threadIdx.x == 0) *n_rows = R;
+  if (blockIdx.x == 0 && threadIdx.x < 32) {  // N and the plan's vocabulary parts for it
+    const int gv = plan_gv_warp(plan, R > 0 ? cdiv(R, plan_bm(plan, R)) : 1);
+    if (threadIdx.x == 0) {
+      n_rows[0] = R;
+      n_rows[1] = gv;
+    }
+  }
 }
 
 cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,
-                               cudaStream_t st) {
+                               const BandPlan& plan, cudaStream_t st) {
   const int R = n_req * (n_draft + 1);
   int grid = (R + 255) / 256;
   if (grid < 1) grid = 1;
   if (grid > 1024) grid = 1024;
-  prep_verify_kernel<<<grid, 256, 0, st>>>(draft, n_req, n_draft, idx, draft_row, n_rows);
+  prep_verify_kernel<<<grid, 256, 0, st>>>(draft, n_req, n_draft, idx, draft_row, n_rows, plan);
   return cudaGetLastError();
 }
 

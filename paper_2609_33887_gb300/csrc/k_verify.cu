@@ -25,11 +25,11 @@ __global__ void __launch_bounds__(THREADS) merge_verify_kernel(VerifyArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int D = a.n_draft, Rq = D + 1;
   griddep_wait();  // the partials come from the LM-head kernel
-  const int n_rows = *a.n_rows;
+  // partial slots per row: the plan's parts (header word 1) times the CTAs per unit
+  const int ns = a.n_rows[1] * a.plan.cpu;
 
   for (int i = warp; i < Rq; i += THREADS / 32) {
     const int r = q * Rq + i;
-    const int ns = slots_of_row(a.plan, n_rows, r);
     float m = -INFINITY, s = 0.f, t = 0.f, lx = -INFINITY;
     int arg = 0x7fffffff;
     for (int slot = lane; slot < ns; slot += 32) {

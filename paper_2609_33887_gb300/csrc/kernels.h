@@ -25,11 +25,18 @@ struct TauParams {
 // ROWS_F16_POW2 (heads decoded to f16 in the LM head): f16 rows (ldc in
 // elements) holding the bf16 values times 2^s_r, s_r chosen so the row's
 // largest magnitude lands in [2^14, 2^15), tok_scale[r] = 2^-s_r (exact).
-enum : int { ROWS_BF16 = 0, ROWS_E4M3 = 1, ROWS_F16_POW2 = 2 };
+// ROWS_E4M3X2 (E4M3 heads on the 8-bit tensor path, W8A16): each bf16 row,
+// scaled by a power of two 2^s so its largest magnitude lies in [128, 256),
+// as two E4M3 terms hi + lo (hi rows at hc, lo rows at hc + P * ldc, ldc in
+// bytes, a multiple of 16), exact for every element of at least 2^-10 of the
+// row's largest; tok_scale[r] = 2^-s.
+enum : int { ROWS_BF16 = 0, ROWS_E4M3 = 1, ROWS_F16_POW2 = 2, ROWS_E4M3X2 = 3 };
+// n_rows[0] = N and n_rows[1] = the plan's vocabulary parts for N
+// (plan_gv), written by the CTA that holds the last position.
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
-                             int* n_rows, int sm_count, cudaStream_t st, float* tok_scale = nullptr,
-                             int row_format = ROWS_BF16, uint32_t* status = nullptr);
+                             int* n_rows, int sm_count, cudaStream_t st, const BandPlan& plan,
+                             float* tok_scale = nullptr, int row_format = ROWS_BF16, uint32_t* status = nullptr);
 
 // Decodes FP8 e4m3 weight codes to bf16 (exact), row by row: out[v] = code(w[v]).
 cudaError_t launch_dequant_e4m3(const uint8_t* w, int64_t ldw, int V, int d, void* out, int64_t ldo,
@@ -81,7 +88,9 @@ struct PairTokenMaps {
 // 16 x 128-byte boxes).
 // HF_W8A8: E4M3 head and E4M3 token rows (per-row scales), multiplied with
 // tcgen05.mma kind::f8f6f4 (the W8A8 variant of the precision lever).
-enum : int { HF_BF16 = 0, HF_E4M3 = 1, HF_NVFP4 = 2, HF_W8A8 = 3 };
+// HF_E4M3X2: E4M3 head times bf16 token rows packed as two E4M3 terms
+// (ROWS_E4M3X2), both multiplied on kind::f8f6f4 into one accumulator (W8A16).
+enum : int { HF_BF16 = 0, HF_E4M3 = 1, HF_NVFP4 = 2, HF_W8A8 = 3, HF_E4M3X2 = 4 };
 struct PairQuantMaps {
   CUtensorMap codes;
   CUtensorMap scales;
@@ -91,8 +100,9 @@ cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs);
 // hf: HF_BF16 (tmW describes the bf16 head; tmQ unused, may be null) or
 // HF_E4M3 / HF_NVFP4 (tmQ describes the codes, and the NVFP4 block scales;
 // tmW unused). E4M3 and NVFP4 need the TcArgs row scale wscale.
-cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ, int hf,
-                               const TcArgs& a, cudaStream_t st);
+// tmLo: the lo-term maps of HF_E4M3X2 (same boxes as tmH), else may be null.
+cudaError_t launch_lmhead_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW, const PairQuantMaps* tmQ,
+                               const PairTokenMaps* tmLo, int hf, const TcArgs& a, cudaStream_t st);
 
 // a1+a2 with fp32 FMA on the CUDA cores (exact fp32 path; any dtype combo).
 struct SimtArgs {
@@ -139,15 +149,26 @@ struct CommitArgs {
   uint32_t* out_commit;
   int32_t* out_counts;
   uint32_t* status = nullptr;  // device status word (index checks of the bounds-checked build)
+  // vocabulary-parallel split: MERGE_EMIT writes each position's merged
+  // partial (token id + vocab_offset; -inf / 0 / -1 where nothing is
+  // predicted) to emit_*; MERGE_GATHERED reads n_parts partials per position
+  // from part_* laid out [n_parts, P] (position-indexed, no compaction)
+  int vocab_offset = 0;
+  int n_parts = 0;
+  float* emit_m = nullptr;
+  float* emit_s = nullptr;
+  int* emit_a = nullptr;
 };
-cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st);
+enum : int { MERGE_ROWS = 0, MERGE_EMIT = 1, MERGE_GATHERED = 2 };
+cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st, int mode = MERGE_ROWS);
 
 // Verification path (speculative decoding, typical acceptance). Rows are
 // r = q * (n_draft + 1) + i; row i < n_draft of request q verifies draft
 // token draft[q * n_draft + i], the last row of a request gives its bonus token.
-// Prep: idx[r] = r, draft_row[r] = that draft token or -1, *n_rows = R.
+// Prep: idx[r] = r, draft_row[r] = that draft token or -1, n_rows[0] = R,
+// n_rows[1] = the plan's vocabulary parts for R rows.
 cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,
-                               cudaStream_t st);
+                               const BandPlan& plan, cudaStream_t st);
 
 struct VerifyArgs {
   const int* draft_row;

@@ -1,0 +1,54 @@
+// Host check of the LM-head work plan (common.cuh): for each case given on
+// the command line as "n_rows BM GM rows_l2 G n_vt cpu", every (m-tile,
+// v-tile) pair is taken by exactly one unit, the part indices stay below the
+// partial slots the merge reads, and the busiest runner's v-tiles are
+// reported against the even share. Prints one line per case:
+//   ok <n_mt> <gv> <slots> <max_vtiles> <ideal_vtiles>   or   FAIL <reason>
+#include <cstdio>
+#include <cstdlib>
+#include <vector>
+
+#include "common.cuh"
+
+int main(int argc, char** argv) {
+  for (int i = 1; i + 6 < argc; i += 7) {
+    bd::BandPlan p;
+    const int n_rows = std::atoi(argv[i]);
+    p.BM = std::atoi(argv[i + 1]);
+    p.GM = std::atoi(argv[i + 2]);
+    p.rows_l2 = std::atoi(argv[i + 3]);
+    p.G = std::atoi(argv[i + 4]);
+    p.n_vt = std::atoi(argv[i + 5]);
+    p.cpu = std::atoi(argv[i + 6]);
+    const int bm = bd::plan_bm(p, n_rows);
+    const int n_mt = n_rows > 0 ? bd::cdiv(n_rows, bm) : 0;
+    std::vector<int> cover(static_cast<size_t>(n_mt) * p.n_vt, 0);
+    const int slots = n_rows > 0 ? bd::slots_of_row(p, n_rows, 0) : 0;
+    const char* fail = nullptr;
+    long long max_load = 0;
+    for (int r = 0; r < p.G && !fail; ++r) {
+      bd::TileIter it;
+      // the parts the compaction kernel stores beside N (plan_gv_warp: the same rule)
+      it.init(p, n_rows, bd::plan_gv(p, n_mt > 0 ? n_mt : 1), r);
+      long long load = 0;
+      while (it.next_unit()) {
+        if (it.m_tile < 0 || it.m_tile >= n_mt) fail = "m-tile out of range";
+        else if ((it.part + 1) * p.cpu > slots) fail = "part beyond the partial slots";
+        else if (it.vt < 0 || it.vt_end > p.n_vt || it.vt >= it.vt_end) fail = "empty or out-of-range v-tiles";
+        if (fail) break;
+        for (int v = it.vt; v < it.vt_end; ++v) ++cover[static_cast<size_t>(it.m_tile) * p.n_vt + v];
+        load += it.vt_end - it.vt;
+      }
+      if (load > max_load) max_load = load;
+    }
+    for (size_t k = 0; !fail && k < cover.size(); ++k)
+      if (cover[k] != 1) fail = "a (m-tile, v-tile) pair is not taken exactly once";
+    if (fail) {
+      std::printf("FAIL %s\n", fail);
+    } else {
+      std::printf("ok %d %d %d %lld %.3f\n", n_mt, slots / (p.cpu > 0 ? p.cpu : 1), slots, max_load,
+                  static_cast<double>(n_mt) * p.n_vt / p.G);
+    }
+  }
+  return 0;
+}

@@ -38,8 +38,9 @@ def declared_functions():
 
 def test_header_declares_the_abi():
     assert declared_functions() == sorted([
-        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status", "bd_selftest_timeout",
-        "bd_shutdown",
+        "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status",
+        "bd_selftest_timeout", "bd_static_device_status", "bd_static_selftest_timeout", "bd_shutdown",
+        "bd_lmhead_partials", "bd_merge_commit",
         "bd_status_string", "bd_version", "bd_workspace_size", "bd_verify_step", "bd_verify_workspace_size",
         "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
         "bd_redline_select", "bd_redline_sweep", "bd_redline_critical_count", "bd_redline_power",

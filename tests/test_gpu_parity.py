@@ -103,21 +103,71 @@ def test_small_one_cta_tensor_core_variant(name):
 @pytest.mark.parametrize("name", ["e4m3", "e4m3_ktail"])
 @pytest.mark.parametrize("fused", [True, False])
 def test_e4m3_pair_fused_and_decoded(name, fused, monkeypatch):
-    # the pair kernel decodes E4M3 codes in shared memory (rows of 16-byte
-    # multiples), or reads a bf16 copy decoded beforehand
+    # with the two-term 8-bit path switched off, the pair kernel decodes E4M3
+    # codes in shared memory (rows of 16-byte multiples), or reads a bf16 copy
+    # decoded beforehand
+    monkeypatch.setenv("BD_E4M3_SPLIT", "0")
     if not fused:
         monkeypatch.setenv("BD_FUSED_DECODE", "0")
     check(generate(SMALL[name]), variant=3)
 
 
-def test_e4m3_pair_fused_row_magnitudes():
-    # the fused E4M3 path packs the token rows as f16 scaled by a power of two
-    # per row: rows spanning the bf16 exponent range
-    wl = generate(SMALL["e4m3_ktail"])
+def _spread_row_magnitudes(wl):
     exps = (-90, -40, -12, 0, 12, 40, 90)
     k = torch.tensor(exps, dtype=torch.float64)[torch.arange(wl.hidden.shape[0]) % len(exps)]
     wl.hidden = (wl.hidden.double() * torch.exp2(k)[:, None]).to(wl.hidden.dtype)
-    check(wl, variant=3)
+    return wl
+
+
+@pytest.mark.parametrize("split", ["0", "1"])
+def test_e4m3_pair_row_magnitudes(split, monkeypatch):
+    # both E4M3 paths scale each packed row by a power of two (f16 rows for the
+    # converter path, two E4M3 terms for the 8-bit path): rows spanning the
+    # bf16 exponent range
+    monkeypatch.setenv("BD_E4M3_SPLIT", split)
+    check(_spread_row_magnitudes(generate(SMALL["e4m3_ktail"])), variant=3)
+
+
+@pytest.mark.parametrize("name", ["e4m3", "e4m3_ktail"])
+def test_e4m3_two_term_rows_within_the_bf16_tolerance(name):
+    # the 8-bit path represents every bf16 element of at least 2^-10 of its
+    # row's largest exactly as hi + lo and multiplies exact E4M3 products into
+    # fp32: it meets the bf16 confidence tolerance, not only the FP8 one
+    _, _, rep = check(generate(SMALL[name]))
+    assert rep.max_dconf < 2e-3
+
+
+def test_e4m3_two_term_path_keeps_small_products():
+    """Two vocabulary entries per position whose logits differ only through
+    products 2^16 times smaller than the logit (16 + 8 * 2^-12 against 16):
+    the exact gap, 2^-9, is above the 1e-3 tie exemption, so the token is
+    decided by whether the tensor path keeps those products in its fp32 sum.
+    Half the positions need the higher index to win, half the lower."""
+    L, d, V = 32, 128, 512
+    w = torch.zeros(V, d)
+    h = torch.zeros(L, d)
+    small = list(range(1, 5)) + list(range(65, 69))  # in both 64-column halves of the row
+    for p in range(L):
+        a, b = 2 * p + 3, 2 * p + 300  # two entries in different v-tiles
+        k_p = 8 + p  # this position's own column: only its pair sees the large product
+        w[a, k_p] = w[b, k_p] = 1.0
+        winner = b if p % 2 == 0 else a
+        for k in small:
+            w[winner, k] = 2.0 ** -6
+        h[p, k_p] = 16.0
+        h[p, small] = 2.0 ** -6
+    from workloads.generate import Workload
+
+    cfg = scaled(B256X8X64_E4M3, n_seq=1, n_slots=1, block_len=L, d=d, V=V, mask_frac=1.0, tau=(0.4, 0.6),
+                 name="small_products")
+    wl = Workload(cfg=cfg, hidden=h.to(torch.bfloat16), weight=w.to(torch.float8_e4m3fn),
+                  weight_scale=torch.ones(V), pos_masked=torch.ones(L, dtype=torch.uint8),
+                  block_flags=torch.tensor([3], dtype=torch.uint8), tau=cfg.tau, mask_token_id=-1)
+    out, ref, rep = check(wl)
+    expect = np.array([2 * p + 300 if p % 2 == 0 else 2 * p + 3 for p in range(L)])
+    assert np.array_equal(ref["tokens"], expect)
+    assert np.array_equal(out["tokens"], expect)
+    assert rep.token_mismatch_exempt == 0
 
 
 @pytest.mark.parametrize("name", ["bf16_1mt", "bf16_5mt_ktail", "e4m3"])
@@ -219,25 +269,64 @@ def _sample_blocks(cfg, n, seed=99):
     return sorted(rng.choice(cfg.n_blocks, size=min(n, cfg.n_blocks), replace=False).tolist())
 
 
+def _edge_blocks(wl):
+    """Blocks holding the compacted rows where a work plan can break: the first
+    row, the rows at either side of every 128- and 256-row tile boundary of the
+    last two tiles (the ragged last m-tile / token group and the one before),
+    and the last row. Compacted rows are the masked positions of active blocks
+    in ascending order."""
+    cfg = wl.cfg
+    act = np.repeat((wl.block_flags.numpy() & 1) != 0, cfg.block_len)
+    rows = np.flatnonzero((wl.pos_masked.numpy() != 0) & act)  # compacted row -> position
+    n = rows.size
+    if n == 0:
+        return []
+    pick = {0, n - 1}
+    for tile in (128, 256):
+        last = (n - 1) // tile * tile  # first row of the last tile
+        for r in (last - tile - 1, last - tile, last - 1, last):
+            if 0 <= r < n:
+                pick.add(r)
+    return sorted({int(rows[r]) // cfg.block_len for r in pick})
+
+
+def _sample_with_edges(wl, n, seed=99):
+    return sorted(set(_edge_blocks(wl)) | set(_sample_blocks(wl.cfg, n, seed)))
+
+
 def test_full_size_b8_all_positions():
     wl = generate(B8X2X32_BF16)
     _, _, rep = check(wl)
     assert rep.n_live > 250
 
 
-@pytest.mark.parametrize("i,n_blocks", [(2, 8), (3, 4), (4, 3)])
+@pytest.mark.parametrize("i,n_blocks", [(2, 8), (3, 16), (4, 16)])
 def test_full_size_sampled_blocks(i, n_blocks):
+    # seeded random blocks plus the blocks of the first and last compacted rows
+    # and of the last two tiles' boundaries
     wl = generate(CONFIGS[i])
-    blocks = _sample_blocks(CONFIGS[i], n_blocks)
+    blocks = _sample_with_edges(wl, n_blocks)
+    assert set(_edge_blocks(wl)) <= set(blocks) and len(blocks) >= n_blocks
     _, _, rep = check(wl, blocks=blocks)
     assert rep.n_live > 0
 
 
-@pytest.mark.parametrize("i,variant,n_blocks", [(1, 2, None), (3, 3, 3), (4, 3, 2)])
+@pytest.mark.parametrize("i,variant,n_blocks", [(1, 2, None), (3, 2, 3), (4, 2, 2)])
 def test_full_size_with_the_other_tensor_core_kernel(i, variant, n_blocks):
-    # the automatic choice takes the CTA-pair kernel for the 8x2x32 window and
-    # the one-CTA kernel for the two largest; check each with the other kernel
+    # the automatic choice takes the CTA-pair kernel at every window size (for
+    # the E4M3 head on the 8-bit path); check each workload with the one-CTA
+    # kernel (tokens on M; E4M3 heads decoded to a bf16 copy first)
     wl = generate(CONFIGS[i])
-    blocks = None if n_blocks is None else _sample_blocks(CONFIGS[i], n_blocks, seed=5)
+    blocks = None if n_blocks is None else _sample_with_edges(wl, n_blocks, seed=5)
     _, _, rep = check(wl, variant=variant, blocks=blocks)
+    assert rep.n_live > 0
+
+
+def test_full_size_e4m3_head_decoded_in_the_pair_kernel(monkeypatch):
+    # the largest window with the 8-bit path switched off: the pair kernel's
+    # converter warps decode the E4M3 head (f16 operands) at every v-tile
+    monkeypatch.setenv("BD_E4M3_SPLIT", "0")
+    monkeypatch.setenv("BD_PAIR_MAX_P", str(1 << 30))
+    wl = generate(B256X8X64_E4M3)
+    _, _, rep = check(wl, variant=3, blocks=_sample_with_edges(wl, 2, seed=6))
     assert rep.n_live > 0

@@ -58,6 +58,20 @@ def test_e4m3_weights_apply_the_row_scale():
     assert np.array_equal(w, np.array([[0.5, 1.0], [3.0, -3.0]]))
 
 
+def test_e4m3_weights_equal_the_elementwise_decode_times_the_row_scale():
+    # every code (NaN codes included) in random rows against the format's
+    # decode applied element by element, times the row scale
+    rng = np.random.default_rng(3)
+    codes = rng.integers(0, 256, size=(300, 77), dtype=np.uint8)
+    codes[0, :] = np.arange(77, dtype=np.uint8) + 179  # the top codes, 0xFF (NaN) among them
+    scale = rng.uniform(1e-4, 3.0, size=300).astype(np.float32)
+    w = oracle.weights_f64(codes, "e4m3", scale)
+    ref = oracle.decode_e4m3(codes) * scale.astype(np.float64)[:, None]
+    nan = np.isnan(ref)
+    assert nan.any() and np.array_equal(np.isnan(w), nan)
+    assert np.array_equal(w[~nan], ref[~nan])
+
+
 # ----------------------------------------------------------- closed forms --
 
 def _planted_head(V, d, v_star, k_star):

@@ -1,0 +1,86 @@
+"""The LM-head work plan (csrc/common.cuh), compiled for the host and checked
+without a GPU: every (m-tile, v-tile) pair of the logits is computed by
+exactly one unit, partial-slot indices stay within what the merge reads, and
+the busiest runner carries close to an even share of the v-tiles. The cases
+are the five workloads' windows in each kernel's plan plus ragged and
+degenerate ones."""
+
+import os
+import shutil
+import subprocess
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+CSRC = os.path.join(ROOT, "paper_2609_33887_gb300", "csrc")
+
+
+def _nvcc():
+    for cand in (os.environ.get("NVCC"), shutil.which("nvcc"), "/usr/local/cuda/bin/nvcc"):
+        if cand and os.path.exists(cand):
+            return cand
+    return None
+
+
+@pytest.fixture(scope="module")
+def plan_check(tmp_path_factory):
+    nvcc = _nvcc()
+    if nvcc is None:
+        pytest.skip("no CUDA toolkit")
+    exe = str(tmp_path_factory.mktemp("plan") / "plan_check")
+    r = subprocess.run([nvcc, "-std=c++17", "-O1", "-I" + CSRC, os.path.join(ROOT, "tests", "plan_check.cu"),
+                        "-o", exe], capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr
+    return exe
+
+
+def run_cases(exe, cases):
+    args = [str(x) for c in cases for x in c]
+    out = subprocess.run([exe] + args, capture_output=True, text=True, check=True).stdout.split("\n")
+    return [l.split() for l in out if l.strip()]
+
+
+PAIR_G, SMS = 76, 152
+# (n_rows, BM, GM, rows_l2, G, n_vt, cpu)
+CASES = [
+    # pair kernel (BM = 0: token groups from N; GM = 0: bands from the L2 row budget)
+    (294, 0, 0, 16384, PAIR_G, 594, 2),      # 8 x 2 x 32, d = 2048
+    (2048, 0, 0, 16384, PAIR_G, 614, 2),     # 32 x 4 x 32
+    (8191, 0, 0, 8192, PAIR_G, 594, 2),      # 64 x 4 x 64, d = 4096
+    (8200, 0, 0, 8192, PAIR_G, 594, 2),      # one row past a full band
+    (52429, 0, 0, 6553, PAIR_G, 614, 2),     # 256 x 8 x 64, d = 5120
+    (32, 0, 0, 1 << 20, PAIR_G, 16, 2),      # the tiny window
+    (1, 0, 0, 1 << 20, PAIR_G, 1, 2),        # one row, one v-tile
+    (257, 0, 0, 300, 3, 7, 2),               # few runners, band of one group
+    # one-CTA kernel (BM = 128) and the SIMT kernel (BM = 32)
+    (8191, 128, 0, 8192, SMS, 594, 1),
+    (52429, 128, 0, 6553, SMS, 614, 1),
+    (294, 32, 8, 0, 2 * SMS, 594, 1),
+    (5, 32, 0, 100, 2 * SMS, 3, 1),
+]
+
+
+def test_plan_covers_every_tile_once_with_balanced_runners(plan_check):
+    res = run_cases(plan_check, CASES)
+    assert len(res) == len(CASES)
+    for case, r in zip(CASES, res):
+        assert r[0] == "ok", (case, r)
+        n_mt, gv, slots, max_load, ideal = int(r[1]), int(r[2]), int(r[3]), int(r[4]), float(r[5])
+        G, n_vt, cpu = case[4], case[5], case[6]
+        assert 1 <= gv <= min(G, n_vt) and slots == gv * cpu
+        # the busiest runner: within 10% of an even share plus one unit of
+        # work (ceil(n_vt / gv) v-tiles), which no static split can avoid
+        assert max_load <= 1.10 * ideal + -(-n_vt // gv), (case, r)
+
+
+def test_plan_without_rows(plan_check):
+    (r,) = run_cases(plan_check, [(0, 0, 0, 1000, PAIR_G, 594, 2)])
+    assert r[0] == "ok" and int(r[1]) == 0
+
+
+def test_large_windows_read_the_head_once_per_band(plan_check):
+    # with the L2 row budget of the 64 x 4 x 64 window (64 MiB of 8 KiB rows)
+    # every token group sits in one band: the plan streams the head once
+    (r,) = run_cases(plan_check, [(8191, 0, 0, 8192, PAIR_G, 594, 2)])
+    n_mt = int(r[1])
+    assert n_mt == 32 and 8192 // 256 >= n_mt
