@@ -218,6 +218,15 @@ int64_t row_operand_bytes(const Call& c) {
   return 2 * c.ldc;
 }
 
+// Bytes of one head row as the LM-head kernel reads it: the stored row for
+// bf16 / E4M3 heads on the tensor-core kernels, the decoded bf16 copy where
+// one is made, fp32 / stored rows for the SIMT kernel.
+int64_t head_operand_bytes(const Call& c) {
+  if (c.tc && !c.fused && !c.fp8_act && !c.split && (c.wdt == BD_E4M3 || c.wdt == BD_NVFP4)) return 2 * c.ldq;
+  if (c.wdt == BD_NVFP4) return (c.d + 1) / 2;
+  return c.d * esize(c.wdt);
+}
+
 BandPlan make_plan(const Call& c, int sm_count, int pairs) {
   BandPlan p;
   if (c.pair) {
@@ -236,13 +245,11 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs) {
     p.G = 2 * sm_count;
     p.cpu = 1;
   }
-  // bands: as many m-tiles as keep their rows within the L2 budget (they are
-  // re-read for every v-tile while the head streams through once per band)
+  // bands: GM derived on the device from the head and row bytes (0), or fixed
   p.GM = env_int("BD_PLAN_GM", 0, 0, 1 << 20);
-  const int64_t budget = int64_t(env_int("BD_L2_ROWS_MB", 64, 1, 1 << 16)) << 20;
-  const int64_t rows = budget / std::max<int64_t>(1, row_operand_bytes(c));
-  p.rows_l2 = static_cast<int>(std::min<int64_t>(rows, int64_t(1) << 30));
   p.n_vt = static_cast<int>((c.V + p.BN - 1) / p.BN);
+  p.vt_kb = static_cast<int>(std::max<int64_t>(1, int64_t(p.BN) * head_operand_bytes(c) / 1024));
+  p.row_bytes = static_cast<int>(std::min<int64_t>(row_operand_bytes(c), int64_t(1) << 30));
   return p;
 }
 

@@ -41,24 +41,29 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // row in slot `part` (times the CTAs per unit) of the partial arrays.
 //
 // Units are numbered band by band: a band holds at most GM consecutive
-// m-tiles, sized so that its rows stay resident in L2, and inside a band the
-// units go part by part (all m-tiles of part 0, then part 1, ...). Runner c
-// takes units c, c + G, c + 2G, ...: the G units in flight at any time are
-// consecutive, i.e. a few parts of one band, so every head tile is fetched
-// from HBM about once per band and re-read from L2 by the m-tiles that share
-// it while the band's rows stay in L2. gv minimises the makespan
+// m-tiles, and inside a band the units go part by part (all m-tiles of part
+// 0, then part 1, ...). Runner c takes units c, c + G, c + 2G, ...: the G
+// units in flight at any time are consecutive, about GM m-tiles times G / GM
+// parts, so every head tile is fetched from HBM about once per band and
+// re-read from L2 by the band's m-tiles, and each runner re-reads its
+// m-tile's rows from L2 at every v-tile. A window whose packed rows fit
+// ROWS_ONE_BAND bytes is one band (the head is streamed once); a larger one
+// keeps about GM m-tiles of rows plus G / GM head tiles in L2 at a time, and
+// GM = sqrt(G * head tile bytes / m-tile bytes) minimises that sum. gv
+// minimises the makespan
 // ceil(units / G) * (ceil(n_vt / gv) + 1/2) (half a v-tile for each unit's
 // start and finish). N is only known on the device, so kernels recompute the
 // plan from it.
 // -------------------------------------------------------------------------
 struct BandPlan {
-  int BM;       // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
-  int BN;       // vocabulary entries per v-tile
-  int GM;       // m-tiles per band at most; 0 = derived from rows_l2
-  int rows_l2;  // rows a band may hold (GM = 0): the L2 budget over the packed row bytes
-  int G;        // units that can run at once (CTAs, or CTA pairs)
-  int n_vt;     // ceil(V / BN)
-  int cpu;      // CTAs per unit: each writes its own partial, so a part has cpu slots
+  int BM;         // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
+  int BN;         // vocabulary entries per v-tile
+  int GM;         // m-tiles per band at most; 0 = derived (see plan_gm)
+  int G;          // units that can run at once (CTAs, or CTA pairs)
+  int n_vt;       // ceil(V / BN)
+  int cpu;        // CTAs per unit: each writes its own partial, so a part has cpu slots
+  int vt_kb;      // KiB of head per v-tile (BN rows as the kernel reads them)
+  int row_bytes;  // bytes of one packed token row as the kernel reads it
 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
@@ -75,10 +80,17 @@ __host__ __device__ __forceinline__ int plan_bm(const BandPlan& p, int n_rows) {
   return p.BM > 0 ? p.BM : pair_group_rows(n_rows);
 }
 
-// m-tiles per band (all bands but the last are full)
-__host__ __device__ __forceinline__ int plan_gm(const BandPlan& p, int bm) {
+// Packed rows up to this size are one band.
+constexpr double ROWS_ONE_BAND = 64.0 * 1024 * 1024;
+
+// m-tiles per band (all bands but the last are full): all n_mt when their
+// rows fit ROWS_ONE_BAND, else the integer nearest sqrt(G * head tile bytes /
+// m-tile bytes), at least 1
+__host__ __device__ __forceinline__ int plan_gm(const BandPlan& p, int bm, int n_mt) {
   if (p.GM > 0) return p.GM;
-  const int g = p.rows_l2 / bm;
+  const double tile = static_cast<double>(bm) * (p.row_bytes > 0 ? p.row_bytes : 1);
+  if (n_mt * tile <= ROWS_ONE_BAND) return n_mt > 0 ? n_mt : 1;
+  const int g = static_cast<int>(sqrt(static_cast<double>(p.G) * p.vt_kb * 1024.0 / tile) + 0.5);
   return g < 1 ? 1 : g;
 }
 
@@ -145,7 +157,7 @@ struct TileIter {
     n_vt = plan.n_vt;
     const int bm = plan_bm(plan, n_rows);
     n_mt = n_rows > 0 ? cdiv(n_rows, bm) : 0;
-    gm_full = plan_gm(plan, bm);
+    gm_full = plan_gm(plan, bm, n_mt);
     gv = parts;
     n_units = static_cast<int64_t>(n_mt) * gv;
     u = static_cast<int64_t>(runner) - G;
@@ -412,6 +424,12 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
   asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
   return p;
 }
+
+// L2 policy of the LM head's weight tiles: evict-first. The band's token
+// groups re-read each head tile from L2 shortly after the first of them
+// fetched it; the default priority measured slower at every window size
+// (8 x 2 x 32: 143 against 139 us; 64 x 4 x 64: 6.36 against 5.88 ms).
+__device__ __forceinline__ uint64_t head_policy() { return policy_evict_first(); }
 
 __device__ __forceinline__ uint64_t policy_evict_last() {
   uint64_t p;

@@ -4,6 +4,11 @@
 // the tensor-core kernel, with 32-row m-tiles and 256-entry v-tiles. The
 // verification instantiation (VERIFY = true) also carries the entropy
 // accumulator and the logit of each row's draft entry.
+//
+// A CTA of 256 threads computes a 32-row x 64-entry tile: thread t owns
+// vocabulary column t % 64 of the tile for rows 8 (t / 64) .. 8 (t / 64) + 7,
+// so a small window still spreads over many CTAs (the 32 x 4096 fp32 window:
+// 64 v-tiles).
 #include <cuda_fp16.h>
 
 #include "bdcommit.h"
@@ -15,7 +20,10 @@ namespace {
 
 constexpr int KC = 32;      // hidden columns staged per step
 constexpr int THREADS = 256;
-static_assert(SIMT_BN == THREADS, "one vocabulary column per thread");
+constexpr int ROW_GROUPS = THREADS / SIMT_BN;   // 4 groups of rows
+constexpr int RPT = SIMT_BM / ROW_GROUPS;        // 8 rows per thread
+constexpr int CPL = SIMT_BN / 32;                // columns a lane scans in the reductions
+static_assert(THREADS % SIMT_BN == 0 && SIMT_BM % ROW_GROUPS == 0, "column x row-group split");
 static_assert(SIMT_BM == 32, "one row per lane in the reductions");
 
 __device__ __forceinline__ float load_h(const void* p, int64_t i, int dt) {
@@ -65,6 +73,7 @@ template <bool VERIFY>
 __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   __shared__ SimtSmem sm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int col = tid % SIMT_BN, rg = tid / SIMT_BN;  // this thread's column and row group
   griddep_wait();  // idx and N come from the preceding kernel
   const int n_rows = a.n_rows[0];
   const int parts = a.n_rows[1];  // vocabulary parts of the plan (see common.cuh)
@@ -85,10 +94,10 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
     }
     __syncthreads();
     for (int vt = it.vt; vt < it.vt_end; ++vt) {
-      const int v = vt * SIMT_BN + tid;
-      float acc[SIMT_BM];
+      const int v = vt * SIMT_BN + col;
+      float acc[RPT];
 #pragma unroll
-      for (int r = 0; r < SIMT_BM; ++r) acc[r] = 0.f;
+      for (int r = 0; r < RPT; ++r) acc[r] = 0.f;
       for (int k0 = 0; k0 < a.d; k0 += KC) {
         // stage 32 hidden rows x KC columns (rows gathered through idx)
         for (int e = tid; e < SIMT_BM * KC; e += THREADS) {
@@ -109,39 +118,40 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
           sm.u.ws[vr][kk] = x;
         }
         __syncthreads();
-#pragma unroll 4
+#pragma unroll 8
         for (int kk = 0; kk < KC; ++kk) {
-          const float wv = sm.u.ws[tid][kk];
+          const float wv = sm.u.ws[col][kk];
 #pragma unroll
-          for (int r = 0; r < SIMT_BM; ++r) acc[r] = fmaf(sm.hs[r][kk], wv, acc[r]);
+          for (int r = 0; r < RPT; ++r) acc[r] = fmaf(sm.hs[rg * RPT + r][kk], wv, acc[r]);
         }
         __syncthreads();
       }
       const bool dead = (v >= a.V) || (v == a.mask_id);
       const float sc = (a.wscale != nullptr && v < a.V) ? a.wscale[v] : 1.f;
 #pragma unroll
-      for (int r = 0; r < SIMT_BM; ++r) {
+      for (int r = 0; r < RPT; ++r) {
+        const int row = rg * RPT + r;
         const float l = dead ? -INFINITY : acc[r] * sc;
-        sm.u.lg[r][tid] = l;
+        sm.u.lg[row][col] = l;
         if constexpr (VERIFY) {
-          if (v == sm.xd[r]) sm.rx[r] = l;  // one column per row holds the draft entry
+          if (v == sm.xd[row]) sm.rx[row] = l;  // one column per row holds the draft entry
         }
       }
       __syncthreads();
-      // warp w reduces rows 4w..4w+3; lane l scans columns 8l..8l+7 in order
+      // warp w reduces rows 4w..4w+3; lane l scans columns CPL l .. CPL l + CPL - 1 in order
       for (int rr = 0; rr < SIMT_BM / 8; ++rr) {
         const int r = warp * (SIMT_BM / 8) + rr;
         float m = -INFINITY, s = 0.f, t = 0.f;
         int arg = 0x7fffffff;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          const float x = sm.u.lg[r][lane * 8 + j];
+        for (int j = 0; j < CPL; ++j) {
+          const float x = sm.u.lg[r][lane * CPL + j];
           if (x != -INFINITY) {
             // one logit is a state of max x, sum 1 and first moment 0
             if constexpr (VERIFY)
-              softmax_combine_t(m, s, arg, t, x, 1.f, vt * SIMT_BN + lane * 8 + j, 0.f);
+              softmax_combine_t(m, s, arg, t, x, 1.f, vt * SIMT_BN + lane * CPL + j, 0.f);
             else
-              softmax_combine(m, s, arg, x, 1.f, vt * SIMT_BN + lane * 8 + j);
+              softmax_combine(m, s, arg, x, 1.f, vt * SIMT_BN + lane * CPL + j);
           }
         }
 #pragma unroll

@@ -127,7 +127,7 @@ struct SimtArgs {
   float* part_x = nullptr;
 };
 constexpr int SIMT_BM = 32;
-constexpr int SIMT_BN = 256;
+constexpr int SIMT_BN = 64;
 cudaError_t launch_lmhead_simt(const SimtArgs& a, cudaStream_t st);
 
 // a3+a4: merge of the partials per row, then the threshold commit with the

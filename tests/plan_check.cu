@@ -1,5 +1,5 @@
 // Host check of the LM-head work plan (common.cuh): for each case given on
-// the command line as "n_rows BM GM rows_l2 G n_vt cpu", every (m-tile,
+// the command line as "n_rows BM GM vt_kb row_bytes G n_vt cpu", every (m-tile,
 // v-tile) pair is taken by exactly one unit, the part indices stay below the
 // partial slots the merge reads, and the busiest runner's v-tiles are
 // reported against the even share. Prints one line per case:
@@ -11,15 +11,16 @@
 #include "common.cuh"
 
 int main(int argc, char** argv) {
-  for (int i = 1; i + 6 < argc; i += 7) {
+  for (int i = 1; i + 7 < argc; i += 8) {
     bd::BandPlan p;
     const int n_rows = std::atoi(argv[i]);
     p.BM = std::atoi(argv[i + 1]);
     p.GM = std::atoi(argv[i + 2]);
-    p.rows_l2 = std::atoi(argv[i + 3]);
-    p.G = std::atoi(argv[i + 4]);
-    p.n_vt = std::atoi(argv[i + 5]);
-    p.cpu = std::atoi(argv[i + 6]);
+    p.vt_kb = std::atoi(argv[i + 3]);
+    p.row_bytes = std::atoi(argv[i + 4]);
+    p.G = std::atoi(argv[i + 5]);
+    p.n_vt = std::atoi(argv[i + 6]);
+    p.cpu = std::atoi(argv[i + 7]);
     const int bm = bd::plan_bm(p, n_rows);
     const int n_mt = n_rows > 0 ? bd::cdiv(n_rows, bm) : 0;
     std::vector<int> cover(static_cast<size_t>(n_mt) * p.n_vt, 0);
@@ -46,8 +47,8 @@ int main(int argc, char** argv) {
     if (fail) {
       std::printf("FAIL %s\n", fail);
     } else {
-      std::printf("ok %d %d %d %lld %.3f\n", n_mt, slots / (p.cpu > 0 ? p.cpu : 1), slots, max_load,
-                  static_cast<double>(n_mt) * p.n_vt / p.G);
+      std::printf("ok %d %d %d %lld %.3f %d\n", n_mt, slots / (p.cpu > 0 ? p.cpu : 1), slots, max_load,
+                  static_cast<double>(n_mt) * p.n_vt / p.G, bd::plan_gm(p, bm, n_mt));
     }
   }
   return 0;

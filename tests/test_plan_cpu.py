@@ -41,22 +41,25 @@ def run_cases(exe, cases):
 
 
 PAIR_G, SMS = 76, 152
-# (n_rows, BM, GM, rows_l2, G, n_vt, cpu)
+# (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu); vt_kb = KiB of head per
+# v-tile, row_bytes = bytes of a packed token row, as the kernels read them
 CASES = [
-    # pair kernel (BM = 0: token groups from N; GM = 0: bands from the L2 row budget)
-    (294, 0, 0, 16384, PAIR_G, 594, 2),      # 8 x 2 x 32, d = 2048
-    (2048, 0, 0, 16384, PAIR_G, 614, 2),     # 32 x 4 x 32
-    (8191, 0, 0, 8192, PAIR_G, 594, 2),      # 64 x 4 x 64, d = 4096
-    (8200, 0, 0, 8192, PAIR_G, 594, 2),      # one row past a full band
-    (52429, 0, 0, 6553, PAIR_G, 614, 2),     # 256 x 8 x 64, d = 5120
-    (32, 0, 0, 1 << 20, PAIR_G, 16, 2),      # the tiny window
-    (1, 0, 0, 1 << 20, PAIR_G, 1, 2),        # one row, one v-tile
-    (257, 0, 0, 300, 3, 7, 2),               # few runners, band of one group
-    # one-CTA kernel (BM = 128) and the SIMT kernel (BM = 32)
-    (8191, 128, 0, 8192, SMS, 594, 1),
-    (52429, 128, 0, 6553, SMS, 614, 1),
-    (294, 32, 8, 0, 2 * SMS, 594, 1),
-    (5, 32, 0, 100, 2 * SMS, 3, 1),
+    # pair kernel (BM = 0: token groups from N; GM = 0: bands by the square-root rule)
+    (294, 0, 0, 1024, 4096, PAIR_G, 594, 2),       # 8 x 2 x 32, d = 2048, bf16
+    (2048, 0, 0, 1024, 4096, PAIR_G, 614, 2),      # 32 x 4 x 32
+    (8191, 0, 0, 2048, 8192, PAIR_G, 594, 2),      # 64 x 4 x 64, d = 4096
+    (8200, 0, 0, 2048, 8192, PAIR_G, 594, 2),      # one row into another group
+    (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2),    # 256 x 8 x 64, d = 5120, E4M3 head, two-term rows
+    (32, 0, 0, 64, 1024, PAIR_G, 16, 2),           # the tiny window
+    (1, 0, 0, 1, 16, PAIR_G, 1, 2),                # one row, one v-tile
+    (257, 0, 0, 1024, 4096, 3, 7, 2),              # few runners
+    (5000, 0, 7, 1024, 4096, PAIR_G, 100, 2),      # a fixed band size
+    # one-CTA kernel (BM = 128) and the SIMT kernel (BM = 32, 64-entry v-tiles)
+    (8191, 128, 0, 2048, 8192, SMS, 594, 1),
+    (52429, 128, 0, 2560, 10240, SMS, 614, 1),
+    (294, 32, 0, 512, 4096, 2 * SMS, 2374, 1),
+    (32, 32, 0, 64, 1024, 2 * SMS, 64, 1),
+    (5, 32, 0, 1, 100, 2 * SMS, 3, 1),
 ]
 
 
@@ -66,7 +69,7 @@ def test_plan_covers_every_tile_once_with_balanced_runners(plan_check):
     for case, r in zip(CASES, res):
         assert r[0] == "ok", (case, r)
         n_mt, gv, slots, max_load, ideal = int(r[1]), int(r[2]), int(r[3]), int(r[4]), float(r[5])
-        G, n_vt, cpu = case[4], case[5], case[6]
+        G, n_vt, cpu = case[5], case[6], case[7]
         assert 1 <= gv <= min(G, n_vt) and slots == gv * cpu
         # the busiest runner: within 10% of an even share plus one unit of
         # work (ceil(n_vt / gv) v-tiles), which no static split can avoid
@@ -74,13 +77,18 @@ def test_plan_covers_every_tile_once_with_balanced_runners(plan_check):
 
 
 def test_plan_without_rows(plan_check):
-    (r,) = run_cases(plan_check, [(0, 0, 0, 1000, PAIR_G, 594, 2)])
+    (r,) = run_cases(plan_check, [(0, 0, 0, 1024, 4096, PAIR_G, 594, 2)])
     assert r[0] == "ok" and int(r[1]) == 0
 
 
-def test_large_windows_read_the_head_once_per_band(plan_check):
-    # with the L2 row budget of the 64 x 4 x 64 window (64 MiB of 8 KiB rows)
-    # every token group sits in one band: the plan streams the head once
-    (r,) = run_cases(plan_check, [(8191, 0, 0, 8192, PAIR_G, 594, 2)])
-    n_mt = int(r[1])
-    assert n_mt == 32 and 8192 // 256 >= n_mt
+def test_band_size(plan_check):
+    # rows up to 64 MiB are one band: the 64 x 4 x 64 window's 32 groups of
+    # 256 rows x 8 KiB (64 MiB), the head streamed once; beyond that GM =
+    # round(sqrt(G * head tile bytes / m-tile bytes)): 1.25 MiB E4M3 head tiles
+    # and 2.5 MiB two-term groups (256 x 8 x 64) give sqrt(38) -> 6, and one row
+    # past 64 MiB gives sqrt(76) -> 9; a fixed GM is kept
+    rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, PAIR_G, 594, 2),
+                                  (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2),
+                                  (8200, 0, 0, 2048, 8192, PAIR_G, 594, 2),
+                                  (5000, 0, 7, 1024, 4096, PAIR_G, 100, 2)])
+    assert [int(r[6]) for r in rows] == [32, 6, 9, 7]
