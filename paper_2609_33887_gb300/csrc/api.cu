@@ -415,6 +415,8 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
     a.part_t = part.t;
     a.part_x = part.x;
     a.tok_scale = tok_scale;
+    a.l2_head = env_int("BD_L2_HEAD", bd::L2_EVICT_FIRST, 0, 2);
+    a.l2_rows = env_int("BD_L2_ROWS", bd::L2_EVICT_LAST, 0, 2);
     rc = c.pair ? cuda_status(bd::launch_lmhead_pair(tmTok, tmB, c.fused ? &tmQ : nullptr, c.split ? &tmLo : nullptr,
                                                      hf, a, st))
                 : cuda_status(bd::launch_lmhead_tc(tmA, tmB, a, env_int("BD_TC_STAGES", 4, 3, 4), st));

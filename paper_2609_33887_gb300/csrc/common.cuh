@@ -425,16 +425,23 @@ __device__ __forceinline__ uint64_t policy_evict_first() {
   return p;
 }
 
-// L2 policy of the LM head's weight tiles: evict-first. The band's token
-// groups re-read each head tile from L2 shortly after the first of them
-// fetched it; the default priority measured slower at every window size
-// (8 x 2 x 32: 143 against 139 us; 64 x 4 x 64: 6.36 against 5.88 ms).
-__device__ __forceinline__ uint64_t head_policy() { return policy_evict_first(); }
+__device__ __forceinline__ uint64_t policy_evict_normal() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
 
 __device__ __forceinline__ uint64_t policy_evict_last() {
   uint64_t p;
   asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
   return p;
+}
+
+// L2 eviction priority of a stream of TMA loads: L2_EVICT_FIRST, L2_EVICT_NORMAL
+// or L2_EVICT_LAST (the LM-head kernels take theirs from TcArgs).
+enum : int { L2_EVICT_FIRST = 0, L2_EVICT_NORMAL = 1, L2_EVICT_LAST = 2 };
+__device__ __forceinline__ uint64_t l2_policy(int sel) {
+  return sel == L2_EVICT_LAST ? policy_evict_last() : sel == L2_EVICT_NORMAL ? policy_evict_normal() : policy_evict_first();
 }
 
 // 2-D tiled load global -> shared; completes `bytes` of transaction count on `bar`.

@@ -417,8 +417,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     const bool leader = elect_one();
     // head rows: fetched from HBM once per band and re-read from L2 by the
     // band's other token groups; token rows: re-read for every v-tile
-    const uint64_t pol_w = head_policy();
-    const uint64_t pol_h = policy_evict_last();
+    const uint64_t pol_w = l2_policy(a.l2_head);
+    const uint64_t pol_h = l2_policy(a.l2_rows);
     const uint32_t full0_leader = mapa_shared(smem_u32(&ctl->full[0]), 0);
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
@@ -555,7 +555,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   } else if (QUANT && warp == RAW_PRODUCER) {
     // ------------------------------------------------------ raw-code producer (quantised heads)
     const bool leader = elect_one();
-    const uint64_t pol = head_policy();  // the codes of the band's head tiles, as above
+    const uint64_t pol = l2_policy(a.l2_head);  // the codes of the band's head tiles, as above
     const int RS = RSTAGES;
     const int nkr = cdiv(nk, raw_k<HF>());
     uint32_t r = 0, rph = 0;

@@ -92,8 +92,8 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     // ------------------------------------------------------ TMA producer
     // the whole warp walks the stages (warp-uniform waits); one lane issues
     const bool leader = elect_one();
-    const uint64_t pol_a = policy_evict_last();   // hidden rows: re-read by every part
-    const uint64_t pol_b = head_policy();         // head rows: fetched once per band, re-read from L2 by its m-tiles
+    const uint64_t pol_a = l2_policy(a.l2_rows);  // hidden rows: re-read by every part
+    const uint64_t pol_b = l2_policy(a.l2_head);  // head rows: fetched once per band, re-read from L2 by its m-tiles
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / parity of last issue
     TileIter it;

@@ -66,6 +66,9 @@ struct TcArgs {
   float* part_x = nullptr;
   // W8A8 only: the dequantisation scale of each packed token row
   const float* tok_scale = nullptr;
+  // L2 eviction priorities (L2_EVICT_*) of the head tiles and of the token rows
+  int l2_head = L2_EVICT_FIRST;
+  int l2_rows = L2_EVICT_LAST;
 };
 constexpr int TC_BM = 128;
 constexpr int TC_BN = 256;
