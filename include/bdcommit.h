@@ -103,13 +103,17 @@ typedef struct {
  *                   e2m1(code) * e4m3(block scale) * scale[v].
  *   For BD_BF16 / BD_E4M3 / BD_NVFP4 the pointer must be 16-byte aligned and
  *   ld * element size (bytes for BD_NVFP4) a multiple of 16.
- *   Both quantised formats decode exactly to bf16. On the CTA-pair LM-head
- *   kernel (windows up to 8192 positions) the codes are decoded inside the
- *   kernel, so the workspace holds no bf16 copy of the head, when a row holds
- *   at least 16 bytes of codes and, for BD_NVFP4, `block_scale` is 16-byte
- *   aligned with block_ld a multiple of 16; otherwise the head is first
- *   decoded into a bf16 copy in the workspace (bd_workspace_size accounts
- *   for it). The environment variable BD_FUSED_DECODE=0 forces the copy. */
+ *   Both quantised formats decode exactly to bf16. A BD_E4M3 head on the
+ *   commit step is read as it is by the 8-bit tensor path of the CTA-pair
+ *   kernel at every window size (see bd_exec.variant), with no copy. For the
+ *   other cases, on the CTA-pair kernel (windows up to 8192 positions) the
+ *   codes are decoded inside the kernel, so the workspace holds no bf16 copy
+ *   of the head, when a row holds at least 16 bytes of codes and, for
+ *   BD_NVFP4, `block_scale` is 16-byte aligned with block_ld a multiple of
+ *   16; otherwise the head is first decoded into a bf16 copy in the
+ *   workspace (bd_workspace_size accounts for it). The environment variables
+ *   BD_E4M3_SPLIT=0 (no 8-bit path) and BD_FUSED_DECODE=0 (no decode in the
+ *   kernel) select the other paths. */
 typedef struct {
   const void* data;
   int32_t dtype;

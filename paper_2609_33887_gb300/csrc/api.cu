@@ -27,6 +27,7 @@ struct DevCtx {
   bool ready = false;
   int sm_count = 0;
   int pairs = 0;               // CTA pairs of the pair kernel that fit on the device at once
+  int quads = 0;               // ... clusters of two pairs
   uint32_t* status = nullptr;  // device status word (bd::DEV_* bits)
   void* ws = nullptr;          // library-owned workspace
   size_t ws_bytes = 0;
@@ -58,12 +59,14 @@ int device_ctx(DevCtx** out, int* dev_out = nullptr) {
         return BD_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
-    int pairs = 0;
-    if (bd::lmhead_pair_max_pairs(sms, &pairs) != cudaSuccess) return BD_ERR_CUDA;
+    int pairs = 0, quads = 0;
+    if (bd::lmhead_pair_max_clusters(sms, 1, &pairs) != cudaSuccess) return BD_ERR_CUDA;
+    if (bd::lmhead_pair_max_clusters(sms, 2, &quads) != cudaSuccess) return BD_ERR_CUDA;
     if (cudaMalloc(&c.status, 256) != cudaSuccess) return BD_ERR_CUDA;
     if (cudaMemset(c.status, 0, 256) != cudaSuccess) return BD_ERR_CUDA;
     c.sm_count = sms;
     c.pairs = pairs;
+    c.quads = quads;
     c.ready = true;
   }
   *out = &c;
@@ -227,13 +230,20 @@ int64_t head_operand_bytes(const Call& c) {
   return c.d * esize(c.wdt);
 }
 
-BandPlan make_plan(const Call& c, int sm_count, int pairs) {
+BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
   BandPlan p;
+  p.mc = 1;
   if (c.pair) {
     p.BM = 0;  // token groups derived from N on the device
     p.BN = 256;
     p.G = pairs;
     p.cpu = 2;
+    // heads staged by TMA as they are (bf16, the 8-bit paths): clusters of
+    // two pairs that share every head tile (BD_PAIR_MC=1: single pairs)
+    if (!c.fused && env_int("BD_PAIR_MC", 2, 1, 2) == 2 && quads > 0) {
+      p.mc = 2;
+      p.G = quads;
+    }
   } else if (c.tc) {
     p.BM = bd::TC_BM;
     p.BN = bd::TC_BN;
@@ -385,12 +395,12 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
                                      ld_rows, 128, 16 * (i + 1), true))
           return BD_ERR_CUDA;
       }
-      if (!encode_u8_2d(&tmB, weight->data, c.d, c.V, c.ldw, 128, 128, true)) return BD_ERR_CUDA;
+      if (!encode_u8_2d(&tmB, weight->data, c.d, c.V, c.ldw, 128, 64, true)) return BD_ERR_CUDA;
     } else if (c.pair) {
       // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
       for (int i = 0; i < 8; ++i)
         if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 16 * (i + 1))) return BD_ERR_CUDA;
-      if (!c.fused && !encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 128)) return BD_ERR_CUDA;
+      if (!c.fused && !encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 64)) return BD_ERR_CUDA;
     } else {
       if (!encode_bf16_2d(&tmA, rows, c.d, c.P, ld_rows, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
       if (!encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, bd::TC_BK, bd::TC_BN)) return BD_ERR_CUDA;
@@ -564,7 +574,7 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const
   if (check_args(hidden, weight, mask_state, tau_grid, 0, &c) != BD_OK) return 0;
   DevCtx* ctx = nullptr;
   if (device_ctx(&ctx) != BD_OK) return 0;
-  return make_layout(c, make_plan(c, ctx->sm_count, ctx->pairs)).total;
+  return make_layout(c, make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads)).total;
 }
 
 int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
@@ -594,7 +604,7 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd
   DevCtx* ctx = nullptr;
   rc = device_ctx(&ctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs);
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads);
   const Layout lay = make_layout(c, plan);
 
   uint8_t* ws = nullptr;
@@ -649,7 +659,7 @@ int bd_lmhead_partials(const bd_hidden* hidden, const bd_weight* shard, int64_t 
   DevCtx* ctx = nullptr;
   rc = device_ctx(&ctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs);
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads);
   const Layout lay = make_layout(c, plan);
   uint8_t* ws = nullptr;
   if (exec && exec->workspace) {
@@ -790,6 +800,7 @@ struct StaticCtx {
   bool ready = false;
   int sm_count = 0;
   int pairs = 0;
+  int quads = 0;
   uint8_t* scratch = nullptr;  // device address of g_static_scratch on this device
 };
 StaticCtx g_static[MAX_DEVICES];
@@ -826,8 +837,9 @@ int static_ctx(StaticCtx** out) {
         return BD_ERR_CUDA;
       g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     }
-    int pairs = 0;
-    if (bd::lmhead_pair_max_pairs(sms, &pairs) != cudaSuccess) return BD_ERR_CUDA;
+    int pairs = 0, quads = 0;
+    if (bd::lmhead_pair_max_clusters(sms, 1, &pairs) != cudaSuccess) return BD_ERR_CUDA;
+    if (bd::lmhead_pair_max_clusters(sms, 2, &quads) != cudaSuccess) return BD_ERR_CUDA;
     void* p = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&p, g_static_scratch);
     if (e != cudaSuccess || p == nullptr) return e == cudaSuccess ? BD_ERR_CUDA : cuda_status(e);
@@ -836,6 +848,7 @@ int static_ctx(StaticCtx** out) {
     if (cudaMemset(s.scratch + STATIC_STATUS_OFFSET, 0, sizeof(uint32_t)) != cudaSuccess) return BD_ERR_CUDA;
     s.sm_count = sms;
     s.pairs = pairs;
+    s.quads = quads;
     s.ready = true;
   }
   *out = &s;
@@ -858,7 +871,7 @@ extern "C" int bd_commit_step_static(const bd_hidden* hidden, const bd_weight* w
   StaticCtx* sctx = nullptr;
   rc = static_ctx(&sctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(c, sctx->sm_count, sctx->pairs);
+  const BandPlan plan = make_plan(c, sctx->sm_count, sctx->pairs, sctx->quads);
   const Layout lay = make_layout(c, plan);
   if (lay.total > BD_STATIC_SCRATCH_BYTES) return BD_ERR_WORKSPACE;
 
@@ -1027,7 +1040,7 @@ size_t bd_verify_workspace_size(const bd_hidden* hidden, const bd_weight* weight
   if (check_verify(hidden, weight, draft, eps, 0, &vc) != BD_OK) return 0;
   DevCtx* ctx = nullptr;
   if (device_ctx(&ctx) != BD_OK) return 0;
-  return make_verify_layout(vc.c, make_plan(vc.c, ctx->sm_count, ctx->pairs)).total;
+  return make_verify_layout(vc.c, make_plan(vc.c, ctx->sm_count, ctx->pairs, ctx->quads)).total;
 }
 
 int bd_verify_step(const bd_hidden* hidden, const bd_weight* weight, const bd_draft* draft, const bd_eps_grid* eps,
@@ -1049,7 +1062,7 @@ int bd_verify_step(const bd_hidden* hidden, const bd_weight* weight, const bd_dr
   DevCtx* ctx = nullptr;
   rc = device_ctx(&ctx);
   if (rc != BD_OK) return rc;
-  const BandPlan plan = make_plan(vc.c, ctx->sm_count, ctx->pairs);
+  const BandPlan plan = make_plan(vc.c, ctx->sm_count, ctx->pairs, ctx->quads);
   const VerifyLayout lay = make_verify_layout(vc.c, plan);
   uint8_t* ws = nullptr;
   if (exec && exec->workspace) {

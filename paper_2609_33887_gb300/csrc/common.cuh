@@ -54,6 +54,12 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // ceil(units / G) * (ceil(n_vt / gv) + 1/2) (half a v-tile for each unit's
 // start and finish). N is only known on the device, so kernels recompute the
 // plan from it.
+//
+// A runner may hold MC consecutive m-tiles of one unit at once (the pair
+// kernel's 4-CTA clusters: two CTA pairs, one m-tile each, sharing every
+// head tile through multicast loads); units, bands and the rules above then
+// count runner m-tiles of MC m-tiles (a missing last m-tile is computed on
+// zero rows and written nowhere).
 // -------------------------------------------------------------------------
 struct BandPlan {
   int BM;         // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
@@ -64,6 +70,7 @@ struct BandPlan {
   int cpu;        // CTAs per unit: each writes its own partial, so a part has cpu slots
   int vt_kb;      // KiB of head per v-tile (BN rows as the kernel reads them)
   int row_bytes;  // bytes of one packed token row as the kernel reads it
+  int mc;         // m-tiles a runner holds at once (1, or 2 for 4-CTA clusters)
 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
@@ -80,15 +87,22 @@ __host__ __device__ __forceinline__ int plan_bm(const BandPlan& p, int n_rows) {
   return p.BM > 0 ? p.BM : pair_group_rows(n_rows);
 }
 
+__host__ __device__ __forceinline__ int plan_mc(const BandPlan& p) { return p.mc > 1 ? p.mc : 1; }
+
+// Runner m-tiles (of plan_mc m-tiles each) for N rows; 0 without rows.
+__host__ __device__ __forceinline__ int plan_runner_mts(const BandPlan& p, int n_rows) {
+  return n_rows > 0 ? cdiv(cdiv(n_rows, plan_bm(p, n_rows)), plan_mc(p)) : 0;
+}
+
 // Packed rows up to this size are one band.
 constexpr double ROWS_ONE_BAND = 64.0 * 1024 * 1024;
 
-// m-tiles per band (all bands but the last are full): all n_mt when their
-// rows fit ROWS_ONE_BAND, else the integer nearest sqrt(G * head tile bytes /
-// m-tile bytes), at least 1
+// runner m-tiles per band (all bands but the last are full): all n_mt when
+// their rows fit ROWS_ONE_BAND, else the integer nearest sqrt(G * head tile
+// bytes / runner m-tile bytes), at least 1
 __host__ __device__ __forceinline__ int plan_gm(const BandPlan& p, int bm, int n_mt) {
   if (p.GM > 0) return p.GM;
-  const double tile = static_cast<double>(bm) * (p.row_bytes > 0 ? p.row_bytes : 1);
+  const double tile = static_cast<double>(bm) * plan_mc(p) * (p.row_bytes > 0 ? p.row_bytes : 1);
   if (n_mt * tile <= ROWS_ONE_BAND) return n_mt > 0 ? n_mt : 1;
   const int g = static_cast<int>(sqrt(static_cast<double>(p.G) * p.vt_kb * 1024.0 / tile) + 0.5);
   return g < 1 ? 1 : g;
@@ -136,17 +150,17 @@ __device__ __forceinline__ int plan_gv_warp(const BandPlan& p, int n_mt) {
 
 // Number of partial slots of every compacted row.
 __host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int /*row*/) {
-  const int n_mt = cdiv(n_rows, plan_bm(p, n_rows));
-  return plan_gv(p, n_mt) * p.cpu;
+  const int n_mt = plan_runner_mts(p, n_rows);
+  return plan_gv(p, n_mt > 0 ? n_mt : 1) * p.cpu;
 }
 
 // Iterates the (m-tile, v-tile range) units of unit-runner `runner` (a CTA,
-// or a CTA pair) under the plan.
+// a CTA pair, or a cluster of pairs) under the plan.
 struct TileIter {
   int runner, G;
-  int n_mt, gm_full, gv, n_vt;
+  int n_mt, gm_full, gv, n_vt, mc;
   int64_t u, n_units;
-  int m_tile;  // current m-tile
+  int m_tile;  // current m-tile (the first of the runner's mc m-tiles)
   int part;    // vocabulary part of the current unit
   int vt, vt_end;
 
@@ -156,7 +170,8 @@ struct TileIter {
     G = plan.G;
     n_vt = plan.n_vt;
     const int bm = plan_bm(plan, n_rows);
-    n_mt = n_rows > 0 ? cdiv(n_rows, bm) : 0;
+    mc = plan_mc(plan);
+    n_mt = plan_runner_mts(plan, n_rows);
     gm_full = plan_gm(plan, bm, n_mt);
     gv = parts;
     n_units = static_cast<int64_t>(n_mt) * gv;
@@ -176,7 +191,7 @@ struct TileIter {
     const int m0 = b * gm_full;
     const int gm = n_mt - m0 < gm_full ? n_mt - m0 : gm_full;
     part = i / gm;
-    m_tile = m0 + i % gm;
+    m_tile = (m0 + i % gm) * mc;
     vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
     vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
     return true;
@@ -598,6 +613,18 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const void* tmap,
       "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint"
       " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(mbar), "l"(policy)
+      : "memory");
+}
+
+// The same load multicast to the CTAs of `cta_mask` (same CTA-relative
+// address in each); each destination's bytes are counted on the mbarrier at
+// mbar's offset in that destination's pair-issuing (even) CTA.
+__device__ __forceinline__ void tma_load_2d_pair_mc(uint32_t dst, const void* tmap, uint32_t mbar, int x, int y,
+                                                    uint16_t cta_mask, uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.multicast::cluster.cta_group::2"
+      ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5, %6;" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(mbar), "h"(cta_mask), "l"(policy)
       : "memory");
 }
 

@@ -113,8 +113,8 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // the CTA holding the last position knows N: it writes N and the plan's
     // vocabulary parts for it into the header the later kernels read
     const int N = prefix + local_total;
-    const int n_mt = N > 0 ? cdiv(N, plan_bm(plan, N)) : 1;
-    const int gv = plan_gv_warp(plan, n_mt);
+    const int n_mt = plan_runner_mts(plan, N);
+    const int gv = plan_gv_warp(plan, n_mt > 0 ? n_mt : 1);
     if (lane == 0) {
       n_rows[0] = N;
       n_rows[1] = gv;
@@ -136,6 +136,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
       float amax = 0.f;
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -155,6 +156,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const float up = __uint_as_float(static_cast<uint32_t>(sh + 127) << 23);  // 2^s, exact
       __half* dst = reinterpret_cast<__half*>(hc) + static_cast<int64_t>(prefix + i) * ldc;
       uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -192,6 +194,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
       float amax = 0.f;
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -209,6 +212,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const float up = __uint_as_float(static_cast<uint32_t>(sh + 127) << 23);  // 2^s, exact
       uint8_t* dh = hq + static_cast<int64_t>(prefix + i) * ldc;
       uint8_t* dl = lq + static_cast<int64_t>(prefix + i) * ldc;
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -255,6 +259,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
       float amax = 0.f;
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -269,6 +274,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       for (int o = 16; o > 0; o >>= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
       const float inv = amax > 0.f ? __fdiv_rn(448.f, amax) : 0.f;
       uint8_t* dst = hq + static_cast<int64_t>(prefix + i) * ldc;
+#pragma unroll 4
       for (int v = lane; v < nvec; v += 32) {
         const uint4 q = __ldg(s4 + v);
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
@@ -297,6 +303,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     __nv_bfloat16* dst = hc + static_cast<int64_t>(prefix + i) * ldc;
     const uint4* s4 = reinterpret_cast<const uint4*>(src);
     uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll 4
     for (int v = lane; v < nvec; v += 32) d4[v] = __ldg(s4 + v);
     for (int e = nvec * 8 + lane; e < d; e += 32) dst[e] = src[e];
   }
@@ -344,7 +351,8 @@ __global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restr
     draft_row[r] = i < n_draft ? draft[q * n_draft + i] : -1;
   }
   if (blockIdx.x == 0 && threadIdx.x < 32) {  // N and the plan's vocabulary parts for it
-    const int gv = plan_gv_warp(plan, R > 0 ? cdiv(R, plan_bm(plan, R)) : 1);
+    const int n_mt = plan_runner_mts(plan, R);
+    const int gv = plan_gv_warp(plan, n_mt > 0 ? n_mt : 1);
     if (threadIdx.x == 0) {
       n_rows[0] = R;
       n_rows[1] = gv;

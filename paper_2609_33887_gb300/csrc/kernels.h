@@ -80,8 +80,9 @@ cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, con
 
 // a1+a2 on a CTA pair (tcgen05 cta_group::2), vocabulary on the MMA M side.
 // tmH.m[i] describes hc [P, d] bf16 with 64-column boxes of 16 * (i + 1) rows
-// (one per possible half token group), tmW the head [V, d] bf16 with 64 x 128
-// boxes. plan.G = CTA pairs, plan.BM = 0, plan.cpu = 2.
+// (one per possible half token group), tmW the head [V, d] bf16 with 64 x 64
+// boxes (64 rows: half of a CTA's head rows, see the kernel). plan.G = runners
+// (clusters of plan.mc CTA pairs), plan.BM = 0, plan.cpu = 2.
 struct PairTokenMaps {
   CUtensorMap m[8];
 };
@@ -99,7 +100,8 @@ struct PairQuantMaps {
   CUtensorMap scales;
 };
 size_t pair_smem_bytes();
-cudaError_t lmhead_pair_max_pairs(int sm_count, int* pairs);
+// CTA-pair clusters of mc pairs (clusters of 2 * mc CTAs) that fit on the device at once.
+cudaError_t lmhead_pair_max_clusters(int sm_count, int mc, int* clusters);
 // hf: HF_BF16 (tmW describes the bf16 head; tmQ unused, may be null) or
 // HF_E4M3 / HF_NVFP4 (tmQ describes the codes, and the NVFP4 block scales;
 // tmW unused). E4M3 and NVFP4 need the TcArgs row scale wscale.

@@ -1,5 +1,5 @@
 // Host check of the LM-head work plan (common.cuh): for each case given on
-// the command line as "n_rows BM GM vt_kb row_bytes G n_vt cpu", every (m-tile,
+// the command line as "n_rows BM GM vt_kb row_bytes G n_vt cpu mc", every (m-tile,
 // v-tile) pair is taken by exactly one unit, the part indices stay below the
 // partial slots the merge reads, and the busiest runner's v-tiles are
 // reported against the even share. Prints one line per case:
@@ -11,7 +11,7 @@
 #include "common.cuh"
 
 int main(int argc, char** argv) {
-  for (int i = 1; i + 7 < argc; i += 8) {
+  for (int i = 1; i + 8 < argc; i += 9) {
     bd::BandPlan p;
     const int n_rows = std::atoi(argv[i]);
     p.BM = std::atoi(argv[i + 1]);
@@ -21,8 +21,11 @@ int main(int argc, char** argv) {
     p.G = std::atoi(argv[i + 5]);
     p.n_vt = std::atoi(argv[i + 6]);
     p.cpu = std::atoi(argv[i + 7]);
+    p.mc = std::atoi(argv[i + 8]);
     const int bm = bd::plan_bm(p, n_rows);
-    const int n_mt = n_rows > 0 ? bd::cdiv(n_rows, bm) : 0;
+    const int n_mt = n_rows > 0 ? bd::cdiv(n_rows, bm) : 0;  // m-tiles
+    const int n_rmt = bd::plan_runner_mts(p, n_rows);        // runner m-tiles (mc m-tiles each)
+    const int mc = bd::plan_mc(p);
     std::vector<int> cover(static_cast<size_t>(n_mt) * p.n_vt, 0);
     const int slots = n_rows > 0 ? bd::slots_of_row(p, n_rows, 0) : 0;
     const char* fail = nullptr;
@@ -30,14 +33,16 @@ int main(int argc, char** argv) {
     for (int r = 0; r < p.G && !fail; ++r) {
       bd::TileIter it;
       // the parts the compaction kernel stores beside N (plan_gv_warp: the same rule)
-      it.init(p, n_rows, bd::plan_gv(p, n_mt > 0 ? n_mt : 1), r);
+      it.init(p, n_rows, bd::plan_gv(p, n_rmt > 0 ? n_rmt : 1), r);
       long long load = 0;
       while (it.next_unit()) {
-        if (it.m_tile < 0 || it.m_tile >= n_mt) fail = "m-tile out of range";
+        if (it.m_tile < 0 || it.m_tile >= n_mt || it.m_tile % mc != 0) fail = "m-tile out of range";
         else if ((it.part + 1) * p.cpu > slots) fail = "part beyond the partial slots";
         else if (it.vt < 0 || it.vt_end > p.n_vt || it.vt >= it.vt_end) fail = "empty or out-of-range v-tiles";
         if (fail) break;
-        for (int v = it.vt; v < it.vt_end; ++v) ++cover[static_cast<size_t>(it.m_tile) * p.n_vt + v];
+        // the runner's mc m-tiles (one beyond the last is computed on no rows)
+        for (int q = 0; q < mc && it.m_tile + q < n_mt; ++q)
+          for (int v = it.vt; v < it.vt_end; ++v) ++cover[static_cast<size_t>(it.m_tile + q) * p.n_vt + v];
         load += it.vt_end - it.vt;
       }
       if (load > max_load) max_load = load;
@@ -48,7 +53,7 @@ int main(int argc, char** argv) {
       std::printf("FAIL %s\n", fail);
     } else {
       std::printf("ok %d %d %d %lld %.3f %d\n", n_mt, slots / (p.cpu > 0 ? p.cpu : 1), slots, max_load,
-                  static_cast<double>(n_mt) * p.n_vt / p.G, bd::plan_gm(p, bm, n_mt));
+                  static_cast<double>(n_rmt) * p.n_vt / p.G, bd::plan_gm(p, bm, n_rmt));
     }
   }
   return 0;

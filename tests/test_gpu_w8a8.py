@@ -160,3 +160,19 @@ def test_w8a8_lossless_rows_match_the_exact_step():
     rep = compare(out, oracle_on_workload(wl), wl.tau, "e4m3", wl.cfg.block_len, wl.cfg.n_slots)
     assert rep.ok(), rep.failures
     assert rep.n_live > 0
+
+
+def test_w8a8_largest_window_sampled_blocks():
+    """The largest window (256 x 8 x 64, d = 5120, more than 8192 positions:
+    205 token groups of 256, several bands of the plan) with W8A8, on sampled
+    whole blocks including those of the first and last compacted rows."""
+    wl = generate(B256X8X64_E4M3)
+    cfg = wl.cfg
+    act = np.repeat((wl.block_flags.numpy() & 1) != 0, cfg.block_len)
+    rows = np.flatnonzero((wl.pos_masked.numpy() != 0) & act)
+    rng = np.random.default_rng(8)
+    blocks = sorted({int(rows[0]) // cfg.block_len, int(rows[-1]) // cfg.block_len,
+                     int(rows[len(rows) // 2]) // cfg.block_len}
+                    | set(rng.choice(cfg.n_blocks, size=5, replace=False).tolist()))
+    _, rep = check(wl, blocks=blocks)
+    assert rep.n_live > 0

@@ -40,26 +40,31 @@ def run_cases(exe, cases):
     return [l.split() for l in out if l.strip()]
 
 
-PAIR_G, SMS = 76, 152
-# (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu); vt_kb = KiB of head per
-# v-tile, row_bytes = bytes of a packed token row, as the kernels read them
+PAIR_G, QUAD_G, SMS = 76, 38, 152
+# (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu, mc); vt_kb = KiB of head per
+# v-tile, row_bytes = bytes of a packed token row, as the kernels read them;
+# mc = m-tiles a runner holds (2: clusters of two CTA pairs)
 CASES = [
-    # pair kernel (BM = 0: token groups from N; GM = 0: bands by the square-root rule)
-    (294, 0, 0, 1024, 4096, PAIR_G, 594, 2),       # 8 x 2 x 32, d = 2048, bf16
-    (2048, 0, 0, 1024, 4096, PAIR_G, 614, 2),      # 32 x 4 x 32
-    (8191, 0, 0, 2048, 8192, PAIR_G, 594, 2),      # 64 x 4 x 64, d = 4096
-    (8200, 0, 0, 2048, 8192, PAIR_G, 594, 2),      # one row into another group
-    (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2),    # 256 x 8 x 64, d = 5120, E4M3 head, two-term rows
-    (32, 0, 0, 64, 1024, PAIR_G, 16, 2),           # the tiny window
-    (1, 0, 0, 1, 16, PAIR_G, 1, 2),                # one row, one v-tile
-    (257, 0, 0, 1024, 4096, 3, 7, 2),              # few runners
-    (5000, 0, 7, 1024, 4096, PAIR_G, 100, 2),      # a fixed band size
+    # pair kernel in clusters of two pairs (BM = 0: token groups from N; GM = 0: bands by rule)
+    (294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2),       # 8 x 2 x 32, d = 2048, bf16
+    (2048, 0, 0, 1024, 4096, QUAD_G, 614, 2, 2),      # 32 x 4 x 32
+    (8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),      # 64 x 4 x 64, d = 4096
+    (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),      # one row into another group (33 groups: odd)
+    (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2),    # 256 x 8 x 64, d = 5120, E4M3 head, two-term rows
+    (32, 0, 0, 64, 1024, QUAD_G, 16, 2, 2),           # the tiny window
+    (1, 0, 0, 1, 16, QUAD_G, 1, 2, 2),                # one row, one v-tile
+    (257, 0, 0, 1024, 4096, 3, 7, 2, 2),              # few runners
+    (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2),      # a fixed band size
+    # single CTA pairs (quantised heads decoded in the kernel)
+    (294, 0, 0, 1024, 4096, PAIR_G, 594, 2, 1),
+    (8191, 0, 0, 2048, 8192, PAIR_G, 594, 2, 1),
+    (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1),
     # one-CTA kernel (BM = 128) and the SIMT kernel (BM = 32, 64-entry v-tiles)
-    (8191, 128, 0, 2048, 8192, SMS, 594, 1),
-    (52429, 128, 0, 2560, 10240, SMS, 614, 1),
-    (294, 32, 0, 512, 4096, 2 * SMS, 2374, 1),
-    (32, 32, 0, 64, 1024, 2 * SMS, 64, 1),
-    (5, 32, 0, 1, 100, 2 * SMS, 3, 1),
+    (8191, 128, 0, 2048, 8192, SMS, 594, 1, 1),
+    (52429, 128, 0, 2560, 10240, SMS, 614, 1, 1),
+    (294, 32, 0, 512, 4096, 2 * SMS, 2374, 1, 1),
+    (32, 32, 0, 64, 1024, 2 * SMS, 64, 1, 1),
+    (5, 32, 0, 1, 100, 2 * SMS, 3, 1, 1),
 ]
 
 
@@ -77,18 +82,20 @@ def test_plan_covers_every_tile_once_with_balanced_runners(plan_check):
 
 
 def test_plan_without_rows(plan_check):
-    (r,) = run_cases(plan_check, [(0, 0, 0, 1024, 4096, PAIR_G, 594, 2)])
+    (r,) = run_cases(plan_check, [(0, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2)])
     assert r[0] == "ok" and int(r[1]) == 0
 
 
 def test_band_size(plan_check):
     # rows up to 64 MiB are one band: the 64 x 4 x 64 window's 32 groups of
     # 256 rows x 8 KiB (64 MiB), the head streamed once; beyond that GM =
-    # round(sqrt(G * head tile bytes / m-tile bytes)): 1.25 MiB E4M3 head tiles
-    # and 2.5 MiB two-term groups (256 x 8 x 64) give sqrt(38) -> 6, and one row
-    # past 64 MiB gives sqrt(76) -> 9; a fixed GM is kept
-    rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, PAIR_G, 594, 2),
-                                  (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2),
-                                  (8200, 0, 0, 2048, 8192, PAIR_G, 594, 2),
-                                  (5000, 0, 7, 1024, 4096, PAIR_G, 100, 2)])
-    assert [int(r[6]) for r in rows] == [32, 6, 9, 7]
+    # round(sqrt(G * head tile bytes / runner m-tile bytes)) runner m-tiles:
+    # 1.25 MiB E4M3 head tiles and 2 x 2.5 MiB two-term groups on 38 clusters
+    # (256 x 8 x 64) give sqrt(9.5) -> 3, on 76 single pairs sqrt(38) -> 6; one
+    # row past 64 MiB on 38 clusters gives sqrt(19) -> 4; a fixed GM is kept
+    rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),
+                                  (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2),
+                                  (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1),
+                                  (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),
+                                  (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2)])
+    assert [int(r[6]) for r in rows] == [16, 3, 6, 4, 7]
