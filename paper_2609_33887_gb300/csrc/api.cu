@@ -239,8 +239,14 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
     p.G = pairs;
     p.cpu = 2;
     // heads staged by TMA as they are (bf16, the 8-bit paths): clusters of
-    // two pairs that share every head tile (BD_PAIR_MC=1: single pairs)
-    if (!c.fused && env_int("BD_PAIR_MC", 2, 1, 2) == 2 && quads > 0) {
+    // two pairs that share every head tile where that measured faster than
+    // single pairs on all SMs (clusters of 4 leave 8 of 152 SMs idle): windows
+    // of at most two token groups, and windows whose packed rows exceed
+    // 256 MiB (several bands: the head's L2 and DRAM re-reads dominate).
+    // BD_PAIR_MC = 1 or 2 forces the choice.
+    const int64_t rows_bytes = c.P * row_operand_bytes(c);
+    const int mc_auto = (c.P <= 512 || rows_bytes > (int64_t(256) << 20)) ? 2 : 1;
+    if (!c.fused && env_int("BD_PAIR_MC", mc_auto, 1, 2) == 2 && quads > 0) {
       p.mc = 2;
       p.G = quads;
     }

@@ -330,3 +330,26 @@ def test_full_size_e4m3_head_decoded_in_the_pair_kernel(monkeypatch):
     wl = generate(B256X8X64_E4M3)
     _, _, rep = check(wl, variant=3, blocks=_sample_with_edges(wl, 2, seed=6))
     assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("mc", ["1", "2"])
+@pytest.mark.parametrize("name", ["bf16_5mt_ktail", "bf16_g294", "e4m3", "bf16_L64"])
+def test_pair_kernel_with_and_without_clusters_of_two_pairs(name, mc, monkeypatch):
+    # BD_PAIR_MC forces single CTA pairs (1) or clusters of two pairs sharing
+    # each head tile by multicast (2). bf16_5mt_ktail: 3 token groups of 224
+    # rows (an odd count: the second pair of the last cluster holds no rows)
+    # and a K tail; bf16_g294: two groups; e4m3: the 8-bit path; bf16_L64:
+    # blocks of 64 positions and 16 thresholds
+    monkeypatch.setenv("BD_PAIR_MC", mc)
+    _, _, rep = check(generate(SMALL[name]), variant=3)
+    assert rep.n_live > 0
+
+
+def test_clusters_of_two_pairs_on_many_bands(monkeypatch):
+    # forced clusters and bands of one runner m-tile: every unit boundary of
+    # the plan with multicast head tiles, 9 token groups (odd)
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PLAN_GM", "1")
+    wl = generate(scaled(B32X4X32_TIED, n_seq=16, n_slots=4, block_len=64, d=256, V=3000, mask_frac=0.55))
+    _, _, rep = check(wl, variant=3)
+    assert rep.n_live > 2048
