@@ -118,6 +118,9 @@ EXTRA_CONFIGS = (
     dataclasses.replace(B8X2X32_BF16, name="b8x2x32_d2048_v151936_nvfp4", weight_dtype="nvfp4"),
     # the 8-bit levers on the same window: an E4M3 head (W8A16 and W8A8)
     dataclasses.replace(B8X2X32_BF16, name="b8x2x32_d2048_v151936_e4m3", weight_dtype="e4m3"),
+    # a quarter of the largest window (64 of its 256 sequences, the same head): the same LM-head plan
+    # regime (clusters of two pairs, several bands) at a size multi-pass profiler captures can hold
+    dataclasses.replace(B256X8X64_E4M3, name="b64x8x64_d5120_v157184_e4m3", n_seq=64),
 )
 
 
