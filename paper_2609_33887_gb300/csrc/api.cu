@@ -263,6 +263,8 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
   }
   // bands: GM derived on the device from the head and row bytes (0), or fixed
   p.GM = env_int("BD_PLAN_GM", 0, 0, 1 << 20);
+  p.gv_fixed = env_int("BD_PLAN_GV", 0, 0, 1 << 20);
+  p.rr = env_int("BD_PLAN_RR", 0, 0, 1);
   p.n_vt = static_cast<int>((c.V + p.BN - 1) / p.BN);
   p.vt_kb = static_cast<int>(std::max<int64_t>(1, int64_t(p.BN) * head_operand_bytes(c) / 1024));
   p.row_bytes = static_cast<int>(std::min<int64_t>(row_operand_bytes(c), int64_t(1) << 30));

@@ -34,43 +34,47 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // Work plan of the LM-head kernels.
 //
 // The N compacted rows are cut into m-tiles of BM rows (token groups of the
-// pair kernel) and the vocabulary into v-tiles of BN entries, split into gv
-// contiguous parts of (nearly) equal length. A unit of work is one (m-tile,
-// part): a runner (a CTA, or a CTA pair) walks the part's v-tiles with the
-// m-tile's rows and leaves one partial (max, sum of exponentials, argmax) per
-// row in slot `part` (times the CTAs per unit) of the partial arrays.
+// pair kernel) and the vocabulary into v-tiles of BN entries. A runner (a CTA,
+// a CTA pair, or a cluster of pairs) holds MC consecutive m-tiles at once
+// (the pair kernel's 4-CTA clusters: two CTA pairs, one m-tile each, sharing
+// every head tile through multicast loads); "m-tiles" below count runner
+// m-tiles of MC m-tiles (a missing last m-tile is computed on zero rows and
+// written nowhere).
 //
-// Units are numbered band by band: a band holds at most GM consecutive
-// m-tiles, and inside a band the units go part by part (all m-tiles of part
-// 0, then part 1, ...). Runner c takes units c, c + G, c + 2G, ...: the G
-// units in flight at any time are consecutive, about GM m-tiles times G / GM
-// parts, so every head tile is fetched from HBM about once per band and
-// re-read from L2 by the band's m-tiles, and each runner re-reads its
-// m-tile's rows from L2 at every v-tile. A window whose packed rows fit
-// ROWS_ONE_BAND bytes is one band (the head is streamed once); a larger one
-// keeps about GM m-tiles of rows plus G / GM head tiles in L2 at a time, and
-// GM = sqrt(G * head tile bytes / m-tile bytes) minimises that sum. gv
-// minimises the makespan
-// ceil(units / G) * (ceil(n_vt / gv) + 1/2) (half a v-tile for each unit's
-// start and finish). N is only known on the device, so kernels recompute the
-// plan from it.
+// The m-tiles are cut into bands of GM (the last band may be smaller) and the
+// vocabulary into gv contiguous parts of (nearly) equal length. A part of a
+// band is the gm units (m-tile, part) that share the same head slice; a unit
+// leaves one partial (max, sum of exponentials, argmax) per row in slot `part`
+// (times the CTAs per unit) of the partial arrays. Parts, ordered band by
+// band, are packed whole into rounds of G units (G runners): a part that does
+// not fit what is left of a round starts the next round, and runner c takes
+// slot c of every round (a slot past the round's parts is idle). All m-tiles
+// of a part therefore run at the same time, so its head slice is fetched from
+// HBM once and re-read from L2 by the others; a part split across two rounds
+// (an earlier round-robin plan) was fetched twice, a round apart.
 //
-// A runner may hold MC consecutive m-tiles of one unit at once (the pair
-// kernel's 4-CTA clusters: two CTA pairs, one m-tile each, sharing every
-// head tile through multicast loads); units, bands and the rules above then
-// count runner m-tiles of MC m-tiles (a missing last m-tile is computed on
-// zero rows and written nowhere).
+// (GM, gv): among the pairs whose makespan rounds * (2 ceil(n_vt / gv) + 1)
+// (in half v-tiles: half a v-tile for each unit's start and finish) is within
+// MAKESPAN_SLACK of the best, the fewest bands (each band streams the head
+// once), then the smaller makespan, then the smaller gv; over GM <= min(n_mt,
+// G) with GM m-tiles of rows within the in-flight budget below (they stay in
+// L2 while their parts run) and gv <= min(G, n_vt). N is only known on the
+// device: the compaction kernel evaluates the rule with one warp and stores
+// GM and gv beside N in the workspace header, which the LM-head and merge
+// kernels read.
 // -------------------------------------------------------------------------
 struct BandPlan {
   int BM;         // rows per m-tile; 0 = derived from N (token groups of the pair kernel)
   int BN;         // vocabulary entries per v-tile
-  int GM;         // m-tiles per band at most; 0 = derived (see plan_gm)
-  int G;          // units that can run at once (CTAs, or CTA pairs)
+  int GM;         // m-tiles per band when > 0 (clamped to 1..n_mt); 0 = chosen with gv
+  int G;          // runners that can run at once (CTAs, CTA pairs or clusters)
   int n_vt;       // ceil(V / BN)
   int cpu;        // CTAs per unit: each writes its own partial, so a part has cpu slots
   int vt_kb;      // KiB of head per v-tile (BN rows as the kernel reads them)
   int row_bytes;  // bytes of one packed token row as the kernel reads it
   int mc;         // m-tiles a runner holds at once (1, or 2 for 4-CTA clusters)
+  int gv_fixed;   // vocabulary parts when > 0 (clamped to 1..min(G, n_vt)), else chosen
+  int rr;         // 1: units taken round-robin (runner c: units c, c + G, ...) instead of packed rounds
 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
@@ -94,49 +98,137 @@ __host__ __device__ __forceinline__ int plan_runner_mts(const BandPlan& p, int n
   return n_rows > 0 ? cdiv(cdiv(n_rows, plan_bm(p, n_rows)), plan_mc(p)) : 0;
 }
 
-// Packed rows up to this size are one band.
-constexpr double ROWS_ONE_BAND = 64.0 * 1024 * 1024;
+// Rows of the m-tiles in flight (one band) are kept within ROWS_IN_FLIGHT
+// bytes, or ROWS_IN_FLIGHT_MANY when there are more than two rounds' worth of
+// m-tiles: over many rounds the runners drift apart, the units in flight span
+// neighbouring bands, and larger bands no longer stay in L2 (the 256 x 8 x 64
+// window read 134 GB with bands of 12 runner m-tiles, 52 GB with bands of 2).
+constexpr double ROWS_IN_FLIGHT = 64.0 * 1024 * 1024;
+constexpr double ROWS_IN_FLIGHT_MANY = 12.0 * 1024 * 1024;
+// Among (GM, gv) within this factor of the best makespan, the fewest bands win.
+constexpr double MAKESPAN_SLACK = 1.05;
 
-// runner m-tiles per band (all bands but the last are full): all n_mt when
-// their rows fit ROWS_ONE_BAND, else the integer nearest sqrt(G * head tile
-// bytes / runner m-tile bytes), at least 1
-__host__ __device__ __forceinline__ int plan_gm(const BandPlan& p, int bm, int n_mt) {
-  if (p.GM > 0) return p.GM;
-  const double tile = static_cast<double>(bm) * plan_mc(p) * (p.row_bytes > 0 ? p.row_bytes : 1);
-  if (n_mt * tile <= ROWS_ONE_BAND) return n_mt > 0 ? n_mt : 1;
-  const int g = static_cast<int>(sqrt(static_cast<double>(p.G) * p.vt_kb * 1024.0 / tile) + 0.5);
-  return g < 1 ? 1 : g;
-}
+// The packing of the parts into rounds, for n_mt m-tiles, bands of gm and gv
+// parts: nb full bands (their parts hold gm units, k1 per round) and, when
+// rem > 0, a last band whose parts hold rem units (kr per round). The full
+// bands' parts fill rounds 0..R0-1 and u0 units of round R0; f of the last
+// band's parts share round R0 (when u0 > 0), the others follow kr per round.
+struct Packing {
+  int nb, rem, k1, kr, R0, u0, f, rounds;
+};
 
-// The makespan of gv parts, in half v-tiles, packed with gv into one key:
-// the smallest key is the smallest makespan, then the fewest parts.
-__host__ __device__ __forceinline__ uint64_t plan_gv_key(const BandPlan& p, int n_mt, int gv) {
-  const uint64_t rounds = (static_cast<uint64_t>(n_mt) * gv + p.G - 1) / p.G;
-  const uint64_t cost = rounds * (2 * static_cast<uint64_t>(cdiv(p.n_vt, gv)) + 1);
-  return (cost << 10) | static_cast<uint64_t>(gv);  // gv <= G < 2^10
-}
-
-// vocabulary parts per m-tile: the makespan rule above, over 1..min(G, n_vt)
-__host__ __device__ __forceinline__ int plan_gv(const BandPlan& p, int n_mt) {
-  const int hi = p.G < p.n_vt ? p.G : p.n_vt;
-  uint64_t best = ~uint64_t(0);
-  for (int gv = 1; gv <= hi; ++gv) {
-    const uint64_t k = plan_gv_key(p, n_mt, gv);
-    best = k < best ? k : best;
+__host__ __device__ __forceinline__ Packing plan_pack(int n_mt, int G, int gm, int gv) {
+  Packing k;
+  k.nb = n_mt / gm;
+  k.rem = n_mt - k.nb * gm;
+  k.k1 = G / gm;
+  k.kr = k.rem > 0 ? G / k.rem : 0;
+  const int64_t full_parts = static_cast<int64_t>(k.nb) * gv;
+  k.R0 = static_cast<int>(full_parts / k.k1);
+  k.u0 = static_cast<int>(full_parts - static_cast<int64_t>(k.R0) * k.k1) * gm;
+  int left = k.rem > 0 ? gv : 0;
+  k.f = 0;
+  if (k.u0 > 0 && k.rem > 0) {
+    const int fit = (G - k.u0) / k.rem;
+    k.f = fit < left ? fit : left;
   }
-  return static_cast<int>(best & 1023u);
+  left -= k.f;
+  k.rounds = k.R0 + (k.u0 > 0 ? 1 : 0) + (left > 0 ? cdiv(left, k.kr) : 0);
+  return k;
+}
+
+// The makespan of (gm, gv) in half v-tiles (saturated at 2^33 - 1).
+__host__ __device__ __forceinline__ uint64_t plan_cost(const BandPlan& p, int n_mt, int gm, int gv) {
+  const Packing k = plan_pack(n_mt, p.G, gm, gv);
+  const uint64_t cost = static_cast<uint64_t>(k.rounds) * (2 * static_cast<uint64_t>(cdiv(p.n_vt, gv)) + 1);
+  return cost < (uint64_t(1) << 33) ? cost : (uint64_t(1) << 33) - 1;
+}
+
+// The choice key of (gm, gv) among those within the slack: bands, then
+// makespan, then gv (smallest wins), gm in the low bits for decoding.
+__host__ __device__ __forceinline__ uint64_t plan_key(const BandPlan& p, int n_mt, int gm, int gv, uint64_t cost) {
+  uint64_t nbands = static_cast<uint64_t>(cdiv(n_mt, gm));
+  if (nbands > 1023) nbands = 1023;
+  return (nbands << 53) | (cost << 20) | (static_cast<uint64_t>(gv) << 10) | static_cast<uint64_t>(gm);
+}
+
+// The range of band sizes the choice may take: GM if fixed; else 1..min(n_mt,
+// G) limited to ROWS_IN_FLIGHT of rows (at least 1).
+__host__ __device__ __forceinline__ void plan_gm_range(const BandPlan& p, int bm, int n_mt, int* lo, int* hi) {
+  const int top = n_mt < p.G ? n_mt : p.G;
+  if (p.GM > 0) {
+    *lo = *hi = p.GM < top ? p.GM : (top > 0 ? top : 1);
+    return;
+  }
+  const double tile = static_cast<double>(bm) * plan_mc(p) * (p.row_bytes > 0 ? p.row_bytes : 1);
+  int cap = static_cast<int>((n_mt > 2 * p.G ? ROWS_IN_FLIGHT_MANY : ROWS_IN_FLIGHT) / tile);
+  if (cap < 1) cap = 1;
+  *lo = 1;
+  *hi = top < cap ? top : cap;
+  if (*hi < 1) *hi = 1;
+}
+
+__host__ __device__ __forceinline__ void plan_gv_range(const BandPlan& p, int* lo, int* hi) {
+  const int top = p.G < p.n_vt ? p.G : p.n_vt;
+  if (p.gv_fixed > 0) {
+    *lo = *hi = p.gv_fixed < top ? p.gv_fixed : top;
+  } else {
+    *lo = 1;
+    *hi = top;
+  }
+}
+
+// (GM, gv) for n_mt runner m-tiles, sequentially (host).
+__host__ __device__ __forceinline__ void plan_choose(const BandPlan& p, int n_rows, int* gm_out, int* gv_out) {
+  const int n_mt = plan_runner_mts(p, n_rows) > 0 ? plan_runner_mts(p, n_rows) : 1;
+  int glo, ghi, vlo, vhi;
+  plan_gm_range(p, plan_bm(p, n_rows), n_mt, &glo, &ghi);
+  plan_gv_range(p, &vlo, &vhi);
+  uint64_t c_min = ~uint64_t(0);
+  for (int gm = glo; gm <= ghi; ++gm)
+    for (int gv = vlo; gv <= vhi; ++gv) {
+      const uint64_t c = plan_cost(p, n_mt, gm, gv);
+      c_min = c < c_min ? c : c_min;
+    }
+  const uint64_t c_max = static_cast<uint64_t>(static_cast<double>(c_min) * MAKESPAN_SLACK);
+  uint64_t best = ~uint64_t(0);
+  for (int gm = glo; gm <= ghi; ++gm)
+    for (int gv = vlo; gv <= vhi; ++gv) {
+      const uint64_t c = plan_cost(p, n_mt, gm, gv);
+      if (c > c_max) continue;
+      const uint64_t k = plan_key(p, n_mt, gm, gv, c);
+      best = k < best ? k : best;
+    }
+  *gm_out = static_cast<int>(best & 1023u);
+  *gv_out = static_cast<int>((best >> 10) & 1023u);
 }
 
 #ifdef __CUDACC__
-// The same choice by a whole warp, 32 candidates at a time. The kernel that
-// learns N (compaction, or the verification rows) evaluates it once and
-// stores gv beside N in the workspace header (plan_hdr[0] = N, plan_hdr[1] =
-// gv), so the LM-head and merge kernels only read it.
-__device__ __forceinline__ int plan_gv_warp(const BandPlan& p, int n_mt) {
-  const int hi = p.G < p.n_vt ? p.G : p.n_vt;
+// The same choice by a whole warp, 32 candidates at a time (the kernel that
+// learns N calls it once and stores GM and gv in the workspace header).
+__device__ __forceinline__ void plan_choose_warp(const BandPlan& p, int n_rows, int* gm_out, int* gv_out) {
+  const int n_mt = plan_runner_mts(p, n_rows) > 0 ? plan_runner_mts(p, n_rows) : 1;
+  int glo, ghi, vlo, vhi;
+  plan_gm_range(p, plan_bm(p, n_rows), n_mt, &glo, &ghi);
+  plan_gv_range(p, &vlo, &vhi);
+  const int nv = vhi - vlo + 1;
+  const int total = (ghi - glo + 1) * nv;
+  uint64_t c_min = ~uint64_t(0);
+  for (int i = static_cast<int>(threadIdx.x & 31); i < total; i += 32) {
+    const uint64_t c = plan_cost(p, n_mt, glo + i / nv, vlo + i % nv);
+    c_min = c < c_min ? c : c_min;
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t other = __shfl_xor_sync(0xffffffffu, c_min, o);
+    c_min = other < c_min ? other : c_min;
+  }
+  const uint64_t c_max = static_cast<uint64_t>(static_cast<double>(c_min) * MAKESPAN_SLACK);
   uint64_t best = ~uint64_t(0);
-  for (int gv = static_cast<int>(threadIdx.x & 31) + 1; gv <= hi; gv += 32) {
-    const uint64_t k = plan_gv_key(p, n_mt, gv);
+  for (int i = static_cast<int>(threadIdx.x & 31); i < total; i += 32) {
+    const uint64_t c = plan_cost(p, n_mt, glo + i / nv, vlo + i % nv);
+    if (c > c_max) continue;
+    const uint64_t k = plan_key(p, n_mt, glo + i / nv, vlo + i % nv, c);
     best = k < best ? k : best;
   }
 #pragma unroll
@@ -144,57 +236,96 @@ __device__ __forceinline__ int plan_gv_warp(const BandPlan& p, int n_mt) {
     const uint64_t other = __shfl_xor_sync(0xffffffffu, best, o);
     best = other < best ? other : best;
   }
-  return static_cast<int>(best & 1023u);
+  *gm_out = static_cast<int>(best & 1023u);
+  *gv_out = static_cast<int>((best >> 10) & 1023u);
 }
 #endif
 
-// Number of partial slots of every compacted row.
-__host__ __device__ __forceinline__ int slots_of_row(const BandPlan& p, int n_rows, int /*row*/) {
-  const int n_mt = plan_runner_mts(p, n_rows);
-  return plan_gv(p, n_mt > 0 ? n_mt : 1) * p.cpu;
-}
-
-// Iterates the (m-tile, v-tile range) units of unit-runner `runner` (a CTA,
-// a CTA pair, or a cluster of pairs) under the plan.
+// Iterates the units of runner `runner` under the packed plan.
 struct TileIter {
   int runner, G;
-  int n_mt, gm_full, gv, n_vt, mc;
-  int64_t u, n_units;
+  int n_mt, gm, gv, n_vt, mc, rr;
+  Packing k;
+  int round;
   int m_tile;  // current m-tile (the first of the runner's mc m-tiles)
   int part;    // vocabulary part of the current unit
   int vt, vt_end;
 
-  // n_rows and parts: the header the compaction kernel wrote (N, gv)
-  __host__ __device__ void init(const BandPlan& plan, int n_rows, int parts, int runner_index) {
+  // n_rows, bands and parts: the header the compaction kernel wrote (N, GM, gv)
+  __host__ __device__ void init(const BandPlan& plan, int n_rows, int band_mts, int parts, int runner_index) {
     runner = runner_index;
     G = plan.G;
     n_vt = plan.n_vt;
-    const int bm = plan_bm(plan, n_rows);
     mc = plan_mc(plan);
     n_mt = plan_runner_mts(plan, n_rows);
-    gm_full = plan_gm(plan, bm, n_mt);
-    gv = parts;
-    n_units = static_cast<int64_t>(n_mt) * gv;
-    u = static_cast<int64_t>(runner) - G;
+    gm = band_mts > 0 ? band_mts : 1;
+    gv = parts > 0 ? parts : 1;
+    k = plan_pack(n_mt > 0 ? n_mt : 1, G, gm, gv);
+    rr = plan.rr;
+    if (rr) k.rounds = static_cast<int>((static_cast<int64_t>(n_mt) * gv + G - 1) / G);
+    if (n_mt == 0) k.rounds = 0;
+    round = -1;
     vt = vt_end = 0;
   }
 #ifdef __CUDACC__
-  __device__ void init(const BandPlan& plan, int n_rows, int parts) { init(plan, n_rows, parts, blockIdx.x); }
+  __device__ void init(const BandPlan& plan, int n_rows, int band_mts, int parts) {
+    init(plan, n_rows, band_mts, parts, blockIdx.x);
+  }
 #endif
-  // Advances to the next unit; false when there is no more work.
-  __host__ __device__ bool next_unit() {
-    u += G;
-    if (u >= n_units) return false;
-    const int64_t band_units = static_cast<int64_t>(gm_full) * gv;
+  // Round-robin order (plan.rr): unit u = c + r G in band-major, part-major
+  // order; false past the last unit.
+  __host__ __device__ bool unit_rr(int r) {
+    const int64_t u = static_cast<int64_t>(r) * G + runner;
+    if (u >= static_cast<int64_t>(n_mt) * gv) return false;
+    const int64_t band_units = static_cast<int64_t>(gm) * gv;
     const int b = static_cast<int>(u / band_units);
     const int i = static_cast<int>(u - b * band_units);
-    const int m0 = b * gm_full;
-    const int gm = n_mt - m0 < gm_full ? n_mt - m0 : gm_full;
-    part = i / gm;
-    m_tile = (m0 + i % gm) * mc;
+    const int m0 = b * gm;
+    const int g = n_mt - m0 < gm ? n_mt - m0 : gm;
+    part = i / g;
+    m_tile = (m0 + i % g) * mc;
     vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
     vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
     return true;
+  }
+  // This runner's unit of round r: false if its slot is idle there.
+  __host__ __device__ bool unit_of(int r) {
+    if (rr) return unit_rr(r);
+    const int c = runner;
+    int64_t q = -1;  // part index in the global order (full bands first)
+    int mt = 0;
+    if (r < k.R0 || (r == k.R0 && c < k.u0)) {
+      if (c >= k.k1 * gm) return false;
+      q = static_cast<int64_t>(r) * k.k1 + c / gm;
+      if (q >= static_cast<int64_t>(k.nb) * gv) return false;
+      mt = static_cast<int>(q / gv) * gm + c % gm;
+      part = static_cast<int>(q % gv);
+    } else {
+      if (k.rem == 0) return false;
+      int j;  // part of the last band
+      if (r == k.R0 && k.u0 > 0) {
+        j = (c - k.u0) / k.rem;
+        if (j >= k.f) return false;
+        mt = k.nb * gm + (c - k.u0) % k.rem;
+      } else {
+        const int r2 = r - k.R0 - (k.u0 > 0 ? 1 : 0);
+        if (c >= k.kr * k.rem) return false;
+        j = k.f + r2 * k.kr + c / k.rem;
+        if (j >= gv) return false;
+        mt = k.nb * gm + c % k.rem;
+      }
+      part = j;
+    }
+    m_tile = mt * mc;
+    vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
+    vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
+    return true;
+  }
+  // Advances to the next unit; false when there is no more work.
+  __host__ __device__ bool next_unit() {
+    while (++round < k.rounds)
+      if (unit_of(round)) return true;
+    return false;
   }
 };
 

@@ -407,7 +407,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
 
   griddep_wait();  // the packed rows and N come from the preceding kernel
   const int n_rows = a.n_rows[0];
-  const int parts = a.n_rows[1];  // vocabulary parts of the plan (see common.cuh)
+  const int parts = a.n_rows[1];     // vocabulary parts of the plan (see common.cuh)
+  const int band_mts = a.n_rows[2];  // ... and its band size
   constexpr int BK = stage_k<HF>();
   constexpr int ACOLS = atom_cols<HF>();
   constexpr int NATOM = BK / ACOLS;
@@ -443,7 +444,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, parts, pair);
+    it.init(a.plan, n_rows, band_mts, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       const int tok0 = (it.m_tile + pp) * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
@@ -507,7 +508,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
-      it.init(a.plan, n_rows, parts, pair);
+      it.init(a.plan, n_rows, band_mts, parts, pair);
       bool ok = true;
       while (ok && it.next_unit()) {
         for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -589,7 +590,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t r = 0, rph = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, parts, pair);
+    it.init(a.plan, n_rows, band_mts, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -627,7 +628,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     constexpr int RK = raw_k<HF>();
     uint32_t r = 0, rph = 0, stage = 0, phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, parts, pair);
+    it.init(a.plan, n_rows, band_mts, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -673,7 +674,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t epi_phase = 0;
     uint32_t acc = 0, acc_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, parts, pair);
+    it.init(a.plan, n_rows, band_mts, parts, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       float m[MAX_CHUNKS], s[MAX_CHUNKS];

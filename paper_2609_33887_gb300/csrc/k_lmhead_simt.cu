@@ -76,10 +76,11 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   const int col = tid % SIMT_BN, rg = tid / SIMT_BN;  // this thread's column and row group
   griddep_wait();  // idx and N come from the preceding kernel
   const int n_rows = a.n_rows[0];
-  const int parts = a.n_rows[1];  // vocabulary parts of the plan (see common.cuh)
+  const int parts = a.n_rows[1];     // vocabulary parts of the plan (see common.cuh)
+  const int band_mts = a.n_rows[2];  // ... and its band size
 
   TileIter it;
-  it.init(a.plan, n_rows, parts);
+  it.init(a.plan, n_rows, band_mts, parts);
   while (it.next_unit()) {
     const int r0 = it.m_tile * SIMT_BM;
     if (tid < SIMT_BM) {

@@ -111,13 +111,14 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
   }
   if (p1 == P && warp == 0) {
     // the CTA holding the last position knows N: it writes N and the plan's
-    // vocabulary parts for it into the header the later kernels read
+    // vocabulary parts and band size for it into the header the later kernels read
     const int N = prefix + local_total;
-    const int n_mt = plan_runner_mts(plan, N);
-    const int gv = plan_gv_warp(plan, n_mt > 0 ? n_mt : 1);
+    int gm = 1, gv = 1;
+    plan_choose_warp(plan, N, &gm, &gv);
     if (lane == 0) {
       n_rows[0] = N;
       n_rows[1] = gv;
+      n_rows[2] = gm;
     }
   }
   if (hidden == nullptr) return;
@@ -350,12 +351,13 @@ __global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restr
     idx[r] = r;
     draft_row[r] = i < n_draft ? draft[q * n_draft + i] : -1;
   }
-  if (blockIdx.x == 0 && threadIdx.x < 32) {  // N and the plan's vocabulary parts for it
-    const int n_mt = plan_runner_mts(plan, R);
-    const int gv = plan_gv_warp(plan, n_mt > 0 ? n_mt : 1);
+  if (blockIdx.x == 0 && threadIdx.x < 32) {  // N and the plan's parts and band size for it
+    int gm = 1, gv = 1;
+    plan_choose_warp(plan, R, &gm, &gv);
     if (threadIdx.x == 0) {
       n_rows[0] = R;
       n_rows[1] = gv;
+      n_rows[2] = gm;
     }
   }
 }

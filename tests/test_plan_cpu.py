@@ -1,9 +1,10 @@
 """The LM-head work plan (csrc/common.cuh), compiled for the host and checked
 without a GPU: every (m-tile, v-tile) pair of the logits is computed by
-exactly one unit, partial-slot indices stay within what the merge reads, and
-the busiest runner carries close to an even share of the v-tiles. The cases
-are the five workloads' windows in each kernel's plan plus ragged and
-degenerate ones."""
+exactly one unit, the units of every vocabulary part run in the same round
+(so its head slice is fetched once), partial-slot indices stay within what
+the merge reads, and the busiest runner carries close to an even share of the
+v-tiles. The cases are the five workloads' windows in each kernel's plan plus
+ragged and degenerate ones."""
 
 import os
 import shutil
@@ -40,7 +41,7 @@ def run_cases(exe, cases):
     return [l.split() for l in out if l.strip()]
 
 
-PAIR_G, QUAD_G, SMS = 76, 38, 152
+PAIR_G, QUAD_G, SMS = 76, 36, 152
 # (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu, mc); vt_kb = KiB of head per
 # v-tile, row_bytes = bytes of a packed token row, as the kernels read them;
 # mc = m-tiles a runner holds (2: clusters of two CTA pairs)
@@ -87,15 +88,19 @@ def test_plan_without_rows(plan_check):
 
 
 def test_band_size(plan_check):
-    # rows up to 64 MiB are one band: the 64 x 4 x 64 window's 32 groups of
-    # 256 rows x 8 KiB (64 MiB), the head streamed once; beyond that GM =
-    # round(sqrt(G * head tile bytes / runner m-tile bytes)) runner m-tiles:
-    # 1.25 MiB E4M3 head tiles and 2 x 2.5 MiB two-term groups on 38 clusters
-    # (256 x 8 x 64) give sqrt(9.5) -> 3, on 76 single pairs sqrt(38) -> 6; one
-    # row past 64 MiB on 38 clusters gives sqrt(19) -> 4; a fixed GM is kept
+    # the chosen band sizes (runner m-tiles): the 64 x 4 x 64 window on 36
+    # clusters packs bands of 12 runner m-tiles (12 + 4) into exactly full
+    # rounds; the largest window (more than two rounds' worth of m-tiles: rows
+    # in flight within 12 MiB) 2 runner m-tiles on clusters, 4 m-tiles on 76
+    # single pairs; one row past 32 groups on clusters: 12; the 32 x 4 x 32
+    # window is one band (8 m-tiles, within 5% of the best makespan); a fixed GM
+    # is kept
     rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),
                                   (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2),
                                   (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1),
                                   (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2),
+                                  (2048, 0, 0, 1024, 4096, PAIR_G, 614, 2, 1),
                                   (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2)])
-    assert [int(r[6]) for r in rows] == [16, 3, 6, 4, 7]
+    assert [int(r[6]) for r in rows] == [12, 2, 4, 12, 8, 7]
+    # 64 x 4 x 64 on clusters: an even share exactly (16 runner m-tiles x 594 v-tiles / 36)
+    assert int(rows[0][4]) == 264
