@@ -235,6 +235,23 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight,
 size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
                          const bd_mask_state* mask_state, const bd_tau_grid* tau_grid);
 
+/* ------------------------------------------------------------ tuning knobs --
+ * Environment variables read at every call (none is needed; each changes how
+ * the work is done, never what is computed):
+ *   BD_E4M3_SPLIT=0      E4M3 heads not on the 8-bit path (see bd_exec.variant)
+ *   BD_FUSED_DECODE=0    quantised heads decoded to a bf16 copy, not in the kernel
+ *   BD_PAIR_MAX_P=n      the automatic choice takes the CTA-pair kernel for NVFP4
+ *                        heads up to n window positions (default 8192)
+ *   BD_PAIR_MC=1|2       single CTA pairs, or clusters of two pairs sharing each
+ *                        head tile by multicast (default: clusters for windows of
+ *                        at most 512 positions or more than 256 MiB of packed rows)
+ *   BD_PLAN_GM=n, BD_PLAN_GV=n   fix the work plan's band size (runner m-tiles)
+ *                        or vocabulary part count; BD_PLAN_RR=1 takes its units
+ *                        round-robin instead of in packed rounds
+ *   BD_L2_HEAD, BD_L2_ROWS = 0|1|2   L2 eviction priority (first, normal, last) of
+ *                        the head tiles and token rows (default 0 and 2)
+ *   BD_TC_STAGES=3|4     pipeline stages of the one-CTA tensor-core kernel */
+
 /* ------------------------------------------------ vocabulary-parallel split --
  * The head split by vocabulary rows over G ranks (or G calls on one device):
  * rank g holds rows [offset_g, offset_g + V_g) of W. The only exchange is
