@@ -525,14 +525,16 @@ def masked_count(wl_host):
                 (torch.repeat_interleave(wl_host.block_flags & 1, cfg.block_len) != 0)).sum())
 
 
-def launches_per_step(cfg):
-    """Library kernels per commit step: compaction + row packing, LM head, merge +
-    commit, plus the decode of an NVFP4 head where the LM-head kernel reads a
-    bf16 copy (the automatic choice decodes it inside the kernel for windows of
-    at most 8192 positions; E4M3 heads are read as they are at every size).
-    The counts reset is a runtime memset, not a kernel of the library."""
-    decoded = cfg.weight_dtype == "nvfp4" and cfg.P > 8192
-    return 3 + (1 if decoded else 0)
+def launches_per_step(r):
+    """Library kernels one commit step of runner `r` queues, as the library
+    reports them for its arguments (bd_step_kernels): compaction + row packing,
+    the decode of a quantised head where a bf16 copy is made, the LM head (one
+    launch, or two where spill pairs run beside clusters of two CTA pairs),
+    merge + commit. The counts reset is a runtime memset, not a kernel."""
+    n = r.kernels_per_step
+    if n <= 0:
+        raise RuntimeError(f"bd_step_kernels: {n}")
+    return n
 
 
 class StepRunner:
@@ -550,6 +552,9 @@ class StepRunner:
         ws_bytes = bdc.bd_workspace_size(wl.hidden, wl.weight, wl.weight_scale, wl.pos_masked, wl.block_flags,
                                          cfg.n_seq, cfg.n_slots, cfg.block_len, cfg.mask_token_id, cfg.tau)
         self.workspace = torch.empty(max(ws_bytes, 1), dtype=torch.uint8, device=dev)
+        self.kernels_per_step = bdc.bd_step_kernels(wl.hidden, wl.weight, wl.weight_scale, wl.pos_masked,
+                                                    wl.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len,
+                                                    cfg.mask_token_id, cfg.tau)
         self.tokens = torch.empty(P, dtype=torch.int32, device=dev)
         self.conf = torch.empty(P, dtype=torch.float32, device=dev)
         self.commit = torch.empty(P, dtype=torch.int32, device=dev)
@@ -660,7 +665,7 @@ def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
            "masked_positions": r.n_masked, "lmhead_us": roof["lmhead_ms_avg"] * 1e3,
            "tensor_frac": roof["tensor_view"]["frac"], "hbm_frac": roof["hbm_view"]["frac"],
            "traffic_over_algorithmic": roof["traffic_over_algorithmic"], "roofline": roof,
-           "gpu_launches_per_step": launches_per_step(cfg)}
+           "gpu_launches_per_step": launches_per_step(r)}
     del g, r
     torch.cuda.empty_cache()
     return out
@@ -887,6 +892,7 @@ def run_ours(args):
                          f"positions, {tot_t:.1f} s); head decoded to float64 once outside the timed calls"}
 
     conf_obj = config_object(cfg, wl_host, r.n_masked, world)
+    kernels = launches_per_step(r)
     del r
     torch.cuda.empty_cache()
 
@@ -922,7 +928,7 @@ def run_ours(args):
             "roofline": roof,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches_per_step(cfg) * K,
+            "gpu_launches": kernels * K,
             "clocks": clocks,
             "configs": configs or None,
             "sustained": sustained or None,

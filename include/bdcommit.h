@@ -235,6 +235,30 @@ int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight,
 size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
                          const bd_mask_state* mask_state, const bd_tau_grid* tau_grid);
 
+/* Kernels one bd_commit_step_ex call with these arguments queues (the
+ * per-threshold counts' reset is a memset, not a kernel): compaction + row
+ * packing, the decode of a quantised head where the LM head reads a bf16
+ * copy, the LM head (two launches where spill pairs run beside clusters of
+ * two CTA pairs, see BD_PAIR_SPILL), merge + commit; 0 for an empty window.
+ * Arguments as for bd_commit_step_ex (exec may be NULL; only its variant and
+ * flags are read). Returns a negative bd_status if the arguments are
+ * invalid or the device cannot run the library. Host-only: queues nothing. */
+int bd_step_kernels(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                    const bd_tau_grid* tau_grid, const bd_exec* exec);
+
+/* The work plan the LM head takes for a window of n_rows compacted rows
+ * (masked positions of active blocks), as the compaction kernel computes it
+ * on the device once N is known; host-only, for inspection and tests.
+ * Writes min(n_out, 7) int32 words to `out` (host memory): N, the partial
+ * slots per row in vocabulary parts over both LM-head launches, the main
+ * launch's band size (runner m-tiles) and parts, the spill launch's band size
+ * and parts (0, 0 without one) and the v-tile where the spill launch's range
+ * begins (the v-tile count without one). Arguments as for bd_step_kernels;
+ * n_rows in 0..window positions. Returns the number of words of the plan (7),
+ * or a negative bd_status. The plan never changes what is computed. */
+int bd_plan_header(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                   const bd_tau_grid* tau_grid, const bd_exec* exec, int32_t n_rows, int32_t* out, int32_t n_out);
+
 /* ------------------------------------------------------------ tuning knobs --
  * Environment variables read at every call (none is needed; each changes how
  * the work is done, never what is computed):
@@ -245,6 +269,12 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight,
  *   BD_PAIR_MC=1|2       single CTA pairs, or clusters of two pairs sharing each
  *                        head tile by multicast (default: clusters for windows of
  *                        at most 512 positions or more than 256 MiB of packed rows)
+ *   BD_PAIR_SPILL=0|1    with clusters of two pairs, the CTA pairs that still fit
+ *                        on the SMs the clusters leave free (4 on a 152-SM GB300)
+ *                        take the last v-tiles in a second, concurrent launch
+ *                        (default: on for more than 256 MiB of packed rows)
+ *   BD_SPILL_PCT=n       a spill pair's time per v-tile against a cluster pair's,
+ *                        in percent (default 100): sets the vocabulary split
  *   BD_PLAN_GM=n, BD_PLAN_GV=n   fix the work plan's band size (runner m-tiles)
  *                        or vocabulary part count; BD_PLAN_RR=1 takes its units
  *                        round-robin instead of in packed rounds

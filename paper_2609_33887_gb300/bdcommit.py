@@ -126,6 +126,10 @@ def load_library(path: Optional[str] = None) -> ctypes.CDLL:
                                       POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, POINTER(bd_exec)]),
         "bd_workspace_size": (c_size_t, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
                                          POINTER(bd_tau_grid)]),
+        "bd_step_kernels": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                    POINTER(bd_tau_grid), POINTER(bd_exec)]),
+        "bd_plan_header": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
+                                   POINTER(bd_tau_grid), POINTER(bd_exec), c_int32, POINTER(c_int32), c_int32]),
         "bd_commit_step_static": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_mask_state),
                                           POINTER(bd_tau_grid), c_void_p, c_void_p, c_void_p, c_void_p]),
         "bd_verify_step": (c_int, [POINTER(bd_hidden), POINTER(bd_weight), POINTER(bd_draft), POINTER(bd_eps_grid),
@@ -245,6 +249,40 @@ def bd_workspace_size(hidden, weight, weight_scale, pos_masked, block_flags, n_s
     tg, _keep = make_tau_grid(tau)
     return int(load_library().bd_workspace_size(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms),
                                                 ctypes.byref(tg)))
+
+
+def bd_step_kernels(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                    mask_token_id, tau, *, variant=VARIANT_AUTO, flags=0) -> int:
+    """Kernels one bd_commit_step_ex call with these arguments queues (a
+    negative bd_status for invalid arguments). Queues nothing."""
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    ex = bd_exec()
+    ex.variant = variant
+    ex.flags = flags
+    return int(load_library().bd_step_kernels(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms),
+                                              ctypes.byref(tg), ctypes.byref(ex)))
+
+
+def bd_plan_header(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
+                   mask_token_id, tau, n_rows, *, variant=VARIANT_AUTO, flags=0):
+    """The LM head's work plan for n_rows compacted rows (seven int32 words,
+    see include/bdcommit.h), or raises on a negative status."""
+    h = make_hidden(hidden)
+    w = make_weight(weight, weight_scale)
+    ms = make_mask_state(pos_masked, block_flags, n_seq, n_slots, block_len, mask_token_id)
+    tg, _keep = make_tau_grid(tau)
+    ex = bd_exec()
+    ex.variant = variant
+    ex.flags = flags
+    out = (c_int32 * 7)()
+    rc = int(load_library().bd_plan_header(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
+                                           ctypes.byref(ex), int(n_rows), out, 7))
+    if rc < 0:
+        raise RuntimeError(f"bd_plan_header: {bd_status_string(rc)}")
+    return list(out)[:rc]
 
 
 def bd_commit_step_ex(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,

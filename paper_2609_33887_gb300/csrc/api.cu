@@ -231,7 +231,7 @@ int64_t head_operand_bytes(const Call& c) {
 }
 
 BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
-  BandPlan p;
+  BandPlan p{};
   p.mc = 1;
   if (c.pair) {
     p.BM = 0;  // token groups derived from N on the device
@@ -249,6 +249,16 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
     if (!c.fused && env_int("BD_PAIR_MC", mc_auto, 1, 2) == 2 && quads > 0) {
       p.mc = 2;
       p.G = quads;
+      // the pairs the clusters leave room for run as a concurrent spill
+      // launch over the last v-tiles (BD_PAIR_SPILL = 0 / 1 forces it off /
+      // on; BD_SPILL_PCT: a spill pair's time per tile against a cluster
+      // pair's, in percent, which sets the vocabulary split)
+      const int spare = pairs - 2 * quads;
+      const int spill_auto = rows_bytes > (int64_t(256) << 20) ? 1 : 0;  // measured faster there only
+      if (spare > 0 && env_int("BD_PAIR_SPILL", spill_auto, 0, 1) == 1) {
+        p.G2 = spare;
+        p.spill_pct = env_int("BD_SPILL_PCT", 100, 50, 400);
+      }
     }
   } else if (c.tc) {
     p.BM = bd::TC_BM;
@@ -285,7 +295,7 @@ Layout make_layout(const Call& c, const BandPlan& p) {
     return o;
   };
   const size_t P = static_cast<size_t>(c.P);
-  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
+  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(plan_max_parts(p));
   l.hdr = take(256, 256);
   l.idx = take(4 * P, 256);
   l.rowpos = take(4 * P, 256);
@@ -549,6 +559,24 @@ int run_step(const Call& c, const BandPlan& plan, const Layout& lay, uint8_t* ws
   }
   return cuda_status(bd::launch_merge_commit(ca, st));
 }
+
+// check_args plus the bd_exec flags (W8A8 runs on the CTA-pair kernel with an
+// E4M3 head read by TMA).
+int check_exec_args(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                    const bd_tau_grid* tau_grid, int variant, int flags, Call* c) {
+  if (flags & ~BD_EXEC_FP8_ACTIVATIONS) return BD_ERR_ARG;
+  int rc = check_args(hidden, weight, mask_state, tau_grid, variant, c);
+  if (rc != BD_OK) return rc;
+  if (flags & BD_EXEC_FP8_ACTIVATIONS) {
+    if (c->wdt != BD_E4M3 || c->hdt != BD_BF16 || !c->pair) return BD_ERR_ARG;
+    if (!aligned(weight->data, 16) || weight->ld % 16 != 0 || c->d < 16) return BD_ERR_ALIGN;
+    c->fp8_act = true;
+    c->fused = false;
+    c->split = false;
+  }
+  return BD_OK;
+}
+
 // Drops the cached device addresses of the allocation-free entry point's
 // array (defined with it, below); the caller holds g_mu.
 void forget_static_devices();
@@ -585,24 +613,47 @@ size_t bd_workspace_size(const bd_hidden* hidden, const bd_weight* weight, const
   return make_layout(c, make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads)).total;
 }
 
+int bd_plan_header(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                   const bd_tau_grid* tau_grid, const bd_exec* exec, int32_t n_rows, int32_t* out, int32_t n_out) {
+  if (!out || n_out < 0 || n_rows < 0) return BD_ERR_ARG;
+  Call c;
+  const int rc = check_exec_args(hidden, weight, mask_state, tau_grid, exec ? exec->variant : 0,
+                                 exec ? exec->flags : 0, &c);
+  if (rc != BD_OK) return rc;
+  if (n_rows > c.P) return BD_ERR_ARG;
+  DevCtx* ctx = nullptr;
+  if (device_ctx(&ctx) != BD_OK) return BD_ERR_DEVICE;
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads);
+  int hdr[bd::HDR_WORDS] = {0};
+  bd::plan_header(plan, n_rows, hdr);
+  for (int i = 0; i < n_out && i < bd::HDR_WORDS; ++i) out[i] = hdr[i];
+  return bd::HDR_WORDS;
+}
+
+int bd_step_kernels(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
+                    const bd_tau_grid* tau_grid, const bd_exec* exec) {
+  Call c;
+  const int rc = check_exec_args(hidden, weight, mask_state, tau_grid, exec ? exec->variant : 0,
+                                 exec ? exec->flags : 0, &c);
+  if (rc != BD_OK) return rc;
+  if (c.P == 0) return 0;
+  DevCtx* ctx = nullptr;
+  if (device_ctx(&ctx) != BD_OK) return BD_ERR_DEVICE;
+  const BandPlan plan = make_plan(c, ctx->sm_count, ctx->pairs, ctx->quads);
+  // compaction + row packing, the head decode where a bf16 copy is made, the
+  // LM head (two launches with spill pairs), merge + commit
+  return 1 + (c.tc && decoded_head(c) ? 1 : 0) + (c.pair && plan.G2 > 0 ? 2 : 1) + 1;
+}
+
 int bd_commit_step_ex(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
                       const bd_tau_grid* tau_grid, int32_t* out_tokens, float* out_conf, uint32_t* out_commit,
                       const bd_exec* exec) {
   bd::TraceRange trace("bd_commit_step");
   const int variant = exec ? exec->variant : 0;
   const int flags = exec ? exec->flags : 0;
-  if (flags & ~BD_EXEC_FP8_ACTIVATIONS) return BD_ERR_ARG;
   Call c;
-  int rc = check_args(hidden, weight, mask_state, tau_grid, variant, &c);
+  int rc = check_exec_args(hidden, weight, mask_state, tau_grid, variant, flags, &c);
   if (rc != BD_OK) return rc;
-  if (flags & BD_EXEC_FP8_ACTIVATIONS) {
-    // W8A8 runs on the CTA-pair kernel with an E4M3 head read by TMA
-    if (c.wdt != BD_E4M3 || c.hdt != BD_BF16 || !c.pair) return BD_ERR_ARG;
-    if (!aligned(weight->data, 16) || weight->ld % 16 != 0 || c.d < 16) return BD_ERR_ALIGN;
-    c.fp8_act = true;
-    c.fused = false;
-    c.split = false;
-  }
   if (c.P == 0) return BD_OK;
   if (!out_tokens || !out_conf || !out_commit) return BD_ERR_NULL;
   if (!aligned(out_tokens, 4) || !aligned(out_conf, 4) || !aligned(out_commit, 4)) return BD_ERR_ALIGN;
@@ -975,7 +1026,7 @@ VerifyLayout make_verify_layout(const Call& c, const BandPlan& p) {
     return o;
   };
   const size_t R = static_cast<size_t>(c.P);
-  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(p.G < p.n_vt ? p.G : p.n_vt);
+  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(plan_max_parts(p));
   l.hdr = take(256, 256);
   l.idx = take(4 * R, 256);
   l.draft_row = take(4 * R, 256);

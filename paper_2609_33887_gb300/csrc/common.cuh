@@ -55,7 +55,7 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 //
 // (GM, gv): among the pairs whose makespan rounds * (2 ceil(n_vt / gv) + 1)
 // (in half v-tiles: half a v-tile for each unit's start and finish) is within
-// MAKESPAN_SLACK of the best, the fewest bands (each band streams the head
+// 5% (MAKESPAN_SLACK_DIV) of the best, the fewest bands (each band streams the head
 // once), then the smaller makespan, then the smaller gv; over GM <= min(n_mt,
 // G) with GM m-tiles of rows within the in-flight budget below (they stay in
 // L2 while their parts run) and gv <= min(G, n_vt). N is only known on the
@@ -75,7 +75,17 @@ struct BandPlan {
   int mc;         // m-tiles a runner holds at once (1, or 2 for 4-CTA clusters)
   int gv_fixed;   // vocabulary parts when > 0 (clamped to 1..min(G, n_vt)), else chosen
   int rr;         // 1: units taken round-robin (runner c: units c, c + G, ...) instead of packed rounds
+  int G2;         // spill runners: single CTA pairs on the SMs the clusters leave free (0: none)
+  int spill_pct;  // a spill pair's time per tile against a cluster pair's, in percent (0: 100)
+  int role;       // 0: the main launch; 1: the spill launch (single pairs, the last v-tiles)
 };
+
+// Words of the workspace header (int32) the kernel that learns N writes for
+// the LM-head and merge kernels: N, the partial slots per row in parts (all
+// launches), the main launch's band size and parts, the spill launch's band
+// size and parts, and the v-tile where the spill launch's range begins (n_vt
+// without a spill launch).
+enum : int { HDR_N = 0, HDR_PARTS = 1, HDR_GM = 2, HDR_GV = 3, HDR_GM2 = 4, HDR_GV2 = 5, HDR_VSPLIT = 6, HDR_WORDS = 7 };
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
 
@@ -103,10 +113,12 @@ __host__ __device__ __forceinline__ int plan_runner_mts(const BandPlan& p, int n
 // m-tiles: over many rounds the runners drift apart, the units in flight span
 // neighbouring bands, and larger bands no longer stay in L2 (the 256 x 8 x 64
 // window read 134 GB with bands of 12 runner m-tiles, 52 GB with bands of 2).
-constexpr double ROWS_IN_FLIGHT = 64.0 * 1024 * 1024;
-constexpr double ROWS_IN_FLIGHT_MANY = 12.0 * 1024 * 1024;
-// Among (GM, gv) within this factor of the best makespan, the fewest bands win.
-constexpr double MAKESPAN_SLACK = 1.05;
+constexpr int64_t ROWS_IN_FLIGHT = int64_t(64) << 20;
+constexpr int64_t ROWS_IN_FLIGHT_MANY = int64_t(12) << 20;
+// Among (GM, gv) within 1 + 1/MAKESPAN_SLACK_DIV (5%) of the best makespan,
+// the fewest bands win. The plan's arithmetic is integer throughout: the
+// kernel that learns N evaluates it on the device, where float64 is slow.
+constexpr uint64_t MAKESPAN_SLACK_DIV = 20;
 
 // The packing of the parts into rounds, for n_mt m-tiles, bands of gm and gv
 // parts: nb full bands (their parts hold gm units, k1 per round) and, when
@@ -123,9 +135,10 @@ __host__ __device__ __forceinline__ Packing plan_pack(int n_mt, int G, int gm, i
   k.rem = n_mt - k.nb * gm;
   k.k1 = G / gm;
   k.kr = k.rem > 0 ? G / k.rem : 0;
-  const int64_t full_parts = static_cast<int64_t>(k.nb) * gv;
-  k.R0 = static_cast<int>(full_parts / k.k1);
-  k.u0 = static_cast<int>(full_parts - static_cast<int64_t>(k.R0) * k.k1) * gm;
+  // nb * gv < 2^28 (at most 2^19 m-tiles of 2^24 positions, gv <= 304): 32-bit
+  const int full_parts = k.nb * gv;
+  k.R0 = full_parts / k.k1;
+  k.u0 = (full_parts - k.R0 * k.k1) * gm;
   int left = k.rem > 0 ? gv : 0;
   k.f = 0;
   if (k.u0 > 0 && k.rem > 0) {
@@ -160,7 +173,7 @@ __host__ __device__ __forceinline__ void plan_gm_range(const BandPlan& p, int bm
     *lo = *hi = p.GM < top ? p.GM : (top > 0 ? top : 1);
     return;
   }
-  const double tile = static_cast<double>(bm) * plan_mc(p) * (p.row_bytes > 0 ? p.row_bytes : 1);
+  const int64_t tile = static_cast<int64_t>(bm) * plan_mc(p) * (p.row_bytes > 0 ? p.row_bytes : 1);
   int cap = static_cast<int>((n_mt > 2 * p.G ? ROWS_IN_FLIGHT_MANY : ROWS_IN_FLIGHT) / tile);
   if (cap < 1) cap = 1;
   *lo = 1;
@@ -190,7 +203,7 @@ __host__ __device__ __forceinline__ void plan_choose(const BandPlan& p, int n_ro
       const uint64_t c = plan_cost(p, n_mt, gm, gv);
       c_min = c < c_min ? c : c_min;
     }
-  const uint64_t c_max = static_cast<uint64_t>(static_cast<double>(c_min) * MAKESPAN_SLACK);
+  const uint64_t c_max = c_min + c_min / MAKESPAN_SLACK_DIV;
   uint64_t best = ~uint64_t(0);
   for (int gm = glo; gm <= ghi; ++gm)
     for (int gv = vlo; gv <= vhi; ++gv) {
@@ -213,8 +226,18 @@ __device__ __forceinline__ void plan_choose_warp(const BandPlan& p, int n_rows, 
   plan_gv_range(p, &vlo, &vhi);
   const int nv = vhi - vlo + 1;
   const int total = (ghi - glo + 1) * nv;
+  const int lane = static_cast<int>(threadIdx.x & 31);
+  // the first 32 * CACHED candidates' costs stay in registers for the second pass
+  constexpr int CACHED = 4;
+  uint64_t cc[CACHED];
   uint64_t c_min = ~uint64_t(0);
-  for (int i = static_cast<int>(threadIdx.x & 31); i < total; i += 32) {
+#pragma unroll
+  for (int q = 0; q < CACHED; ++q) {
+    const int i = lane + 32 * q;
+    cc[q] = i < total ? plan_cost(p, n_mt, glo + i / nv, vlo + i % nv) : ~uint64_t(0);
+    c_min = cc[q] < c_min ? cc[q] : c_min;
+  }
+  for (int i = lane + 32 * CACHED; i < total; i += 32) {
     const uint64_t c = plan_cost(p, n_mt, glo + i / nv, vlo + i % nv);
     c_min = c < c_min ? c : c_min;
   }
@@ -223,9 +246,17 @@ __device__ __forceinline__ void plan_choose_warp(const BandPlan& p, int n_rows, 
     const uint64_t other = __shfl_xor_sync(0xffffffffu, c_min, o);
     c_min = other < c_min ? other : c_min;
   }
-  const uint64_t c_max = static_cast<uint64_t>(static_cast<double>(c_min) * MAKESPAN_SLACK);
+  const uint64_t c_max = c_min + c_min / MAKESPAN_SLACK_DIV;
   uint64_t best = ~uint64_t(0);
-  for (int i = static_cast<int>(threadIdx.x & 31); i < total; i += 32) {
+#pragma unroll
+  for (int q = 0; q < CACHED; ++q) {
+    const int i = lane + 32 * q;
+    if (i < total && cc[q] <= c_max) {
+      const uint64_t k = plan_key(p, n_mt, glo + i / nv, vlo + i % nv, cc[q]);
+      best = k < best ? k : best;
+    }
+  }
+  for (int i = lane + 32 * CACHED; i < total; i += 32) {
     const uint64_t c = plan_cost(p, n_mt, glo + i / nv, vlo + i % nv);
     if (c > c_max) continue;
     const uint64_t k = plan_key(p, n_mt, glo + i / nv, vlo + i % nv, c);
@@ -241,36 +272,134 @@ __device__ __forceinline__ void plan_choose_warp(const BandPlan& p, int n_rows, 
 }
 #endif
 
+// Spill runners. Clusters of two CTA pairs cannot fill every SM (152 SMs hold
+// 36 clusters of 4 CTAs); the G2 pairs that still fit run as a second,
+// concurrent launch of single pairs (role 1) over the last v-tiles. The
+// vocabulary is split so that both launches carry the same time per pair:
+// the main launch's G runners take n_rmt runner m-tiles (mc m-tiles each, one
+// per pair) of vsplit v-tiles, the spill pairs n_mt m-tiles of the remaining
+// n_vt - vsplit v-tiles at spill_pct percent of a cluster pair's time per tile.
+// Each launch then chooses its own (GM, gv) over its own range.
+__host__ __device__ __forceinline__ int plan_vsplit(const BandPlan& p, int n_rows) {
+  if (p.G2 <= 0 || n_rows <= 0) return p.n_vt;
+  const int64_t n_mt = cdiv(n_rows, plan_bm(p, n_rows));
+  const int64_t n_rmt = plan_runner_mts(p, n_rows);
+  const int64_t pct = p.spill_pct > 0 ? p.spill_pct : 100;
+  // n_rmt vsplit / G = (pct / 100) n_mt (n_vt - vsplit) / G2, rounded to nearest
+  const int64_t num = pct * n_mt * p.n_vt * p.G;
+  const int64_t den = 100 * n_rmt * p.G2 + pct * n_mt * p.G;
+  int vsplit = static_cast<int>((2 * num + den) / (2 * den));
+  if (vsplit > p.n_vt - 1) vsplit = p.n_vt;  // nothing left for the spill launch
+  if (vsplit < 1) vsplit = 1;
+  return vsplit;
+}
+
+// The plan of one launch over its share of the vocabulary (role 0: v-tiles
+// [0, vsplit), role 1: [vsplit, n_vt)).
+__host__ __device__ __forceinline__ BandPlan plan_share(const BandPlan& p, int vsplit, int role) {
+  BandPlan q = p;
+  q.role = role;
+  if (role == 0) {
+    q.n_vt = vsplit;
+  } else {
+    q.n_vt = p.n_vt - vsplit;
+    q.G = p.G2;
+    q.mc = 1;
+    q.GM = 0;
+    q.gv_fixed = 0;
+  }
+  return q;
+}
+
+// The workspace header for N rows, sequentially (host).
+__host__ __device__ __forceinline__ void plan_header(const BandPlan& p, int n_rows, int* hdr) {
+  const int vsplit = plan_vsplit(p, n_rows);
+  int gm = 1, gv = 1, gm2 = 0, gv2 = 0;
+  plan_choose(plan_share(p, vsplit, 0), n_rows, &gm, &gv);
+  if (vsplit < p.n_vt) plan_choose(plan_share(p, vsplit, 1), n_rows, &gm2, &gv2);
+  hdr[HDR_N] = n_rows;
+  hdr[HDR_PARTS] = gv + gv2;
+  hdr[HDR_GM] = gm;
+  hdr[HDR_GV] = gv;
+  hdr[HDR_GM2] = gm2;
+  hdr[HDR_GV2] = gv2;
+  hdr[HDR_VSPLIT] = vsplit;
+}
+
+#ifdef __CUDACC__
+// The same header by one warp (the kernel that learns N calls it once); lane
+// 0 writes it.
+__device__ __forceinline__ void plan_write_header(const BandPlan& p, int n_rows, int* hdr) {
+  const int vsplit = plan_vsplit(p, n_rows);
+  int gm = 1, gv = 1, gm2 = 0, gv2 = 0;
+  plan_choose_warp(plan_share(p, vsplit, 0), n_rows, &gm, &gv);
+  if (vsplit < p.n_vt) plan_choose_warp(plan_share(p, vsplit, 1), n_rows, &gm2, &gv2);
+  if ((threadIdx.x & 31) == 0) {
+    hdr[HDR_N] = n_rows;
+    hdr[HDR_PARTS] = gv + gv2;
+    hdr[HDR_GM] = gm;
+    hdr[HDR_GV] = gv;
+    hdr[HDR_GM2] = gm2;
+    hdr[HDR_GV2] = gv2;
+    hdr[HDR_VSPLIT] = vsplit;
+  }
+}
+#endif
+
+// A header word, read past L1: the spill launch starts without waiting on
+// the kernel that wrote the header (that kernel has completed by then).
+__host__ __device__ __forceinline__ int hdr_word(const int* hdr, int i) {
+#ifdef __CUDA_ARCH__
+  return __ldcg(hdr + i);
+#else
+  return hdr[i];
+#endif
+}
+
+// Parts the partial arrays hold per row at most, over both launches.
+__host__ __device__ __forceinline__ int plan_max_parts(const BandPlan& p) {
+  const int g = p.G + (p.G2 > 0 ? p.G2 : 0);
+  return g < p.n_vt ? g : p.n_vt;
+}
+
 // Iterates the units of runner `runner` under the packed plan.
 struct TileIter {
   int runner, G;
   int n_mt, gm, gv, n_vt, mc, rr;
+  int vt0;     // first v-tile of this launch's range
+  int slot0;   // parts of the other launch before this one's in the partial slots
   Packing k;
   int round;
   int m_tile;  // current m-tile (the first of the runner's mc m-tiles)
-  int part;    // vocabulary part of the current unit
+  int part;    // vocabulary part of the current unit (this launch's; slot part + slot0)
   int vt, vt_end;
 
-  // n_rows, bands and parts: the header the compaction kernel wrote (N, GM, gv)
-  __host__ __device__ void init(const BandPlan& plan, int n_rows, int band_mts, int parts, int runner_index) {
+  // hdr: the workspace header the kernel that learns N wrote (HDR_*)
+  __host__ __device__ void init(const BandPlan& plan, const int* hdr, int runner_index) {
     runner = runner_index;
     G = plan.G;
-    n_vt = plan.n_vt;
     mc = plan_mc(plan);
+    const int n_rows = hdr_word(hdr, HDR_N);
     n_mt = plan_runner_mts(plan, n_rows);
-    gm = band_mts > 0 ? band_mts : 1;
-    gv = parts > 0 ? parts : 1;
+    const bool spill = plan.role == 1;
+    const int vsplit = hdr_word(hdr, HDR_VSPLIT);
+    gm = hdr_word(hdr, spill ? HDR_GM2 : HDR_GM);
+    gv = hdr_word(hdr, spill ? HDR_GV2 : HDR_GV);
+    vt0 = spill ? vsplit : 0;
+    n_vt = spill ? plan.n_vt - vsplit : vsplit;
+    slot0 = spill ? hdr_word(hdr, HDR_GV) : 0;
+    if (gm < 1) gm = 1;
+    const bool none = n_mt == 0 || gv < 1 || n_vt < 1;
+    if (gv < 1) gv = 1;
     k = plan_pack(n_mt > 0 ? n_mt : 1, G, gm, gv);
     rr = plan.rr;
     if (rr) k.rounds = static_cast<int>((static_cast<int64_t>(n_mt) * gv + G - 1) / G);
-    if (n_mt == 0) k.rounds = 0;
+    if (none) k.rounds = 0;
     round = -1;
     vt = vt_end = 0;
   }
 #ifdef __CUDACC__
-  __device__ void init(const BandPlan& plan, int n_rows, int band_mts, int parts) {
-    init(plan, n_rows, band_mts, parts, blockIdx.x);
-  }
+  __device__ void init(const BandPlan& plan, const int* hdr) { init(plan, hdr, blockIdx.x); }
 #endif
   // Round-robin order (plan.rr): unit u = c + r G in band-major, part-major
   // order; false past the last unit.
@@ -284,8 +413,8 @@ struct TileIter {
     const int g = n_mt - m0 < gm ? n_mt - m0 : gm;
     part = i / g;
     m_tile = (m0 + i % g) * mc;
-    vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
-    vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
+    vt = vt0 + static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
+    vt_end = vt0 + static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
     return true;
   }
   // This runner's unit of round r: false if its slot is idle there.
@@ -317,8 +446,8 @@ struct TileIter {
       part = j;
     }
     m_tile = mt * mc;
-    vt = static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
-    vt_end = static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
+    vt = vt0 + static_cast<int>(static_cast<int64_t>(part) * n_vt / gv);
+    vt_end = vt0 + static_cast<int>(static_cast<int64_t>(part + 1) * n_vt / gv);
     return true;
   }
   // Advances to the next unit; false when there is no more work.

@@ -405,10 +405,14 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   const uint32_t tmem_base = ctl->tmem_base;
   volatile int* abort_flag = &ctl->abort_flag;
 
-  griddep_wait();  // the packed rows and N come from the preceding kernel
-  const int n_rows = a.n_rows[0];
-  const int parts = a.n_rows[1];     // vocabulary parts of the plan (see common.cuh)
-  const int band_mts = a.n_rows[2];  // ... and its band size
+  // The packed rows and the header (N, the plan) come from the preceding
+  // kernel. A spill launch (role 1) follows the main launch, which waited for
+  // that kernel before letting it start; with a spill launch behind it the
+  // main launch lets it start at once, onto the SMs this grid leaves free.
+  const bool spill = a.plan.role == 1;
+  if (!spill) griddep_wait();
+  if (!spill && a.plan.G2 > 0) griddep_launch_dependents();
+  const int n_rows = hdr_word(a.n_rows, HDR_N);
   constexpr int BK = stage_k<HF>();
   constexpr int ACOLS = atom_cols<HF>();
   constexpr int NATOM = BK / ACOLS;
@@ -444,7 +448,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts, pair);
+    it.init(a.plan, a.n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       const int tok0 = (it.m_tile + pp) * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
@@ -508,7 +512,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
       uint32_t stage = 0, phase = 0;
       uint32_t acc = 0, acc_phase = 0;
       TileIter it;
-      it.init(a.plan, n_rows, band_mts, parts, pair);
+      it.init(a.plan, a.n_rows, pair);
       bool ok = true;
       while (ok && it.next_unit()) {
         for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -590,7 +594,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t r = 0, rph = 0;
     uint32_t issued_mask = 0, issued_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts, pair);
+    it.init(a.plan, a.n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -628,7 +632,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     constexpr int RK = raw_k<HF>();
     uint32_t r = 0, rph = 0, stage = 0, phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts, pair);
+    it.init(a.plan, a.n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -674,7 +678,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     uint32_t epi_phase = 0;
     uint32_t acc = 0, acc_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts, pair);
+    it.init(a.plan, a.n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
       float m[MAX_CHUNKS], s[MAX_CHUNKS];
@@ -859,7 +863,7 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         }
         const int row = (it.m_tile + pp) * NT + j;
         if (row < n_rows) {
-          const int64_t o = static_cast<int64_t>(it.part * 2 + static_cast<int>(rank)) * a.P + row;
+          const int64_t o = static_cast<int64_t>((it.slot0 + it.part) * 2 + static_cast<int>(rank)) * a.P + row;
           a.part_m[o] = M;
           a.part_s[o] = S;
           a.part_a[o] = A;
@@ -889,6 +893,9 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     else
       tmem_dealloc_pair(tmem_base, TMEM_COLS);
   }
+  // the spill launch completes only after the main launch: the kernel after
+  // it (the merge) waits on this grid alone
+  if (spill) griddep_wait();
 }
 
 size_t pair_smem_bytes() { return SMEM_BYTES; }
@@ -953,6 +960,22 @@ static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
+  if (a.plan.G2 > 0) {
+    // clusters of two pairs and the spill launch of single pairs behind them
+    // (the header's vocabulary split assumes both run)
+    if (!pair_cluster<HF>() || plan_mc(a.plan) != 2) return cudaErrorInvalidValue;
+    TcArgs main = a;
+    main.plan.role = 0;
+    pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, true, 2);
+    e = cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, main);
+    if (e != cudaSuccess) return e;
+    TcArgs side = a;
+    side.plan.role = 1;
+    side.plan.G = a.plan.G2;
+    side.plan.mc = 1;
+    pair_config(&cfg, attr, side.plan.G, pair_threads<HF>(), st, true, true, 1);
+    return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, side);
+  }
   pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, pair_cluster<HF>(),
               pair_cluster<HF>() ? plan_mc(a.plan) : 1);
   return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, a);

@@ -75,12 +75,10 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int col = tid % SIMT_BN, rg = tid / SIMT_BN;  // this thread's column and row group
   griddep_wait();  // idx and N come from the preceding kernel
-  const int n_rows = a.n_rows[0];
-  const int parts = a.n_rows[1];     // vocabulary parts of the plan (see common.cuh)
-  const int band_mts = a.n_rows[2];  // ... and its band size
+  const int n_rows = a.n_rows[HDR_N];
 
   TileIter it;
-  it.init(a.plan, n_rows, band_mts, parts);
+  it.init(a.plan, a.n_rows);
   while (it.next_unit()) {
     const int r0 = it.m_tile * SIMT_BM;
     if (tid < SIMT_BM) {

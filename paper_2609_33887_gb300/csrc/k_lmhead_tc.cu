@@ -84,9 +84,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
   volatile int* abort_flag = &ctl->abort_flag;
 
   griddep_wait();  // the packed rows and N come from the preceding kernel
-  const int n_rows = a.n_rows[0];
-  const int parts = a.n_rows[1];     // vocabulary parts of the plan (see common.cuh)
-  const int band_mts = a.n_rows[2];  // ... and its band size
+  const int n_rows = a.n_rows[HDR_N];
   const int nk = cdiv(a.d, BK);
 
   if (warp == 0) {
@@ -98,7 +96,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     uint32_t stage = 0, phase = 0;
     uint32_t issued_mask = 0, issued_phase = 0;  // per stage: issued at least once / parity of last issue
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts);
+    it.init(a.plan, a.n_rows);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -135,7 +133,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     uint32_t stage = 0, phase = 0;
     uint32_t acc = 0, acc_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts);
+    it.init(a.plan, a.n_rows);
     bool ok = true;
     while (ok && it.next_unit()) {
       for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
@@ -190,7 +188,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
     const uint32_t lane_addr = static_cast<uint32_t>(quarter * 32) << 16;
     uint32_t acc = 0, acc_phase = 0;
     TileIter it;
-    it.init(a.plan, n_rows, band_mts, parts);
+    it.init(a.plan, a.n_rows);
     bool ok = true;
     while (ok && it.next_unit()) {
       float m = -INFINITY, s = 0.f;

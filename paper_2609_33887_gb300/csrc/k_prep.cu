@@ -109,20 +109,22 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       }
     }
   }
-  if (p1 == P && warp == 0) {
-    // the CTA holding the last position knows N: it writes N and the plan's
-    // vocabulary parts and band size for it into the header the later kernels read
-    const int N = prefix + local_total;
-    int gm = 1, gv = 1;
-    plan_choose_warp(plan, N, &gm, &gv);
-    if (lane == 0) {
-      n_rows[0] = N;
-      n_rows[1] = gv;
-      n_rows[2] = gm;
-    }
+  // The CTA holding the last position knows N: its warp 0 writes N and the
+  // plan for it into the header the later kernels read, while the CTA's other
+  // warps pack its rows (the plan's evaluation stays off the packing's path).
+  const bool header_warp = p1 == P && warp == 0;
+  if (hidden == nullptr) {
+    if (header_warp) plan_write_header(plan, prefix + local_total, n_rows);
+    return;
   }
-  if (hidden == nullptr) return;
   __syncthreads();
+  if (header_warp) {
+    plan_write_header(plan, prefix + local_total, n_rows);
+    return;
+  }
+  // the packing warps: all of them, or all but warp 0 in the header's CTA
+  const int w0 = p1 == P ? 1 : 0;
+  const int n_pack = PREP_THREADS / 32 - w0;
 
   const int nvec = d / 8;
   if constexpr (FMT == ROWS_F16_POW2) {
@@ -131,7 +133,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // magnitude lands in [2^14, 2^15) and every bf16 value at or above 2^-14
     // after scaling is exact in f16), s at most 126 so 2^-s stays a normal
     // float; tok_scale = 2^-s, 0 for an all-zero row.
-    for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+    for (int i = warp - w0; i < local_total; i += n_pack) {
       if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
@@ -189,7 +191,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // in bytes); tok_scale = 2^-s (0 for an all-zero row).
     uint8_t* hq = reinterpret_cast<uint8_t*>(hc);
     uint8_t* lq = hq + static_cast<int64_t>(P) * ldc;
-    for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+    for (int i = warp - w0; i < local_total; i += n_pack) {
       if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
@@ -254,7 +256,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // to nearest even, saturating), scale = a / 448; an all-zero row gets codes
     // 0 and scale 0. Each float32 step is one correctly rounded operation.
     uint8_t* hq = reinterpret_cast<uint8_t*>(hc);  // ldc counts bytes here
-    for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+    for (int i = warp - w0; i < local_total; i += n_pack) {
       if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
@@ -297,7 +299,7 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
   }
 
   // 3. copy the chunk's live rows, one warp per row, 16-byte vectors
-  for (int i = warp; i < local_total; i += PREP_THREADS / 32) {
+  for (int i = warp - w0; i < local_total; i += n_pack) {
     if (!index_ok(prefix + i, P, status)) continue;
     const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
     const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
@@ -351,15 +353,7 @@ __global__ void __launch_bounds__(256) prep_verify_kernel(const int32_t* __restr
     idx[r] = r;
     draft_row[r] = i < n_draft ? draft[q * n_draft + i] : -1;
   }
-  if (blockIdx.x == 0 && threadIdx.x < 32) {  // N and the plan's parts and band size for it
-    int gm = 1, gv = 1;
-    plan_choose_warp(plan, R, &gm, &gv);
-    if (threadIdx.x == 0) {
-      n_rows[0] = R;
-      n_rows[1] = gv;
-      n_rows[2] = gm;
-    }
-  }
+  if (blockIdx.x == 0 && threadIdx.x < 32) plan_write_header(plan, R, n_rows);  // N and the plan for it
 }
 
 cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,

@@ -1,10 +1,14 @@
 // Host check of the LM-head work plan (common.cuh): for each case given on
-// the command line as "n_rows BM GM vt_kb row_bytes G n_vt cpu mc", every (m-tile,
-// v-tile) pair is taken by exactly one unit, the units of every part run in
-// the same round, the part indices stay below the partial slots the merge
-// reads, and the busiest runner's v-tiles are reported against the even
-// share. Prints one line per case:
-//   ok <n_mt> <gv> <slots> <max_vtiles> <ideal_vtiles>   or   FAIL <reason>
+// the command line as "n_rows BM GM vt_kb row_bytes G n_vt cpu mc G2 spill_pct",
+// the header the compaction kernel would write is formed, and over both
+// launches (the main one and, with G2 > 0, the spill launch of G2 single
+// pairs over the last v-tiles) every (m-tile, v-tile) pair is taken by
+// exactly one unit, the units of every part run in the same round of their
+// launch, the partial slots of the two launches do not overlap and stay below
+// the slots the merge reads, and the busiest runner's v-tiles are reported
+// against the even share. Prints one line per case:
+//   ok <n_mt> <parts> <slots> <max_vtiles> <ideal_time> <gm> <vsplit> <max_vtiles_spill> <gm2> <gv2>
+//   or FAIL <reason>
 #include <cstdio>
 #include <cstdlib>
 #include <vector>
@@ -12,8 +16,9 @@
 #include "common.cuh"
 
 int main(int argc, char** argv) {
-  for (int i = 1; i + 8 < argc; i += 9) {
-    bd::BandPlan p;
+  constexpr int NA = 11;
+  for (int i = 1; i + NA - 1 < argc; i += NA) {
+    bd::BandPlan p{};
     const int n_rows = std::atoi(argv[i]);
     p.BM = std::atoi(argv[i + 1]);
     p.GM = std::atoi(argv[i + 2]);
@@ -23,49 +28,75 @@ int main(int argc, char** argv) {
     p.n_vt = std::atoi(argv[i + 6]);
     p.cpu = std::atoi(argv[i + 7]);
     p.mc = std::atoi(argv[i + 8]);
-    p.gv_fixed = 0;
-    p.rr = 0;
+    p.G2 = std::atoi(argv[i + 9]);
+    p.spill_pct = std::atoi(argv[i + 10]);
     const int bm = bd::plan_bm(p, n_rows);
     const int n_mt = n_rows > 0 ? bd::cdiv(n_rows, bm) : 0;  // m-tiles
     const int n_rmt = bd::plan_runner_mts(p, n_rows);        // runner m-tiles (mc m-tiles each)
-    const int mc = bd::plan_mc(p);
+    int hdr[64] = {0};
+    bd::plan_header(p, n_rows, hdr);  // what the compaction kernel stores
+    const int parts = hdr[bd::HDR_PARTS];
+    const int slots = n_rows > 0 ? parts * p.cpu : 0;
     std::vector<int> cover(static_cast<size_t>(n_mt) * p.n_vt, 0);
-    int gm = 1, gv = 1;
-    bd::plan_choose(p, n_rows, &gm, &gv);  // what the compaction kernel stores beside N
-    const int slots = n_rows > 0 ? gv * p.cpu : 0;
-    // the round of each (band, part): every unit of a part must run in the same round
-    std::vector<int> part_round(static_cast<size_t>(bd::cdiv(n_rmt > 0 ? n_rmt : 1, gm)) * gv, -1);
+    std::vector<int> slot_owner(static_cast<size_t>(parts > 0 ? parts : 1), -1);
     const char* fail = nullptr;
-    long long max_load = 0;
-    for (int r = 0; r < p.G && !fail; ++r) {
-      bd::TileIter it;
-      it.init(p, n_rows, gm, gv, r);
-      long long load = 0;
-      while (it.next_unit()) {
-        if (it.m_tile < 0 || it.m_tile >= n_mt || it.m_tile % mc != 0) fail = "m-tile out of range";
-        else if ((it.part + 1) * p.cpu > slots) fail = "part beyond the partial slots";
-        else if (it.vt < 0 || it.vt_end > p.n_vt || it.vt >= it.vt_end) fail = "empty or out-of-range v-tiles";
-        if (fail) break;
-        int& pr = part_round[static_cast<size_t>(it.m_tile / mc / gm) * gv + it.part];
-        if (pr >= 0 && pr != it.round) {
-          fail = "the units of one part run in different rounds";
-          break;
-        }
-        pr = it.round;
-        // the runner's mc m-tiles (one beyond the last is computed on no rows)
-        for (int q = 0; q < mc && it.m_tile + q < n_mt; ++q)
-          for (int v = it.vt; v < it.vt_end; ++v) ++cover[static_cast<size_t>(it.m_tile + q) * p.n_vt + v];
-        load += it.vt_end - it.vt;
+    if (parts > bd::plan_max_parts(p)) fail = "more parts than the workspace holds";
+    long long max_load[2] = {0, 0};
+    for (int role = 0; role < 2 && !fail; ++role) {
+      bd::BandPlan q = p;  // the launch's own arguments
+      q.role = role;
+      if (role == 1) {
+        if (p.G2 <= 0) break;
+        q.G = p.G2;
+        q.mc = 1;
       }
-      if (load > max_load) max_load = load;
+      const int mc = bd::plan_mc(q);
+      const int gm = role ? hdr[bd::HDR_GM2] : hdr[bd::HDR_GM];
+      const int gv = role ? hdr[bd::HDR_GV2] : hdr[bd::HDR_GV];
+      const int lo = role ? hdr[bd::HDR_VSPLIT] : 0, hi = role ? p.n_vt : hdr[bd::HDR_VSPLIT];
+      if (role == 1 && lo == p.n_vt) break;  // nothing for the spill launch
+      const int runner_mts = bd::plan_runner_mts(q, n_rows);
+      // the round of each (band, part): every unit of a part must run in the same round
+      std::vector<int> part_round(static_cast<size_t>(bd::cdiv(runner_mts > 0 ? runner_mts : 1, gm > 0 ? gm : 1)) *
+                                      (gv > 0 ? gv : 1), -1);
+      for (int r = 0; r < q.G && !fail; ++r) {
+        bd::TileIter it;
+        it.init(q, hdr, r);
+        long long load = 0;
+        while (it.next_unit()) {
+          const int slot = it.slot0 + it.part;
+          if (it.m_tile < 0 || it.m_tile >= n_mt || it.m_tile % mc != 0) fail = "m-tile out of range";
+          else if ((slot + 1) * p.cpu > slots) fail = "part beyond the partial slots";
+          else if (slot_owner[slot] >= 0 && slot_owner[slot] != role) fail = "both launches write one slot";
+          else if (it.vt < lo || it.vt_end > hi || it.vt >= it.vt_end) fail = "empty or out-of-range v-tiles";
+          if (fail) break;
+          slot_owner[slot] = role;
+          int& pr = part_round[static_cast<size_t>(it.m_tile / mc / gm) * gv + it.part];
+          if (pr >= 0 && pr != it.round) {
+            fail = "the units of one part run in different rounds";
+            break;
+          }
+          pr = it.round;
+          // the runner's mc m-tiles (one beyond the last is computed on no rows)
+          for (int m = 0; m < mc && it.m_tile + m < n_mt; ++m)
+            for (int v = it.vt; v < it.vt_end; ++v) ++cover[static_cast<size_t>(it.m_tile + m) * p.n_vt + v];
+          load += it.vt_end - it.vt;
+        }
+        if (load > max_load[role]) max_load[role] = load;
+      }
     }
     for (size_t k = 0; !fail && k < cover.size(); ++k)
       if (cover[k] != 1) fail = "a (m-tile, v-tile) pair is not taken exactly once";
     if (fail) {
       std::printf("FAIL %s\n", fail);
     } else {
-      std::printf("ok %d %d %d %lld %.3f %d\n", n_mt, slots / (p.cpu > 0 ? p.cpu : 1), slots, max_load,
-                  static_cast<double>(n_rmt) * p.n_vt / p.G, gm);
+      // the even share: time of a main runner's v-tile = 1, of a spill pair's = w
+      const double w = (p.spill_pct > 0 ? p.spill_pct : 100) / 100.0;
+      const double ideal = p.G2 > 0 && n_rows > 0
+                               ? w * n_mt * n_rmt * static_cast<double>(p.n_vt) / (p.G2 * n_rmt + w * n_mt * p.G)
+                               : static_cast<double>(n_rmt) * p.n_vt / p.G;
+      std::printf("ok %d %d %d %lld %.3f %d %d %lld %d %d\n", n_mt, parts, slots, max_load[0], ideal,
+                  hdr[bd::HDR_GM], hdr[bd::HDR_VSPLIT], max_load[1], hdr[bd::HDR_GM2], hdr[bd::HDR_GV2]);
     }
   }
   return 0;

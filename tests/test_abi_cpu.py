@@ -41,7 +41,7 @@ def test_header_declares_the_abi():
         "bd_commit_step", "bd_commit_step_ex", "bd_commit_step_static", "bd_commit_sweep", "bd_get_device_status",
         "bd_selftest_timeout", "bd_static_device_status", "bd_static_selftest_timeout", "bd_shutdown",
         "bd_lmhead_partials", "bd_merge_commit",
-        "bd_status_string", "bd_version", "bd_workspace_size", "bd_verify_step", "bd_verify_workspace_size",
+        "bd_status_string", "bd_version", "bd_workspace_size", "bd_step_kernels", "bd_plan_header", "bd_verify_step", "bd_verify_workspace_size",
         "bd_binom_cdf", "bd_redline_violations", "bd_redline_pvalues", "bd_redline_test", "bd_redline_deploy",
         "bd_redline_select", "bd_redline_sweep", "bd_redline_critical_count", "bd_redline_power",
         "bd_redline_min_calibration", "bd_redline_tpf"])
@@ -157,6 +157,7 @@ def test_null_structs_rejected(lib):
     assert lib.bd_commit_step(None, ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg), FAKE, FAKE, FAKE) == \
         B.BD_ERR_NULL
     assert lib.bd_workspace_size(ctypes.byref(h), None, ctypes.byref(ms), ctypes.byref(tg)) == 0
+    assert lib.bd_step_kernels(ctypes.byref(h), None, ctypes.byref(ms), ctypes.byref(tg), None) == B.BD_ERR_NULL
 
 
 def test_empty_window_is_a_no_op(lib):

@@ -345,6 +345,76 @@ def test_pair_kernel_with_and_without_clusters_of_two_pairs(name, mc, monkeypatc
     assert rep.n_live > 0
 
 
+def _kernels_per_step(wl):
+    cfg = wl.cfg
+    g = wl.to("cuda")
+    return bdc.bd_step_kernels(g.hidden, g.weight, g.weight_scale, g.pos_masked, g.block_flags, cfg.n_seq,
+                               cfg.n_slots, cfg.block_len, wl.mask_token_id, wl.tau)
+
+
+@pytest.mark.parametrize("pct", ["50", "100", "400"])
+@pytest.mark.parametrize("name", ["bf16_5mt_ktail", "bf16_g294", "e4m3", "bf16_L64"])
+def test_spill_pairs_beside_clusters(name, pct, monkeypatch):
+    # clusters of two pairs plus the concurrent launch of single CTA pairs on
+    # the SMs the clusters leave free, over the last v-tiles; the spill
+    # pair's relative time per tile sets the split (50: more v-tiles for the
+    # spill launch, 400: few or none at these sizes)
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SPILL", "1")
+    monkeypatch.setenv("BD_SPILL_PCT", pct)
+    wl = generate(SMALL[name])
+    assert _kernels_per_step(wl) in (3, 4)  # 4 where the device leaves room for spill pairs
+    _, _, rep = check(wl, variant=3)
+    assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("spill", ["0", "1"])
+def test_full_size_b8_with_and_without_spill_pairs(spill, monkeypatch):
+    # the bench window in both layouts the automatic choice can take
+    monkeypatch.setenv("BD_PAIR_SPILL", spill)
+    wl = generate(B8X2X32_BF16)
+    n = _kernels_per_step(wl)
+    assert n == 3 if spill == "0" else n in (3, 4)
+    _, _, rep = check(wl)
+    assert rep.n_live > 250
+
+
+@pytest.mark.parametrize("spill", ["0", "1"])
+@pytest.mark.parametrize("name", ["b8", "bf16_5mt_ktail", "bf16_2bands", "e4m3", "tied_full"])
+def test_device_plan_equals_the_host_plan(name, spill, monkeypatch):
+    # the compaction kernel evaluates the plan rule with one warp once N is
+    # known; the workspace header it writes (the first seven int32 words of
+    # the caller's workspace) must equal the sequential host evaluation of the
+    # same rule for that N (bd_plan_header)
+    monkeypatch.setenv("BD_PAIR_SPILL", spill)
+    cfg = {"b8": B8X2X32_BF16, "tied_full": B32X4X32_TIED}.get(name) or SMALL[name]
+    wl = generate(cfg)
+    g = wl.to("cuda")
+    args = (g.hidden, g.weight, g.weight_scale, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots,
+            cfg.block_len, wl.mask_token_id, wl.tau)
+    ws = torch.zeros(bdc.bd_workspace_size(*args), dtype=torch.uint8, device="cuda")
+    bdc.commit_step(g.hidden, g.weight, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len,
+                    wl.tau, weight_scale=g.weight_scale, mask_token_id=wl.mask_token_id, workspace=ws)
+    torch.cuda.synchronize()
+    hdr = ws[:28].view(torch.int32).cpu().tolist()
+    n = int(((wl.pos_masked != 0) & (wl.block_flags.repeat_interleave(cfg.block_len) & 1 != 0)).sum())
+    assert hdr[0] == n
+    assert hdr == bdc.bd_plan_header(*args, n)
+    for rows in (0, 1, n // 2, cfg.P):  # the host rule at other N stays within the plan's ranges
+        h = bdc.bd_plan_header(*args, rows)
+        assert h[0] == rows and h[1] == h[3] + h[5] and 1 <= h[6]
+
+
+def test_spill_pairs_on_many_bands(monkeypatch):
+    # clusters, spill pairs and bands of one m-tile on both launches' plans
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SPILL", "1")
+    monkeypatch.setenv("BD_PLAN_GM", "1")
+    wl = generate(scaled(B32X4X32_TIED, n_seq=16, n_slots=4, block_len=64, d=256, V=7000, mask_frac=0.55))
+    _, _, rep = check(wl, variant=3)
+    assert rep.n_live > 2048
+
+
 def test_clusters_of_two_pairs_on_many_bands(monkeypatch):
     # forced clusters and bands of one runner m-tile: every unit boundary of
     # the plan with multicast head tiles, 9 token groups (odd)
