@@ -127,6 +127,18 @@ def test_every_lmhead_kernel(variant):
     check(wl, run_gpu(wl, variant), run_oracle(wl))
 
 
+@pytest.mark.parametrize("name", ["bf16_r297_ktail", "bf16_r40"])
+def test_clusters_with_spill_pairs(name, monkeypatch):
+    """Verification rows on clusters of two CTA pairs with the concurrent spill
+    launch of single pairs over the last v-tiles (the entropy and draft-logit
+    partials take the spill launch's slots too)."""
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SPILL", "1")
+    monkeypatch.setenv("BD_SPILL_PCT", "50")
+    wl = generate_verify(SMALL[name])
+    check(wl, run_gpu(wl, 3), run_oracle(wl))
+
+
 def test_full_size_llama_sampled():
     """The Llama-3.1-8B shape (64 requests x 5 rows, d = 4096, V = 128256), every
     row of three sampled requests against the oracle; the lossless tokens per

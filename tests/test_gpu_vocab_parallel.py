@@ -109,6 +109,20 @@ def test_split_agrees_with_the_single_call(name):
     assert np.abs(out["conf"] - conf.cpu().numpy()).max() < 1e-5
 
 
+@pytest.mark.parametrize("name", ["bf16_4", "e4m3_3"])
+def test_split_with_spill_pairs(name, monkeypatch):
+    # each shard's LM head on clusters of two pairs plus the spill launch
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SPILL", "1")
+    monkeypatch.setenv("BD_SPILL_PCT", "50")
+    cfg, cuts = CASES[name]
+    wl = generate(cfg)
+    out, _ = run_split(wl, shard_bounds(cfg.V, cuts))
+    rep = compare(out, oracle_on_workload(wl), wl.tau, cfg.weight_dtype, cfg.block_len, cfg.n_slots)
+    assert rep.ok(), rep.failures
+    assert rep.n_live > 0
+
+
 def test_argument_errors():
     cfg, cuts = CASES["bf16_2"]
     wl = generate(cfg).to("cuda")
