@@ -52,6 +52,10 @@ SUSTAINED = (B8X2X32_BF16.name, B64X4X64_BF16.name)
 KERNEL_SOURCES = ["paper_2609_33887_gb300/csrc/k_lmhead_pair.cu", "paper_2609_33887_gb300/csrc/k_lmhead_tc.cu",
                   "paper_2609_33887_gb300/csrc/common.cuh"]
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "lmhead_traffic.txt")
+# Idle seconds before each side measurement (other workloads, precision
+# levers): the headline's seconds-long legs leave the board at its power limit
+# with lowered clocks, which the next short measurement would otherwise inherit.
+COOLDOWN_S = 2.0
 
 
 def parse_args():
@@ -470,14 +474,19 @@ def lever_timing(dev, stream, lever: str) -> dict:
         step()
     n = 200
     (e0, e1), = timing_events(1, stream)
+    lm = timing_events(20, stream)
+    torch.cuda.synchronize()
+    time.sleep(COOLDOWN_S)
+    smp = ClockSampler(dev.index if dev.index is not None else 0)
+    smp.start()
     e0.record(stream)
     for _ in range(n):
         step()
     e1.record(stream)
-    lm = timing_events(20, stream)
     for ev in lm:
         step(ev)
     torch.cuda.synchronize()
+    clk = smp.stop()
     st = B.bd_get_device_status(stream)
     if st != 0:
         raise B.BdError(st, lever)
@@ -494,7 +503,7 @@ def lever_timing(dev, stream, lever: str) -> dict:
            "step_hbm_frac": abytes / (ms / 1e3) / 1e9 / hbm_gbs,
            "lmhead_tensor_frac": flops / (lm_us * 1e-6) / 1e12 / tc_peak,
            "tensor_peak_tflops": tc_peak,
-           "path": path,
+           "path": path, "clocks": clk, "cooldown_s": COOLDOWN_S,
            "peak_source": src + (" (x2: nominal FP8 : BF16 ratio)" if lever == "w8a8" else "")}
     if lever == "w8a8":
         # the library's own FP8 GEMM on this GPU, measured here, beside the nominal-ratio peak
@@ -645,7 +654,7 @@ def roofline_of(cfg, n_masked, lm_ms, traffic=None, lm_launches=1):
 def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
     """One of the other workloads: positions/s over a graph-replayed timed region
     of at least `steps` steps and ~min_s seconds, and the LM-head roofline from
-    24 event-timed launches."""
+    24 event-timed launches; clocks sampled over both, after COOLDOWN_S idle."""
     wl_host = generate(cfg)
     r = StepRunner(cfg, wl_host, dev)
     for _ in range(warmup):
@@ -663,6 +672,9 @@ def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
     torch.cuda.synchronize()
     stream = torch.cuda.current_stream()
     (e0, e1), = timing_events(1, stream)
+    time.sleep(COOLDOWN_S)
+    smp = ClockSampler(dev.index if dev.index is not None else 0)
+    smp.start()
     e0.record(stream)
     g.replay()
     e1.record(stream)
@@ -670,12 +682,13 @@ def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
     r.check_status("timed region")
     ms = e0.elapsed_time(e1) / k
     lm = r.lmhead_ms()
+    clk = smp.stop()
     roof = roofline_of(cfg, r.n_masked, lm, recorded_traffic(cfg.name), lmhead_launches(r))
     out = {"positions_per_s": r.n_masked / (ms / 1e3), "ms_per_step": ms, "steps": k,
            "masked_positions": r.n_masked, "lmhead_us": roof["lmhead_ms_avg"] * 1e3,
            "tensor_frac": roof["tensor_view"]["frac"], "hbm_frac": roof["hbm_view"]["frac"],
            "traffic_over_algorithmic": roof["traffic_over_algorithmic"], "roofline": roof,
-           "gpu_launches_per_step": launches_per_step(r)}
+           "gpu_launches_per_step": launches_per_step(r), "clocks": clk, "cooldown_s": COOLDOWN_S}
     del g, r
     torch.cuda.empty_cache()
     return out
