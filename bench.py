@@ -439,8 +439,9 @@ def fp8_gemm_tflops(dev, stream, n=8192, reps=30):
 
 def lever_timing(dev, stream, lever: str) -> dict:
     """The bench window (8 x 2 x 32, d = 2048, V = 151936) with a quantised
-    head (the precision levers): device time per commit step (CUDA events
-    around 200 back-to-back steps), the LM-head kernel's own time, and the step
+    head (the precision levers): after COOLDOWN_S idle, the LM-head kernel's
+    own time (20 event-timed steps), then the device time per commit step
+    (CUDA events around 200 back-to-back steps), and the step
     against the lever's algorithmic bytes (the stored head: NVFP4 codes V*d/2
     and block scales V*d/16, or E4M3 codes V*d; row scales 4V; the masked bf16
     rows; 13 B per window position). The tensor fraction of the W8A8 head is
@@ -479,12 +480,12 @@ def lever_timing(dev, stream, lever: str) -> dict:
     time.sleep(COOLDOWN_S)
     smp = ClockSampler(dev.index if dev.index is not None else 0)
     smp.start()
+    for ev in lm:  # the LM head first, from the idle state (see side_config)
+        step(ev)
     e0.record(stream)
     for _ in range(n):
         step()
     e1.record(stream)
-    for ev in lm:
-        step(ev)
     torch.cuda.synchronize()
     clk = smp.stop()
     st = B.bd_get_device_status(stream)
@@ -652,9 +653,11 @@ def roofline_of(cfg, n_masked, lm_ms, traffic=None, lm_launches=1):
 
 
 def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
-    """One of the other workloads: positions/s over a graph-replayed timed region
-    of at least `steps` steps and ~min_s seconds, and the LM-head roofline from
-    24 event-timed launches; clocks sampled over both, after COOLDOWN_S idle."""
+    """One of the other workloads: after COOLDOWN_S idle, the LM-head roofline
+    from 24 event-timed launches, then positions/s over a graph-replayed timed
+    region of at least `steps` steps and ~min_s seconds; clocks sampled over
+    both. (The LM head is timed first: after a region of this length the board
+    sits at its power limit, which the sustained legs report separately.)"""
     wl_host = generate(cfg)
     r = StepRunner(cfg, wl_host, dev)
     for _ in range(warmup):
@@ -675,13 +678,13 @@ def side_config(cfg, dev, min_s=0.25, steps=20, warmup=5):
     time.sleep(COOLDOWN_S)
     smp = ClockSampler(dev.index if dev.index is not None else 0)
     smp.start()
+    lm = r.lmhead_ms()
     e0.record(stream)
     g.replay()
     e1.record(stream)
     torch.cuda.synchronize()
     r.check_status("timed region")
     ms = e0.elapsed_time(e1) / k
-    lm = r.lmhead_ms()
     clk = smp.stop()
     roof = roofline_of(cfg, r.n_masked, lm, recorded_traffic(cfg.name), lmhead_launches(r))
     out = {"positions_per_s": r.n_masked / (ms / 1e3), "ms_per_step": ms, "steps": k,
