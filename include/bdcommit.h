@@ -249,13 +249,15 @@ int bd_step_kernels(const bd_hidden* hidden, const bd_weight* weight, const bd_m
 /* The work plan the LM head takes for a window of n_rows compacted rows
  * (masked positions of active blocks), as the compaction kernel computes it
  * on the device once N is known; host-only, for inspection and tests.
- * Writes min(n_out, 7) int32 words to `out` (host memory): N, the partial
- * slots per row in vocabulary parts over both LM-head launches, the main
- * launch's band size (runner m-tiles) and parts, the spill launch's band size
- * and parts (0, 0 without one) and the v-tile where the spill launch's range
- * begins (the v-tile count without one). Arguments as for bd_step_kernels;
- * n_rows in 0..window positions. Returns the number of words of the plan (7),
- * or a negative bd_status. The plan never changes what is computed. */
+ * Writes min(n_out, 8) int32 words to `out` (host memory): N, the partial
+ * slots per row over both LM-head launches (vocabulary parts times the CTAs
+ * that write a partial per unit), the main launch's band size (runner
+ * m-tiles) and parts, the spill launch's band size and parts (0, 0 without
+ * one), the v-tile where the spill launch's range begins (the v-tile count
+ * without one) and the spill launch's first slot. Arguments as for
+ * bd_step_kernels; n_rows in 0..window positions. Returns the number of
+ * words of the plan (8), or a negative bd_status. The plan never changes what
+ * is computed. */
 int bd_plan_header(const bd_hidden* hidden, const bd_weight* weight, const bd_mask_state* mask_state,
                    const bd_tau_grid* tau_grid, const bd_exec* exec, int32_t n_rows, int32_t* out, int32_t n_out);
 
@@ -269,6 +271,9 @@ int bd_plan_header(const bd_hidden* hidden, const bd_weight* weight, const bd_ma
  *   BD_PAIR_MC=1|2       single CTA pairs, or clusters of two pairs sharing each
  *                        head tile by multicast (default: clusters for windows of
  *                        at most 512 positions or more than 256 MiB of packed rows)
+ *   BD_PAIR_SHARE=0|1    the two pairs of a cluster share head tiles (two token
+ *                        groups, one v-tile at a time; default) or token rows (one
+ *                        token group, two v-tiles at a time)
  *   BD_PAIR_SPILL=0|1    with clusters of two pairs, the CTA pairs that still fit
  *                        on the SMs the clusters leave free (4 on a 152-SM GB300)
  *                        take the last v-tiles in a second, concurrent launch

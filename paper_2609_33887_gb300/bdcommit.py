@@ -268,7 +268,7 @@ def bd_step_kernels(hidden, weight, weight_scale, pos_masked, block_flags, n_seq
 
 def bd_plan_header(hidden, weight, weight_scale, pos_masked, block_flags, n_seq, n_slots, block_len,
                    mask_token_id, tau, n_rows, *, variant=VARIANT_AUTO, flags=0):
-    """The LM head's work plan for n_rows compacted rows (seven int32 words,
+    """The LM head's work plan for n_rows compacted rows (eight int32 words,
     see include/bdcommit.h), or raises on a negative status."""
     h = make_hidden(hidden)
     w = make_weight(weight, weight_scale)
@@ -277,9 +277,9 @@ def bd_plan_header(hidden, weight, weight_scale, pos_masked, block_flags, n_seq,
     ex = bd_exec()
     ex.variant = variant
     ex.flags = flags
-    out = (c_int32 * 7)()
+    out = (c_int32 * 8)()
     rc = int(load_library().bd_plan_header(ctypes.byref(h), ctypes.byref(w), ctypes.byref(ms), ctypes.byref(tg),
-                                           ctypes.byref(ex), int(n_rows), out, 7))
+                                           ctypes.byref(ex), int(n_rows), out, 8))
     if rc < 0:
         raise RuntimeError(f"bd_plan_header: {bd_status_string(rc)}")
     return list(out)[:rc]

@@ -249,6 +249,13 @@ BandPlan make_plan(const Call& c, int sm_count, int pairs, int quads) {
     if (!c.fused && env_int("BD_PAIR_MC", mc_auto, 1, 2) == 2 && quads > 0) {
       p.mc = 2;
       p.G = quads;
+      // the cluster's two pairs share head tiles (two token groups, one v-tile
+      // at a time) or, with BD_PAIR_SHARE = 1, token rows (one token group,
+      // two v-tiles at a time)
+      if (env_int("BD_PAIR_SHARE", 0, 0, 1) == 1) {
+        p.mc = 1;
+        p.vc = 2;
+      }
       // the pairs the clusters leave room for run as a concurrent spill
       // launch over the last v-tiles (BD_PAIR_SPILL = 0 / 1 forces it off /
       // on; BD_SPILL_PCT: a spill pair's time per tile against a cluster
@@ -295,7 +302,7 @@ Layout make_layout(const Call& c, const BandPlan& p) {
     return o;
   };
   const size_t P = static_cast<size_t>(c.P);
-  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(plan_max_parts(p));
+  const size_t slots = static_cast<size_t>(plan_max_slots(p));
   l.hdr = take(256, 256);
   l.idx = take(4 * P, 256);
   l.rowpos = take(4 * P, 256);
@@ -407,17 +414,18 @@ int launch_lmhead(const Call& c, const BandPlan& plan, const bd_hidden* hidden, 
     if (c.pair && (c.fp8_act || c.split)) {
       // W8A8 / two-term rows: E4M3 token rows and head rows, 128-byte
       // (128-column) boxes; the lo terms follow the hi terms' P rows
-      for (int i = 0; i < 8; ++i) {
-        if (!encode_u8_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 128, 16 * (i + 1), true)) return BD_ERR_CUDA;
+      for (int i = 0; i < 16; ++i) {
+        if (!encode_u8_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 128, 8 * (i + 1), true)) return BD_ERR_CUDA;
         if (c.split && !encode_u8_2d(&tmLo.m[i], static_cast<const uint8_t*>(rows) + c.P * ld_rows, c.d, c.P,
-                                     ld_rows, 128, 16 * (i + 1), true))
+                                     ld_rows, 128, 8 * (i + 1), true))
           return BD_ERR_CUDA;
       }
       if (!encode_u8_2d(&tmB, weight->data, c.d, c.V, c.ldw, 128, 64, true)) return BD_ERR_CUDA;
     } else if (c.pair) {
-      // token rows: one map per box height 16, 32, ..., 128 (half of a token group)
-      for (int i = 0; i < 8; ++i)
-        if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 16 * (i + 1))) return BD_ERR_CUDA;
+      // token rows: one map per box height 8, 16, ..., 128 (half of a token group, or
+      // the quarter a CTA loads for both pairs of a cluster that share token rows)
+      for (int i = 0; i < 16; ++i)
+        if (!encode_bf16_2d(&tmTok.m[i], rows, c.d, c.P, ld_rows, 64, 8 * (i + 1))) return BD_ERR_CUDA;
       if (!c.fused && !encode_bf16_2d(&tmB, wsrc, c.d, c.V, wld, 64, 64)) return BD_ERR_CUDA;
     } else {
       if (!encode_bf16_2d(&tmA, rows, c.d, c.P, ld_rows, bd::TC_BK, bd::TC_BM)) return BD_ERR_CUDA;
@@ -1026,7 +1034,7 @@ VerifyLayout make_verify_layout(const Call& c, const BandPlan& p) {
     return o;
   };
   const size_t R = static_cast<size_t>(c.P);
-  const size_t slots = static_cast<size_t>(p.cpu) * static_cast<size_t>(plan_max_parts(p));
+  const size_t slots = static_cast<size_t>(plan_max_slots(p));
   l.hdr = take(256, 256);
   l.idx = take(4 * R, 256);
   l.draft_row = take(4 * R, 256);

@@ -72,7 +72,8 @@ struct BandPlan {
   int cpu;        // CTAs per unit: each writes its own partial, so a part has cpu slots
   int vt_kb;      // KiB of head per v-tile (BN rows as the kernel reads them)
   int row_bytes;  // bytes of one packed token row as the kernel reads it
-  int mc;         // m-tiles a runner holds at once (1, or 2 for 4-CTA clusters)
+  int mc;         // m-tiles a runner holds at once (1, or 2 for 4-CTA clusters sharing head tiles)
+  int vc;         // v-tiles a runner takes at once (1, or 2 for 4-CTA clusters sharing token rows)
   int gv_fixed;   // vocabulary parts when > 0 (clamped to 1..min(G, n_vt)), else chosen
   int rr;         // 1: units taken round-robin (runner c: units c, c + G, ...) instead of packed rounds
   int G2;         // spill runners: single CTA pairs on the SMs the clusters leave free (0: none)
@@ -81,11 +82,15 @@ struct BandPlan {
 };
 
 // Words of the workspace header (int32) the kernel that learns N writes for
-// the LM-head and merge kernels: N, the partial slots per row in parts (all
-// launches), the main launch's band size and parts, the spill launch's band
-// size and parts, and the v-tile where the spill launch's range begins (n_vt
-// without a spill launch).
-enum : int { HDR_N = 0, HDR_PARTS = 1, HDR_GM = 2, HDR_GV = 3, HDR_GM2 = 4, HDR_GV2 = 5, HDR_VSPLIT = 6, HDR_WORDS = 7 };
+// the LM-head and merge kernels: N, the partial slots per row over all
+// launches (parts times the CTAs that write a partial per unit), the main
+// launch's band size and parts, the spill launch's band size and parts, the
+// v-tile where the spill launch's range begins (n_vt without a spill launch)
+// and the spill launch's first slot.
+enum : int {
+  HDR_N = 0, HDR_SLOTS = 1, HDR_GM = 2, HDR_GV = 3, HDR_GM2 = 4, HDR_GV2 = 5, HDR_VSPLIT = 6, HDR_SLOT0 = 7,
+  HDR_WORDS = 8
+};
 
 __host__ __device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
 
@@ -102,6 +107,7 @@ __host__ __device__ __forceinline__ int plan_bm(const BandPlan& p, int n_rows) {
 }
 
 __host__ __device__ __forceinline__ int plan_mc(const BandPlan& p) { return p.mc > 1 ? p.mc : 1; }
+__host__ __device__ __forceinline__ int plan_vc(const BandPlan& p) { return p.vc > 1 ? p.vc : 1; }
 
 // Runner m-tiles (of plan_mc m-tiles each) for N rows; 0 without rows.
 __host__ __device__ __forceinline__ int plan_runner_mts(const BandPlan& p, int n_rows) {
@@ -276,39 +282,64 @@ __device__ __forceinline__ void plan_choose_warp(const BandPlan& p, int n_rows, 
 // 36 clusters of 4 CTAs); the G2 pairs that still fit run as a second,
 // concurrent launch of single pairs (role 1) over the last v-tiles. The
 // vocabulary is split so that both launches carry the same time per pair:
-// the main launch's G runners take n_rmt runner m-tiles (mc m-tiles each, one
-// per pair) of vsplit v-tiles, the spill pairs n_mt m-tiles of the remaining
-// n_vt - vsplit v-tiles at spill_pct percent of a cluster pair's time per tile.
-// Each launch then chooses its own (GM, gv) over its own range.
+// the main launch's G runners take n_rmt runner m-tiles (mc m-tiles each) of
+// vsplit v-tiles, vc at a time (one per pair either way), the spill pairs n_mt
+// m-tiles of the remaining n_vt - vsplit v-tiles at spill_pct percent of a
+// cluster pair's time per tile. With vc = 2 vsplit is even, so the main
+// launch's v-tile pairs stay in its range. Each launch then chooses its own
+// (GM, gv) over its own range.
 __host__ __device__ __forceinline__ int plan_vsplit(const BandPlan& p, int n_rows) {
   if (p.G2 <= 0 || n_rows <= 0) return p.n_vt;
   const int64_t n_mt = cdiv(n_rows, plan_bm(p, n_rows));
   const int64_t n_rmt = plan_runner_mts(p, n_rows);
+  const int64_t vc = plan_vc(p);
   const int64_t pct = p.spill_pct > 0 ? p.spill_pct : 100;
-  // n_rmt vsplit / G = (pct / 100) n_mt (n_vt - vsplit) / G2, rounded to nearest
-  const int64_t num = pct * n_mt * p.n_vt * p.G;
-  const int64_t den = 100 * n_rmt * p.G2 + pct * n_mt * p.G;
+  // n_rmt vsplit / (G vc) = (pct / 100) n_mt (n_vt - vsplit) / G2, rounded to nearest
+  const int64_t num = pct * n_mt * p.n_vt * p.G * vc;
+  const int64_t den = 100 * n_rmt * p.G2 + pct * n_mt * p.G * vc;
   int vsplit = static_cast<int>((2 * num + den) / (2 * den));
-  if (vsplit > p.n_vt - 1) vsplit = p.n_vt;  // nothing left for the spill launch
-  if (vsplit < 1) vsplit = 1;
+  if (vc == 2) vsplit &= ~1;
+  if (vsplit < static_cast<int>(vc)) vsplit = static_cast<int>(vc);
+  if (vsplit > p.n_vt - static_cast<int>(vc)) vsplit = p.n_vt;  // nothing left for the spill launch
   return vsplit;
 }
 
+// Partial slots a unit writes per row: its CTAs' partials (a CTA pair writes
+// one per CTA; with vc = 2 each pair of the cluster writes its own).
+__host__ __device__ __forceinline__ int plan_unit_slots(const BandPlan& p) { return p.cpu * plan_vc(p); }
+constexpr int SPILL_UNIT_SLOTS = 2;  // a single CTA pair
+
 // The plan of one launch over its share of the vocabulary (role 0: v-tiles
-// [0, vsplit), role 1: [vsplit, n_vt)).
+// [0, vsplit), in steps of vc; role 1: [vsplit, n_vt)). n_vt of the result
+// counts the launch's steps.
 __host__ __device__ __forceinline__ BandPlan plan_share(const BandPlan& p, int vsplit, int role) {
   BandPlan q = p;
   q.role = role;
   if (role == 0) {
-    q.n_vt = vsplit;
+    q.n_vt = cdiv(vsplit, plan_vc(p));
   } else {
     q.n_vt = p.n_vt - vsplit;
     q.G = p.G2;
     q.mc = 1;
+    q.vc = 1;
+    q.cpu = SPILL_UNIT_SLOTS;
     q.GM = 0;
     q.gv_fixed = 0;
   }
   return q;
+}
+
+// The header words from the two launches' choices.
+__host__ __device__ __forceinline__ void plan_fill_header(const BandPlan& p, int n_rows, int vsplit, int gm, int gv,
+                                                          int gm2, int gv2, int* hdr) {
+  hdr[HDR_N] = n_rows;
+  hdr[HDR_SLOTS] = gv * plan_unit_slots(p) + gv2 * SPILL_UNIT_SLOTS;
+  hdr[HDR_GM] = gm;
+  hdr[HDR_GV] = gv;
+  hdr[HDR_GM2] = gm2;
+  hdr[HDR_GV2] = gv2;
+  hdr[HDR_VSPLIT] = vsplit;
+  hdr[HDR_SLOT0] = gv * plan_unit_slots(p);
 }
 
 // The workspace header for N rows, sequentially (host).
@@ -317,13 +348,7 @@ __host__ __device__ __forceinline__ void plan_header(const BandPlan& p, int n_ro
   int gm = 1, gv = 1, gm2 = 0, gv2 = 0;
   plan_choose(plan_share(p, vsplit, 0), n_rows, &gm, &gv);
   if (vsplit < p.n_vt) plan_choose(plan_share(p, vsplit, 1), n_rows, &gm2, &gv2);
-  hdr[HDR_N] = n_rows;
-  hdr[HDR_PARTS] = gv + gv2;
-  hdr[HDR_GM] = gm;
-  hdr[HDR_GV] = gv;
-  hdr[HDR_GM2] = gm2;
-  hdr[HDR_GV2] = gv2;
-  hdr[HDR_VSPLIT] = vsplit;
+  plan_fill_header(p, n_rows, vsplit, gm, gv, gm2, gv2, hdr);
 }
 
 #ifdef __CUDACC__
@@ -334,15 +359,7 @@ __device__ __forceinline__ void plan_write_header(const BandPlan& p, int n_rows,
   int gm = 1, gv = 1, gm2 = 0, gv2 = 0;
   plan_choose_warp(plan_share(p, vsplit, 0), n_rows, &gm, &gv);
   if (vsplit < p.n_vt) plan_choose_warp(plan_share(p, vsplit, 1), n_rows, &gm2, &gv2);
-  if ((threadIdx.x & 31) == 0) {
-    hdr[HDR_N] = n_rows;
-    hdr[HDR_PARTS] = gv + gv2;
-    hdr[HDR_GM] = gm;
-    hdr[HDR_GV] = gv;
-    hdr[HDR_GM2] = gm2;
-    hdr[HDR_GV2] = gv2;
-    hdr[HDR_VSPLIT] = vsplit;
-  }
+  if ((threadIdx.x & 31) == 0) plan_fill_header(p, n_rows, vsplit, gm, gv, gm2, gv2, hdr);
 }
 #endif
 
@@ -356,10 +373,12 @@ __host__ __device__ __forceinline__ int hdr_word(const int* hdr, int i) {
 #endif
 }
 
-// Parts the partial arrays hold per row at most, over both launches.
-__host__ __device__ __forceinline__ int plan_max_parts(const BandPlan& p) {
-  const int g = p.G + (p.G2 > 0 ? p.G2 : 0);
-  return g < p.n_vt ? g : p.n_vt;
+// Partial slots per row the arrays hold at most, over both launches.
+__host__ __device__ __forceinline__ int plan_max_slots(const BandPlan& p) {
+  const int steps = cdiv(p.n_vt, plan_vc(p));
+  int s = plan_unit_slots(p) * (p.G < steps ? p.G : steps);
+  if (p.G2 > 0) s += SPILL_UNIT_SLOTS * (p.G2 < p.n_vt ? p.G2 : p.n_vt);
+  return s;
 }
 
 // Iterates the units of runner `runner` under the packed plan.
@@ -367,12 +386,12 @@ struct TileIter {
   int runner, G;
   int n_mt, gm, gv, n_vt, mc, rr;
   int vt0;     // first v-tile of this launch's range
-  int slot0;   // parts of the other launch before this one's in the partial slots
+  int slot0;   // partial slots of the other launch before this one's
   Packing k;
   int round;
   int m_tile;  // current m-tile (the first of the runner's mc m-tiles)
-  int part;    // vocabulary part of the current unit (this launch's; slot part + slot0)
-  int vt, vt_end;
+  int part;    // vocabulary part of the current unit (this launch's)
+  int vt, vt_end;  // its range in steps of vc v-tiles (the spill launch: v-tiles from vt0)
 
   // hdr: the workspace header the kernel that learns N wrote (HDR_*)
   __host__ __device__ void init(const BandPlan& plan, const int* hdr, int runner_index) {
@@ -386,8 +405,8 @@ struct TileIter {
     gm = hdr_word(hdr, spill ? HDR_GM2 : HDR_GM);
     gv = hdr_word(hdr, spill ? HDR_GV2 : HDR_GV);
     vt0 = spill ? vsplit : 0;
-    n_vt = spill ? plan.n_vt - vsplit : vsplit;
-    slot0 = spill ? hdr_word(hdr, HDR_GV) : 0;
+    n_vt = spill ? plan.n_vt - vsplit : cdiv(vsplit, plan_vc(plan));  // steps of vc v-tiles
+    slot0 = spill ? hdr_word(hdr, HDR_SLOT0) : 0;
     if (gm < 1) gm = 1;
     const bool none = n_mt == 0 || gv < 1 || n_vt < 1;
     if (gv < 1) gv = 1;

@@ -36,8 +36,8 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
   const int64_t base = static_cast<int64_t>(blk) * L;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   griddep_wait();  // the partials come from the LM-head kernel
-  // partial slots per row: the parts of the plan's launches times the CTAs per unit
-  const int slots = MODE == MERGE_GATHERED ? a.n_parts : a.n_rows[HDR_PARTS] * a.plan.cpu;
+  // partial slots per row over the plan's launches (header word)
+  const int slots = MODE == MERGE_GATHERED ? a.n_parts : a.n_rows[HDR_SLOTS];
 
   // ---- a3: merge of the partial slots. Thread t takes position t % Lp of the
   // block and every groups-th slot starting at t / Lp; loads are issued four
@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(THREADS) merge_commit_kernel(CommitArgs a) {
     // partial slots the workspace holds (index checks of the bounds-checked build)
     const int64_t part_n = MODE == MERGE_GATHERED
                                ? static_cast<int64_t>(a.n_parts) * a.P
-                               : static_cast<int64_t>(a.plan.cpu) * plan_max_parts(a.plan) * a.P;
+                               : static_cast<int64_t>(plan_max_slots(a.plan)) * a.P;
     int r = -1;  // the slot index of this position: its compacted row, or (gathered) the position itself
     if (jj < L && index_ok(base + jj, a.P, a.status)) {
       if constexpr (MODE == MERGE_GATHERED)

@@ -34,6 +34,15 @@
 // way cut the 8 x 2 x 32 bf16 LM head by ~11% in a diagnostic build in which
 // one of the two pairs skipped its head loads.
 //
+// Or the two pairs share token rows (the plan's vc = 2): they hold the same
+// token group and take the two v-tiles of each step of their vocabulary part
+// (v-tiles 2t and 2t + 1), each CTA loading its own head rows and a quarter
+// of its pair's token rows, multicast to the CTA of the same rank in the
+// other pair. Stage release is the same; each pair keeps its own running
+// state and writes its own partials. This halves the token rows' L2-to-SM
+// traffic instead, the larger operand when the rows are two E4M3 terms per
+// element against a one-byte head.
+//
 // CTA layout (bf16 heads, 192 threads): warp 0 TMA producer, warp 1 TMEM
 // allocation (both CTAs) and the MMA issuer (even CTA), warps 2..5 epilogue.
 // The producer and issuer loops run in the whole warp and one elected lane
@@ -340,7 +349,9 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
 
   // pairs per cluster (two share each head tile by multicast); quantised
   // heads run without clusters
-  const int MC = QUANT ? 1 : plan_mc(a.plan);
+  // pairs per cluster: two sharing head tiles (mc = 2) or token rows (vc = 2)
+  const int VC = QUANT ? 1 : plan_vc(a.plan);
+  const int MC = QUANT ? 1 : plan_mc(a.plan) * VC;
   if constexpr (pair_cluster<HF>()) {
     // launched without its cluster there is no peer CTA to map or to pair
     // MMAs with: report and do nothing
@@ -355,7 +366,8 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   // 0: the CTA that issues the pair's MMAs (bf16 heads); quantised heads: the
   // half of the v-tile this CTA takes on its own
   const uint32_t rank = QUANT ? (blockIdx.x & 1u) : (crank & 1u);
-  const int pp = static_cast<int>(crank >> 1);  // this pair's token group within the runner's m-tiles
+  const int pp = static_cast<int>(crank >> 1);  // this pair's token group (vc = 1) or v-tile (vc = 2) in the runner
+  const int pp_mt = VC == 1 ? pp : 0;           // ... its token group within the runner's m-tiles
   const uint32_t lead = crank & ~1u;            // cluster rank of this pair's issuing CTA
   const uint32_t pair_mask = 3u << (2 * pp);    // both CTAs of this pair
   const uint32_t all_mask = (1u << (2 * MC)) - 1u;
@@ -432,8 +444,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
   // heads: this CTA's token rows only
   const uint32_t tx_total = QUANT ? static_cast<uint32_t>(NT) * ATOM_ROWS_BYTES : 2u * SB;
   const uint32_t raw_base = smem_base + static_cast<uint32_t>(STAGES) * SB;  // quantised heads' raw ring
-  const CUtensorMap* tm_tok = &tmH.m[half / 16 - 1];  // box of exactly `half` rows
-  const CUtensorMap* tm_lo = &tmL.m[half / 16 - 1];   // two-term rows: the lo terms
+  const CUtensorMap* tm_tok = &tmH.m[half / 8 - 1];  // box of exactly `half` rows
+  const CUtensorMap* tm_lo = &tmL.m[half / 8 - 1];   // two-term rows: the lo terms
+  // vc = 2: boxes of a quarter of the group (NT is a multiple of 32)
+  const CUtensorMap* tm_tok_q = &tmH.m[half / 16 - 1];
+  const CUtensorMap* tm_lo_q = &tmL.m[half / 16 - 1];
 
   if (warp == 0) {
     // ------------------------------------------------------ TMA producer
@@ -451,8 +466,12 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
     it.init(a.plan, a.n_rows, pair);
     bool ok = true;
     while (ok && it.next_unit()) {
-      const int tok0 = (it.m_tile + pp) * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
-      for (int vt = it.vt; ok && vt < it.vt_end; ++vt) {
+      const int tok0 = (it.m_tile + pp_mt) * NT + (QUANT ? 0 : static_cast<int>(rank) * half);
+      for (int step = it.vt; ok && step < it.vt_end; ++step) {
+        int vt = step * VC + (VC == 2 ? pp : 0);
+        // vc = 2 and an odd v-tile count: the last step's second v-tile lies past
+        // V; load the one before it (its logits are all dead in the epilogue)
+        if (vt > 0 && vt * 256 >= a.V) --vt;
         const int vrow = vt * 256 + static_cast<int>(rank) * 128;
         for (int kb = 0; kb < nk; ++kb) {
           if (!mbar_wait_warp(smem_u32(&ctl->empty[stage]), phase ^ 1u, abort_flag, a.status)) {
@@ -474,16 +493,28 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
               for (int j = 0; j < NATOM; ++j) {
                 // the head atom's 128 rows as two boxes of 64: both loaded here, or
                 // (two pairs per cluster) this pair's half multicast to both pairs
-                if (MC == 1) {
+                if (MC == 1 || VC == 2) {
                   tma_load_2d_pair(sa + j * A_BLOCK, &tmW, fb, kb * BK + ACOLS * j, vrow, pol_w);
                   tma_load_2d_pair(sa + j * A_BLOCK + A_BLOCK / 2, &tmW, fb, kb * BK + ACOLS * j, vrow + 64, pol_w);
                 } else {
                   tma_load_2d_pair_mc(sa + j * A_BLOCK + pp * (A_BLOCK / 2), &tmW, fb, kb * BK + ACOLS * j,
                                       vrow + 64 * pp, head_mc, pol_w);
                 }
-                tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + ACOLS * j, tok0, pol_h);
+                if (VC == 2) {
+                  // this CTA's quarter of its pair's token rows, for both pairs
+                  tma_load_2d_pair_mc(sa + NATOM * A_BLOCK + j * B_BLOCK + pp * (B_BLOCK / 2), tm_tok_q, fb,
+                                      kb * BK + ACOLS * j, tok0 + pp * (half / 2), head_mc, pol_h);
+                } else {
+                  tma_load_2d_pair(sa + NATOM * A_BLOCK + j * B_BLOCK, tm_tok, fb, kb * BK + ACOLS * j, tok0, pol_h);
+                }
               }
-              if constexpr (X2) tma_load_2d_pair(sa + A_BLOCK + B_BLOCK, tm_lo, fb, kb * BK, tok0, pol_h);
+              if constexpr (X2) {
+                if (VC == 2)
+                  tma_load_2d_pair_mc(sa + A_BLOCK + B_BLOCK + pp * (B_BLOCK / 2), tm_lo_q, fb, kb * BK,
+                                      tok0 + pp * (half / 2), head_mc, pol_h);
+                else
+                  tma_load_2d_pair(sa + A_BLOCK + B_BLOCK, tm_lo, fb, kb * BK, tok0, pol_h);
+              }
             }
           }
           __syncwarp();
@@ -700,16 +731,17 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
         xd[c] = -1;
         ts[c] = 1.f;
         if constexpr (TOKS) {
-          const int row = (it.m_tile + pp) * NT + c * 32 + lane;
+          const int row = (it.m_tile + pp_mt) * NT + c * 32 + lane;
           if (c < nch && row < n_rows && a.tok_scale[row] != 0.f) ts[c] = a.tok_scale[row];
         }
         k2[c] = ts[c] * LOG2E;
         if constexpr (VERIFY) {
-          const int row = (it.m_tile + pp) * NT + c * 32 + lane;
+          const int row = (it.m_tile + pp_mt) * NT + c * 32 + lane;
           if (c < nch && row < n_rows) xd[c] = a.draft_row[row];
         }
       }
-      for (int vt = it.vt; vt < it.vt_end; ++vt) {
+      for (int step = it.vt; step < it.vt_end; ++step) {
+        const int vt = step * VC + (VC == 2 ? pp : 0);
         if (!mbar_wait_warp(smem_u32(&ctl->tfull[acc]), acc_phase, abort_flag, a.status)) {
           ok = false;
           break;
@@ -861,9 +893,11 @@ __global__ void __launch_bounds__(pair_threads<HF>(), 1)
             softmax_combine(M, S, A, tail->w[w].st.m[j], tail->w[w].st.s[j], tail->w[w].st.a[j]);
           }
         }
-        const int row = (it.m_tile + pp) * NT + j;
+        const int row = (it.m_tile + pp_mt) * NT + j;
         if (row < n_rows) {
-          const int64_t o = static_cast<int64_t>((it.slot0 + it.part) * 2 + static_cast<int>(rank)) * a.P + row;
+          // slot: the unit's first (2 per pair, both pairs with vc = 2), then pair and CTA
+          const int slot = it.slot0 + it.part * 2 * VC + (VC == 2 ? 2 * pp : 0) + static_cast<int>(rank);
+          const int64_t o = static_cast<int64_t>(slot) * a.P + row;
           a.part_m[o] = M;
           a.part_s[o] = S;
           a.part_a[o] = A;
@@ -960,10 +994,11 @@ static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg;
   cudaLaunchAttribute attr[2];
+  const int ppc = plan_mc(a.plan) * plan_vc(a.plan);  // pairs per cluster
   if (a.plan.G2 > 0) {
     // clusters of two pairs and the spill launch of single pairs behind them
     // (the header's vocabulary split assumes both run)
-    if (!pair_cluster<HF>() || plan_mc(a.plan) != 2) return cudaErrorInvalidValue;
+    if (!pair_cluster<HF>() || ppc != 2) return cudaErrorInvalidValue;
     TcArgs main = a;
     main.plan.role = 0;
     pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, true, 2);
@@ -973,11 +1008,13 @@ static cudaError_t launch_pair(const PairTokenMaps& tmH, const CUtensorMap& tmW,
     side.plan.role = 1;
     side.plan.G = a.plan.G2;
     side.plan.mc = 1;
+    side.plan.vc = 1;
+    side.plan.cpu = SPILL_UNIT_SLOTS;
     pair_config(&cfg, attr, side.plan.G, pair_threads<HF>(), st, true, true, 1);
     return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, side);
   }
-  pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, pair_cluster<HF>(),
-              pair_cluster<HF>() ? plan_mc(a.plan) : 1);
+  if (!pair_cluster<HF>() && ppc != 1) return cudaErrorInvalidValue;
+  pair_config(&cfg, attr, a.plan.G, pair_threads<HF>(), st, true, pair_cluster<HF>(), pair_cluster<HF>() ? ppc : 1);
   return cudaLaunchKernelEx(&cfg, lmhead_pair_kernel<HF, VERIFY>, tmH, tmW, tmQ, tmL, a);
 }
 

@@ -25,8 +25,8 @@ __global__ void __launch_bounds__(THREADS) merge_verify_kernel(VerifyArgs a) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int D = a.n_draft, Rq = D + 1;
   griddep_wait();  // the partials come from the LM-head kernel
-  // partial slots per row: the parts of the plan's launches times the CTAs per unit
-  const int ns = a.n_rows[HDR_PARTS] * a.plan.cpu;
+  // partial slots per row over the plan's launches (header word)
+  const int ns = a.n_rows[HDR_SLOTS];
 
   for (int i = warp; i < Rq; i += THREADS / 32) {
     const int r = q * Rq + i;

@@ -84,7 +84,7 @@ cudaError_t launch_lmhead_tc(const CUtensorMap& tmA, const CUtensorMap& tmB, con
 // boxes (64 rows: half of a CTA's head rows, see the kernel). plan.G = runners
 // (clusters of plan.mc CTA pairs), plan.BM = 0, plan.cpu = 2.
 struct PairTokenMaps {
-  CUtensorMap m[8];
+  CUtensorMap m[16];  // box heights 8, 16, ..., 128 rows: m[h / 8 - 1]
 };
 // Head formats of the pair kernel: bf16 rows staged as they are, or E4M3 /
 // NVFP4 codes decoded to bf16 inside the kernel (codes: [V, ld] bytes with

@@ -352,9 +352,23 @@ def _kernels_per_step(wl):
                                cfg.n_slots, cfg.block_len, wl.mask_token_id, wl.tau)
 
 
+@pytest.mark.parametrize("name", ["bf16_5mt_ktail", "bf16_g294", "e4m3", "e4m3_ktail", "bf16_L64", "bf16_1mt",
+                                  "bf16_2bands"])
+def test_clusters_whose_pairs_share_token_rows(name, monkeypatch):
+    # BD_PAIR_SHARE = 1: the cluster's two pairs hold the same token group and
+    # take the two v-tiles of each step (each CTA loads a quarter of the token
+    # rows for both pairs); odd v-tile counts (bf16_1mt: 4, e4m3_ktail: 3)
+    # compute a discarded v-tile past the vocabulary
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SHARE", "1")
+    _, _, rep = check(generate(SMALL[name]), variant=3)
+    assert rep.n_live > 0
+
+
+@pytest.mark.parametrize("share", ["0", "1"])
 @pytest.mark.parametrize("pct", ["50", "100", "400"])
 @pytest.mark.parametrize("name", ["bf16_5mt_ktail", "bf16_g294", "e4m3", "bf16_L64"])
-def test_spill_pairs_beside_clusters(name, pct, monkeypatch):
+def test_spill_pairs_beside_clusters(name, pct, share, monkeypatch):
     # clusters of two pairs plus the concurrent launch of single CTA pairs on
     # the SMs the clusters leave free, over the last v-tiles; the spill
     # pair's relative time per tile sets the split (50: more v-tiles for the
@@ -362,6 +376,7 @@ def test_spill_pairs_beside_clusters(name, pct, monkeypatch):
     monkeypatch.setenv("BD_PAIR_MC", "2")
     monkeypatch.setenv("BD_PAIR_SPILL", "1")
     monkeypatch.setenv("BD_SPILL_PCT", pct)
+    monkeypatch.setenv("BD_PAIR_SHARE", share)
     wl = generate(SMALL[name])
     assert _kernels_per_step(wl) in (3, 4)  # 4 where the device leaves room for spill pairs
     _, _, rep = check(wl, variant=3)
@@ -379,14 +394,16 @@ def test_full_size_b8_with_and_without_spill_pairs(spill, monkeypatch):
     assert rep.n_live > 250
 
 
+@pytest.mark.parametrize("share", ["0", "1"])
 @pytest.mark.parametrize("spill", ["0", "1"])
 @pytest.mark.parametrize("name", ["b8", "bf16_5mt_ktail", "bf16_2bands", "e4m3", "tied_full"])
-def test_device_plan_equals_the_host_plan(name, spill, monkeypatch):
+def test_device_plan_equals_the_host_plan(name, spill, share, monkeypatch):
     # the compaction kernel evaluates the plan rule with one warp once N is
-    # known; the workspace header it writes (the first seven int32 words of
+    # known; the workspace header it writes (the first eight int32 words of
     # the caller's workspace) must equal the sequential host evaluation of the
     # same rule for that N (bd_plan_header)
     monkeypatch.setenv("BD_PAIR_SPILL", spill)
+    monkeypatch.setenv("BD_PAIR_SHARE", share)
     cfg = {"b8": B8X2X32_BF16, "tied_full": B32X4X32_TIED}.get(name) or SMALL[name]
     wl = generate(cfg)
     g = wl.to("cuda")
@@ -396,13 +413,13 @@ def test_device_plan_equals_the_host_plan(name, spill, monkeypatch):
     bdc.commit_step(g.hidden, g.weight, g.pos_masked, g.block_flags, cfg.n_seq, cfg.n_slots, cfg.block_len,
                     wl.tau, weight_scale=g.weight_scale, mask_token_id=wl.mask_token_id, workspace=ws)
     torch.cuda.synchronize()
-    hdr = ws[:28].view(torch.int32).cpu().tolist()
+    hdr = ws[:32].view(torch.int32).cpu().tolist()
     n = int(((wl.pos_masked != 0) & (wl.block_flags.repeat_interleave(cfg.block_len) & 1 != 0)).sum())
     assert hdr[0] == n
     assert hdr == bdc.bd_plan_header(*args, n)
     for rows in (0, 1, n // 2, cfg.P):  # the host rule at other N stays within the plan's ranges
         h = bdc.bd_plan_header(*args, rows)
-        assert h[0] == rows and h[1] == h[3] + h[5] and 1 <= h[6]
+        assert h[0] == rows and h[1] >= h[3] + h[5] and h[7] <= h[1] and 1 <= h[6]
 
 
 def test_spill_pairs_on_many_bands(monkeypatch):
@@ -423,3 +440,14 @@ def test_clusters_of_two_pairs_on_many_bands(monkeypatch):
     wl = generate(scaled(B32X4X32_TIED, n_seq=16, n_slots=4, block_len=64, d=256, V=3000, mask_frac=0.55))
     _, _, rep = check(wl, variant=3)
     assert rep.n_live > 2048
+
+
+@pytest.mark.parametrize("share", ["0", "1"])
+def test_full_size_largest_window_in_both_cluster_layouts(share, monkeypatch):
+    # the 256 x 8 x 64 window (clusters and spill pairs by default) with the
+    # clusters' pairs sharing head tiles or token rows; sampled whole blocks
+    # including those of the first and last compacted rows
+    monkeypatch.setenv("BD_PAIR_SHARE", share)
+    wl = generate(B256X8X64_E4M3)
+    _, _, rep = check(wl, blocks=_sample_with_edges(wl, 4, seed=12))
+    assert rep.n_live > 0

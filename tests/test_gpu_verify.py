@@ -127,6 +127,17 @@ def test_every_lmhead_kernel(variant):
     check(wl, run_gpu(wl, variant), run_oracle(wl))
 
 
+@pytest.mark.parametrize("name", ["bf16_r297_ktail", "bf16_d32"])
+def test_clusters_whose_pairs_share_token_rows(name, monkeypatch):
+    """Verification rows on clusters whose two pairs take the two v-tiles of
+    each step for one token group (each pair's own entropy and draft-logit
+    partials)."""
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SHARE", "1")
+    wl = generate_verify(SMALL[name])
+    check(wl, run_gpu(wl, 3), run_oracle(wl))
+
+
 @pytest.mark.parametrize("name", ["bf16_r297_ktail", "bf16_r40"])
 def test_clusters_with_spill_pairs(name, monkeypatch):
     """Verification rows on clusters of two CTA pairs with the concurrent spill

@@ -109,12 +109,15 @@ def test_split_agrees_with_the_single_call(name):
     assert np.abs(out["conf"] - conf.cpu().numpy()).max() < 1e-5
 
 
+@pytest.mark.parametrize("share", ["0", "1"])
 @pytest.mark.parametrize("name", ["bf16_4", "e4m3_3"])
-def test_split_with_spill_pairs(name, monkeypatch):
-    # each shard's LM head on clusters of two pairs plus the spill launch
+def test_split_with_spill_pairs(name, share, monkeypatch):
+    # each shard's LM head on clusters of two pairs (sharing head tiles or
+    # token rows) plus the spill launch
     monkeypatch.setenv("BD_PAIR_MC", "2")
     monkeypatch.setenv("BD_PAIR_SPILL", "1")
     monkeypatch.setenv("BD_SPILL_PCT", "50")
+    monkeypatch.setenv("BD_PAIR_SHARE", share)
     cfg, cuts = CASES[name]
     wl = generate(cfg)
     out, _ = run_split(wl, shard_bounds(cfg.V, cuts))

@@ -42,32 +42,33 @@ def run_cases(exe, cases):
 
 
 PAIR_G, QUAD_G, SMS = 76, 36, 152
-# (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu, mc, G2, spill_pct); vt_kb =
+# (n_rows, BM, GM, vt_kb, row_bytes, G, n_vt, cpu, mc, vc, G2, spill_pct); vt_kb =
 # KiB of head per v-tile, row_bytes = bytes of a packed token row, as the
 # kernels read them; mc = m-tiles a runner holds (2: clusters of two CTA
-# pairs); G2 = spill pairs beside the clusters (0: none), spill_pct = a spill
-# pair's time per tile against a cluster pair's
+# pairs sharing head tiles), vc = v-tiles it takes per step (2: clusters of
+# two pairs sharing token rows); G2 = spill pairs beside the clusters (0:
+# none), spill_pct = a spill pair's time per tile against a cluster pair's
 CASES = [
     # pair kernel in clusters of two pairs (BM = 0: token groups from N; GM = 0: bands by rule)
-    (294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 0, 100),       # 8 x 2 x 32, d = 2048, bf16
-    (2048, 0, 0, 1024, 4096, QUAD_G, 614, 2, 2, 0, 100),      # 32 x 4 x 32
-    (8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 0, 100),      # 64 x 4 x 64, d = 4096
-    (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 0, 100),      # one row into another group (33 groups: odd)
-    (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2, 0, 100),    # 256 x 8 x 64, d = 5120, E4M3 head, two-term rows
-    (32, 0, 0, 64, 1024, QUAD_G, 16, 2, 2, 0, 100),           # the tiny window
-    (1, 0, 0, 1, 16, QUAD_G, 1, 2, 2, 0, 100),                # one row, one v-tile
-    (257, 0, 0, 1024, 4096, 3, 7, 2, 2, 0, 100),              # few runners
-    (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2, 0, 100),      # a fixed band size
+    (294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 1, 0, 100),       # 8 x 2 x 32, d = 2048, bf16
+    (2048, 0, 0, 1024, 4096, QUAD_G, 614, 2, 2, 1, 0, 100),      # 32 x 4 x 32
+    (8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 1, 0, 100),      # 64 x 4 x 64, d = 4096
+    (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 1, 0, 100),      # one row into another group (33 groups: odd)
+    (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2, 1, 0, 100),    # 256 x 8 x 64, d = 5120, E4M3 head, two-term rows
+    (32, 0, 0, 64, 1024, QUAD_G, 16, 2, 2, 1, 0, 100),           # the tiny window
+    (1, 0, 0, 1, 16, QUAD_G, 1, 2, 2, 1, 0, 100),                # one row, one v-tile
+    (257, 0, 0, 1024, 4096, 3, 7, 2, 2, 1, 0, 100),              # few runners
+    (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2, 1, 0, 100),      # a fixed band size
     # single CTA pairs (quantised heads decoded in the kernel)
-    (294, 0, 0, 1024, 4096, PAIR_G, 594, 2, 1, 0, 100),
-    (8191, 0, 0, 2048, 8192, PAIR_G, 594, 2, 1, 0, 100),
-    (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1, 0, 100),
+    (294, 0, 0, 1024, 4096, PAIR_G, 594, 2, 1, 1, 0, 100),
+    (8191, 0, 0, 2048, 8192, PAIR_G, 594, 2, 1, 1, 0, 100),
+    (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1, 1, 0, 100),
     # one-CTA kernel (BM = 128) and the SIMT kernel (BM = 32, 64-entry v-tiles)
-    (8191, 128, 0, 2048, 8192, SMS, 594, 1, 1, 0, 100),
-    (52429, 128, 0, 2560, 10240, SMS, 614, 1, 1, 0, 100),
-    (294, 32, 0, 512, 4096, 2 * SMS, 2374, 1, 1, 0, 100),
-    (32, 32, 0, 64, 1024, 2 * SMS, 64, 1, 1, 0, 100),
-    (5, 32, 0, 1, 100, 2 * SMS, 3, 1, 1, 0, 100),
+    (8191, 128, 0, 2048, 8192, SMS, 594, 1, 1, 1, 0, 100),
+    (52429, 128, 0, 2560, 10240, SMS, 614, 1, 1, 1, 0, 100),
+    (294, 32, 0, 512, 4096, 2 * SMS, 2374, 1, 1, 1, 0, 100),
+    (32, 32, 0, 64, 1024, 2 * SMS, 64, 1, 1, 1, 0, 100),
+    (5, 32, 0, 1, 100, 2 * SMS, 3, 1, 1, 1, 0, 100),
 ]
 
 
@@ -77,16 +78,17 @@ def test_plan_covers_every_tile_once_with_balanced_runners(plan_check):
     for case, r in zip(CASES, res):
         assert r[0] == "ok", (case, r)
         n_mt, gv, slots, max_load, ideal = int(r[1]), int(r[2]), int(r[3]), int(r[4]), float(r[5])
-        G, n_vt, cpu = case[5], case[6], case[7]
-        assert 1 <= gv <= min(G, n_vt) and slots == gv * cpu
+        G, n_vt, cpu, vc = case[5], case[6], case[7], case[9]
+        steps = -(-n_vt // vc)
+        assert 1 <= gv <= min(G, steps) and slots == gv * cpu * vc
         assert int(r[7]) == n_vt  # no spill launch: the main launch takes every v-tile
         # the busiest runner: within 10% of an even share plus one unit of
-        # work (ceil(n_vt / gv) v-tiles), which no static split can avoid
-        assert max_load <= 1.10 * ideal + -(-n_vt // gv), (case, r)
+        # work (ceil(steps / gv) steps), which no static split can avoid
+        assert max_load <= 1.10 * ideal + -(-steps // gv), (case, r)
 
 
 def test_plan_without_rows(plan_check):
-    (r,) = run_cases(plan_check, [(0, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 0, 100)])
+    (r,) = run_cases(plan_check, [(0, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 1, 0, 100)])
     assert r[0] == "ok" and int(r[1]) == 0
 
 
@@ -98,38 +100,57 @@ def test_band_size(plan_check):
     # single pairs; one row past 32 groups on clusters: 12; the 32 x 4 x 32
     # window is one band (8 m-tiles, within 5% of the best makespan); a fixed GM
     # is kept
-    rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 0, 100),
-                                  (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2, 0, 100),
-                                  (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1, 0, 100),
-                                  (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 0, 100),
-                                  (2048, 0, 0, 1024, 4096, PAIR_G, 614, 2, 1, 0, 100),
-                                  (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2, 0, 100)])
+    rows = run_cases(plan_check, [(8191, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 1, 0, 100),
+                                  (52429, 0, 0, 1280, 10240, QUAD_G, 614, 2, 2, 1, 0, 100),
+                                  (52429, 0, 0, 1280, 10240, PAIR_G, 614, 2, 1, 1, 0, 100),
+                                  (8200, 0, 0, 2048, 8192, QUAD_G, 594, 2, 2, 1, 0, 100),
+                                  (2048, 0, 0, 1024, 4096, PAIR_G, 614, 2, 1, 1, 0, 100),
+                                  (5000, 0, 7, 1024, 4096, QUAD_G, 100, 2, 2, 1, 0, 100)])
     assert [int(r[6]) for r in rows] == [12, 2, 4, 12, 8, 7]
     # 64 x 4 x 64 on clusters: an even share exactly (16 runner m-tiles x 594 v-tiles / 36)
     assert int(rows[0][4]) == 264
 
 
 # the clusters-of-two-pairs cases with the 4 spill pairs 152 SMs leave room for
-SPILL_CASES = [c[:9] + (4, pct) for c in CASES if c[8] == 2 and c[5] == QUAD_G for pct in (100, 110)]
+SPILL_CASES = [c[:10] + (4, pct) for c in CASES if c[8] == 2 and c[5] == QUAD_G for pct in (100, 110)]
+# the same clusters with their pairs sharing token rows (one m-tile, two v-tiles per step)
+SHARE_CASES = [c[:8] + (1, 2) + c[10:] for c in CASES if c[8] == 2 and c[5] == QUAD_G]
+SHARE_CASES += [(294, 0, 0, 1024, 4096, QUAD_G, 593, 2, 1, 2, 0, 100),  # odd v-tile count
+                (52429, 0, 0, 1280, 10240, QUAD_G, 613, 2, 1, 2, 0, 100)]
+SHARE_SPILL_CASES = [c[:10] + (4, pct) for c in SHARE_CASES for pct in (100, 110)]
 
 
-def test_spill_launch_covers_the_rest_of_the_vocabulary(plan_check):
-    res = run_cases(plan_check, SPILL_CASES)
-    assert len(res) == len(SPILL_CASES)
-    for case, r in zip(SPILL_CASES, res):
+def test_plan_with_pairs_sharing_token_rows(plan_check):
+    res = run_cases(plan_check, SHARE_CASES)
+    assert len(res) == len(SHARE_CASES)
+    for case, r in zip(SHARE_CASES, res):
         assert r[0] == "ok", (case, r)
-        n_mt, parts, slots, load, ideal, gm = int(r[1]), int(r[2]), int(r[3]), int(r[4]), float(r[5]), int(r[6])
+        gv, slots, max_load, ideal = int(r[2]), int(r[3]), int(r[4]), float(r[5])
+        steps = -(-case[6] // 2)
+        assert slots == 4 * gv  # each pair of a unit writes its own partial per CTA
+        assert max_load <= 1.10 * ideal + -(-steps // gv), (case, r)
+
+
+@pytest.mark.parametrize("cases", ["head", "tokens"])
+def test_spill_launch_covers_the_rest_of_the_vocabulary(plan_check, cases):
+    todo = SPILL_CASES if cases == "head" else SHARE_SPILL_CASES
+    res = run_cases(plan_check, todo)
+    assert len(res) == len(todo)
+    for case, r in zip(todo, res):
+        assert r[0] == "ok", (case, r)
+        n_mt, gv, slots, load, ideal, gm = int(r[1]), int(r[2]), int(r[3]), int(r[4]), float(r[5]), int(r[6])
         vsplit, load2, gm2, gv2 = int(r[7]), int(r[8]), int(r[9]), int(r[10])
-        G, n_vt, cpu, G2, pct = case[5], case[6], case[7], case[9], case[10]
-        assert 1 <= vsplit <= n_vt and slots == parts * cpu and parts <= min(G + G2, n_vt)
+        G, n_vt, cpu, vc, G2, pct = case[5], case[6], case[7], case[9], case[10], case[11]
+        assert 1 <= vsplit <= n_vt and slots == gv * cpu * vc + gv2 * 2
         if n_mt == 0 or vsplit == n_vt:
             continue
-        gv = parts - gv2
-        assert 1 <= gv2 <= min(G2, n_vt - vsplit) and 1 <= gv <= min(G, vsplit)
+        assert vsplit % vc == 0
+        steps = vsplit // vc
+        assert 1 <= gv2 <= min(G2, n_vt - vsplit) and 1 <= gv <= min(G, steps)
         # either launch's busiest runner within 10% of the even share plus one
         # unit of its launch, which no static split avoids
         w = pct / 100
-        assert load <= 1.10 * ideal + -(-vsplit // gv), (case, r)
+        assert load <= 1.10 * ideal + -(-steps // gv), (case, r)
         assert w * load2 <= 1.10 * ideal + w * -(-(n_vt - vsplit) // gv2), (case, r)
 
 
@@ -138,6 +159,14 @@ def test_spill_split_of_the_bench_window(plan_check):
     # on 36 clusters and 4 spill pairs. At equal time per tile the split
     # balances 594 v-tiles as 563 for the clusters (one m-tile pair each) and
     # 31 for the spill pairs (both m-tiles); a spill pair 10% slower gets 29
-    (a, b) = run_cases(plan_check, [(294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 4, 100),
-                                    (294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 4, 110)])
+    (a, b) = run_cases(plan_check, [(294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 1, 4, 100),
+                                    (294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 2, 1, 4, 110)])
     assert int(a[7]) == 563 and int(b[7]) == 565
+
+
+def test_token_sharing_split_is_even(plan_check):
+    # 8 x 2 x 32 window on clusters whose pairs share token rows: the split of
+    # 594 v-tiles keeps an even count for the clusters' v-tile pairs (562 at
+    # equal time per tile against 563 with head sharing)
+    (a,) = run_cases(plan_check, [(294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 1, 2, 4, 100)])
+    assert a[0] == "ok" and int(a[7]) == 562
