@@ -42,10 +42,11 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // written nowhere).
 //
 // The m-tiles are cut into bands of GM (the last band may be smaller) and the
-// vocabulary into gv contiguous parts of (nearly) equal length. A part of a
-// band is the gm units (m-tile, part) that share the same head slice; a unit
-// leaves one partial (max, sum of exponentials, argmax) per row in slot `part`
-// (times the CTAs per unit) of the partial arrays. Parts, ordered band by
+// vocabulary into gv contiguous parts of (nearly) equal length (in steps of vc
+// v-tiles when a runner takes vc at a time). A part of a band is the gm units
+// (m-tile, part) that share the same head slice; a unit leaves one partial
+// (max, sum of exponentials, argmax) per row and CTA (and pair, with vc = 2)
+// in the slots of its part. Parts, ordered band by
 // band, are packed whole into rounds of G units (G runners): a part that does
 // not fit what is left of a round starts the next round, and runner c takes
 // slot c of every round (a slot past the round's parts is idle). All m-tiles
@@ -60,8 +61,8 @@ constexpr float FUSED_SHIFT_LIMIT = 2048.f;
 // G) with GM m-tiles of rows within the in-flight budget below (they stay in
 // L2 while their parts run) and gv <= min(G, n_vt). N is only known on the
 // device: the compaction kernel evaluates the rule with one warp and stores
-// GM and gv beside N in the workspace header, which the LM-head and merge
-// kernels read.
+// the plan beside N in the workspace header (HDR_* below), which the LM-head
+// and merge kernels read.
 // -------------------------------------------------------------------------
 struct BandPlan {
   int BM;         // rows per m-tile; 0 = derived from N (token groups of the pair kernel)

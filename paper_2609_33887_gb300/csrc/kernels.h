@@ -31,8 +31,8 @@ struct TauParams {
 // bytes, a multiple of 16), exact for every element of at least 2^-10 of the
 // row's largest; tok_scale[r] = 2^-s.
 enum : int { ROWS_BF16 = 0, ROWS_E4M3 = 1, ROWS_F16_POW2 = 2, ROWS_E4M3X2 = 3 };
-// n_rows[0] = N, n_rows[1] = the plan's vocabulary parts and n_rows[2] its
-// band size for N (plan_choose), written by the CTA that holds the last position.
+// n_rows: the workspace header (N and the LM head's plan for N, HDR_* words of
+// common.cuh), written by the CTA that holds the last position.
 cudaError_t launch_prep_rows(const uint8_t* pos_masked, const uint8_t* block_flags, int P, int block_len,
                              const void* hidden, int64_t ld, int d, void* hc, int64_t ldc, int* idx, int* rowpos,
                              int* n_rows, int sm_count, cudaStream_t st, const BandPlan& plan,
@@ -170,8 +170,8 @@ cudaError_t launch_merge_commit(const CommitArgs& a, cudaStream_t st, int mode =
 // Verification path (speculative decoding, typical acceptance). Rows are
 // r = q * (n_draft + 1) + i; row i < n_draft of request q verifies draft
 // token draft[q * n_draft + i], the last row of a request gives its bonus token.
-// Prep: idx[r] = r, draft_row[r] = that draft token or -1, n_rows[0] = R,
-// n_rows[1] / n_rows[2] = the plan's vocabulary parts / band size for R rows.
+// Prep: idx[r] = r, draft_row[r] = that draft token or -1, and the workspace
+// header n_rows (R and the LM head's plan for R rows, HDR_* words of common.cuh).
 cudaError_t launch_prep_verify(const int32_t* draft, int n_req, int n_draft, int* idx, int* draft_row, int* n_rows,
                                const BandPlan& plan, cudaStream_t st);
 
