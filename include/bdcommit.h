@@ -277,7 +277,10 @@ int bd_plan_header(const bd_hidden* hidden, const bd_weight* weight, const bd_ma
  *   BD_PAIR_SPILL=0|1    with clusters of two pairs, the CTA pairs that still fit
  *                        on the SMs the clusters leave free (4 on a 152-SM GB300)
  *                        take the last v-tiles in a second, concurrent launch
- *                        (default: on for more than 256 MiB of packed rows)
+ *                        (default: on for more than 256 MiB of packed rows). The
+ *                        split assumes those SMs are free: where other work holds
+ *                        them, the spill launch runs after the clusters and the
+ *                        LM head takes about twice as long; set 0 there
  *   BD_SPILL_PCT=n       a spill pair's time per v-tile against a cluster pair's,
  *                        in percent (default 100): sets the vocabulary split
  *   BD_PLAN_GM=n, BD_PLAN_GV=n   fix the work plan's band size (runner m-tiles)
