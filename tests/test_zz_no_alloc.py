@@ -71,6 +71,23 @@ def test_static_matches_the_allocating_entry_point_twice(cfg):
     assert (ref_tok >= 0).sum() > 0
 
 
+@pytest.mark.parametrize("share", ["0", "1"])
+def test_static_with_spill_pairs_beside_clusters(share, monkeypatch):
+    # the LM head as two launches (clusters of two pairs, sharing head tiles
+    # or token rows, and the spill pairs) inside the fixed array
+    monkeypatch.setenv("BD_PAIR_MC", "2")
+    monkeypatch.setenv("BD_PAIR_SPILL", "1")
+    monkeypatch.setenv("BD_SPILL_PCT", "50")
+    monkeypatch.setenv("BD_PAIR_SHARE", share)
+    wl = generate(scaled(B8X2X32_BF16, n_seq=4, d=256, V=3000, name="b4x2x32_v3000"))
+    ref_tok, ref_conf, ref_com = _run(wl, static=False)
+    tok, conf, com = _run(wl, static=True)
+    assert np.array_equal(tok, ref_tok)
+    assert np.abs(conf.astype(np.float64) - ref_conf).max() <= CONF_TOL
+    assert np.array_equal(com, ref_com)
+    assert (ref_tok >= 0).sum() > 0
+
+
 def test_static_rejects_windows_beyond_its_array():
     # the 64 x 4 x 64, d = 4096 window needs far more than 32 MiB of workspace;
     # the call is refused before anything is queued
