@@ -25,6 +25,9 @@ constexpr int RPT = SIMT_BM / ROW_GROUPS;        // 8 rows per thread
 constexpr int CPL = SIMT_BN / 32;                // columns a lane scans in the reductions
 static_assert(THREADS % SIMT_BN == 0 && SIMT_BM % ROW_GROUPS == 0, "column x row-group split");
 static_assert(SIMT_BM == 32, "one row per lane in the reductions");
+constexpr int HE = SIMT_BM * KC / THREADS;  // hidden elements a thread stages per step
+constexpr int WE = SIMT_BN * KC / THREADS;  // head elements a thread stages per step
+static_assert(HE * THREADS == SIMT_BM * KC && WE * THREADS == SIMT_BN * KC, "whole staging rounds");
 
 __device__ __forceinline__ float load_h(const void* p, int64_t i, int dt) {
   if (dt == BD_F32) return static_cast<const float*>(p)[i];
@@ -56,6 +59,7 @@ __device__ __forceinline__ float load_w_nvfp4(const void* p, const uint8_t* bs, 
 }
 
 struct SimtSmem {
+  int rix[SIMT_BM];  // the m-tile's hidden rows (-1 past N)
   float hs[SIMT_BM][KC + 1];
   union {
     float ws[SIMT_BN][KC + 1];         // head tile during the K loop
@@ -82,6 +86,7 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
   while (it.next_unit()) {
     const int r0 = it.m_tile * SIMT_BM;
     if (tid < SIMT_BM) {
+      sm.rix[tid] = r0 + tid < n_rows ? a.idx[r0 + tid] : -1;
       sm.rm[tid] = -INFINITY;
       sm.rs[tid] = 0.f;
       sm.ra[tid] = 0x7fffffff;
@@ -98,23 +103,36 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
 #pragma unroll
       for (int r = 0; r < RPT; ++r) acc[r] = 0.f;
       for (int k0 = 0; k0 < a.d; k0 += KC) {
-        // stage 32 hidden rows x KC columns (rows gathered through idx)
-        for (int e = tid; e < SIMT_BM * KC; e += THREADS) {
-          const int r = e / KC, kk = e % KC;
-          float x = 0.f;
-          if (r0 + r < n_rows && k0 + kk < a.d)
-            x = load_h(a.hidden, static_cast<int64_t>(a.idx[r0 + r]) * a.ldh + k0 + kk, a.hdtype);
-          sm.hs[r][kk] = x;
+        // stage 32 hidden rows (gathered through idx) and SIMT_BN head rows x
+        // KC columns: every load of the thread first, then its stores, so that
+        // they are all in flight at once
+        float hv[HE], wv[WE];
+#pragma unroll
+        for (int i = 0; i < HE; ++i) {
+          const int e = tid + i * THREADS, r = e / KC, kk = e % KC;
+          const int src = sm.rix[r];
+          hv[i] = (src >= 0 && k0 + kk < a.d) ? load_h(a.hidden, static_cast<int64_t>(src) * a.ldh + k0 + kk, a.hdtype)
+                                              : 0.f;
         }
-        // stage 256 head rows x KC columns
-        for (int e = tid; e < SIMT_BN * KC; e += THREADS) {
-          const int vr = e / KC, kk = e % KC;
+#pragma unroll
+        for (int i = 0; i < WE; ++i) {
+          const int e = tid + i * THREADS, vr = e / KC, kk = e % KC;
           const int vv = vt * SIMT_BN + vr;
           float x = 0.f;
           if (vv < a.V && k0 + kk < a.d)
             x = a.wdtype == BD_NVFP4 ? load_w_nvfp4(a.w, a.wbs, vv, k0 + kk, a.ldw, a.ldbs)
                                      : load_w(a.w, static_cast<int64_t>(vv) * a.ldw + k0 + kk, a.wdtype);
-          sm.u.ws[vr][kk] = x;
+          wv[i] = x;
+        }
+#pragma unroll
+        for (int i = 0; i < HE; ++i) {
+          const int e = tid + i * THREADS;
+          sm.hs[e / KC][e % KC] = hv[i];
+        }
+#pragma unroll
+        for (int i = 0; i < WE; ++i) {
+          const int e = tid + i * THREADS;
+          sm.u.ws[e / KC][e % KC] = wv[i];
         }
         __syncthreads();
 #pragma unroll 8
