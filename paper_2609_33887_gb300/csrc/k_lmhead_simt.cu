@@ -5,7 +5,8 @@
 // verification instantiation (VERIFY = true) also carries the entropy
 // accumulator and the logit of each row's draft entry.
 //
-// A CTA of 256 threads computes a 32-row x 64-entry tile: thread t owns
+// A CTA of 256 threads computes a 32-row x 64-entry tile in 64-column K
+// steps, each step's operands loaded into registers one step ahead: thread t owns
 // vocabulary column t % 64 of the tile for rows 8 (t / 64) .. 8 (t / 64) + 7,
 // so a small window still spreads over many CTAs (the 32 x 4096 fp32 window:
 // 64 v-tiles).
@@ -18,16 +19,18 @@ namespace bd {
 
 namespace {
 
-constexpr int KC = 32;      // hidden columns staged per step
+// hidden columns staged per K step: 64, or 32 for the verification
+// instantiation (its larger epilogue state leaves fewer registers for the
+// step loaded ahead at two CTAs per SM)
+template <bool VERIFY>
+__host__ __device__ constexpr int kc_of() { return VERIFY ? 32 : 64; }
 constexpr int THREADS = 256;
 constexpr int ROW_GROUPS = THREADS / SIMT_BN;   // 4 groups of rows
 constexpr int RPT = SIMT_BM / ROW_GROUPS;        // 8 rows per thread
 constexpr int CPL = SIMT_BN / 32;                // columns a lane scans in the reductions
 static_assert(THREADS % SIMT_BN == 0 && SIMT_BM % ROW_GROUPS == 0, "column x row-group split");
 static_assert(SIMT_BM == 32, "one row per lane in the reductions");
-constexpr int HE = SIMT_BM * KC / THREADS;  // hidden elements a thread stages per step
-constexpr int WE = SIMT_BN * KC / THREADS;  // head elements a thread stages per step
-static_assert(HE * THREADS == SIMT_BM * KC && WE * THREADS == SIMT_BN * KC, "whole staging rounds");
+static_assert((SIMT_BM * 32) % THREADS == 0 && (SIMT_BN * 32) % THREADS == 0, "whole staging rounds");
 
 __device__ __forceinline__ float load_h(const void* p, int64_t i, int dt) {
   if (dt == BD_F32) return static_cast<const float*>(p)[i];
@@ -58,6 +61,7 @@ __device__ __forceinline__ float load_w_nvfp4(const void* p, const uint8_t* bs, 
   return __uint_as_float(mag | ((c & 8u) << 28)) * e4m3_to_float(bs[static_cast<int64_t>(v) * ldbs + k / 16]);
 }
 
+template <int KC>
 struct SimtSmem {
   int rix[SIMT_BM];  // the m-tile's hidden rows (-1 past N)
   float hs[SIMT_BM][KC + 1];
@@ -74,8 +78,11 @@ struct SimtSmem {
 }  // namespace
 
 template <bool VERIFY>
-__global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
-  __shared__ SimtSmem sm;
+__global__ void __launch_bounds__(THREADS, 2) lmhead_simt_kernel(SimtArgs a) {
+  constexpr int KC = kc_of<VERIFY>();
+  constexpr int HE = SIMT_BM * KC / THREADS;  // hidden elements a thread stages per step
+  constexpr int WE = SIMT_BN * KC / THREADS;  // head elements a thread stages per step
+  __shared__ SimtSmem<KC> sm;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int col = tid % SIMT_BN, rg = tid / SIMT_BN;  // this thread's column and row group
   griddep_wait();  // idx and N come from the preceding kernel
@@ -102,11 +109,11 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
       float acc[RPT];
 #pragma unroll
       for (int r = 0; r < RPT; ++r) acc[r] = 0.f;
-      for (int k0 = 0; k0 < a.d; k0 += KC) {
-        // stage 32 hidden rows (gathered through idx) and SIMT_BN head rows x
-        // KC columns: every load of the thread first, then its stores, so that
-        // they are all in flight at once
-        float hv[HE], wv[WE];
+      // 32 hidden rows (gathered through idx) and SIMT_BN head rows x KC
+      // columns per step, loaded into registers one step ahead: the next
+      // step's loads are in flight while this step's FMAs run
+      float hv[HE], wv[WE];
+      auto load_step = [&](int k0) {
 #pragma unroll
         for (int i = 0; i < HE; ++i) {
           const int e = tid + i * THREADS, r = e / KC, kk = e % KC;
@@ -124,6 +131,9 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
                                      : load_w(a.w, static_cast<int64_t>(vv) * a.ldw + k0 + kk, a.wdtype);
           wv[i] = x;
         }
+      };
+      load_step(0);
+      for (int k0 = 0; k0 < a.d; k0 += KC) {
 #pragma unroll
         for (int i = 0; i < HE; ++i) {
           const int e = tid + i * THREADS;
@@ -135,11 +145,12 @@ __global__ void __launch_bounds__(THREADS) lmhead_simt_kernel(SimtArgs a) {
           sm.u.ws[e / KC][e % KC] = wv[i];
         }
         __syncthreads();
+        if (k0 + KC < a.d) load_step(k0 + KC);
 #pragma unroll 8
         for (int kk = 0; kk < KC; ++kk) {
-          const float wv = sm.u.ws[col][kk];
+          const float wk = sm.u.ws[col][kk];
 #pragma unroll
-          for (int r = 0; r < RPT; ++r) acc[r] = fmaf(sm.hs[rg * RPT + r][kk], wv, acc[r]);
+          for (int r = 0; r < RPT; ++r) acc[r] = fmaf(sm.hs[rg * RPT + r][kk], wk, acc[r]);
         }
         __syncthreads();
       }
