@@ -191,21 +191,38 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
     // in bytes); tok_scale = 2^-s (0 for an all-zero row).
     uint8_t* hq = reinterpret_cast<uint8_t*>(hc);
     uint8_t* lq = hq + static_cast<int64_t>(P) * ldc;
+    // rows of up to 32 * RC vectors (5120 bf16) are read once, into
+    // registers: every lane's loads of the row are in flight together
+    constexpr int RC = 20;
+    const bool cached = nvec <= 32 * RC;
+    auto amax_of = [](const uint4& q) {
+      const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+      float m = 0.f;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[j]));
+        m = fmaxf(m, fmaxf(fabsf(f.x), fabsf(f.y)));
+      }
+      return m;
+    };
     for (int i = warp - w0; i < local_total; i += n_pack) {
       if (!index_ok(prefix + i, P, status)) continue;
       const int p = i < 2048 ? rows_s[i] : idx[prefix + i];
       const __nv_bfloat16* src = hidden + static_cast<int64_t>(p) * ld;
       const uint4* s4 = reinterpret_cast<const uint4*>(src);
+      uint4 qc[RC];
       float amax = 0.f;
-#pragma unroll 4
-      for (int v = lane; v < nvec; v += 32) {
-        const uint4 q = __ldg(s4 + v);
-        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+      if (cached) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[j]));
-          amax = fmaxf(amax, fmaxf(fabsf(f.x), fabsf(f.y)));
+        for (int k = 0; k < RC; ++k) {
+          const int v = lane + 32 * k;
+          qc[k] = v < nvec ? __ldg(s4 + v) : make_uint4(0u, 0u, 0u, 0u);
         }
+#pragma unroll
+        for (int k = 0; k < RC; ++k) amax = fmaxf(amax, amax_of(qc[k]));
+      } else {
+#pragma unroll 4
+        for (int v = lane; v < nvec; v += 32) amax = fmaxf(amax, amax_of(__ldg(s4 + v)));
       }
       for (int e = nvec * 8 + lane; e < d; e += 32) amax = fmaxf(amax, fabsf(__bfloat162float(src[e])));
 #pragma unroll
@@ -215,9 +232,8 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
       const float up = __uint_as_float(static_cast<uint32_t>(sh + 127) << 23);  // 2^s, exact
       uint8_t* dh = hq + static_cast<int64_t>(prefix + i) * ldc;
       uint8_t* dl = lq + static_cast<int64_t>(prefix + i) * ldc;
-#pragma unroll 4
-      for (int v = lane; v < nvec; v += 32) {
-        const uint4 q = __ldg(s4 + v);
+      // vector v of the row: eight elements as eight hi and eight lo codes
+      auto convert_store = [&](const uint4& q, int v) {
         const uint32_t w[4] = {q.x, q.y, q.z, q.w};
         uint32_t oh[2], ol[2];
 #pragma unroll
@@ -238,6 +254,16 @@ __global__ void __launch_bounds__(PREP_THREADS) prep_rows_kernel(
         }
         *reinterpret_cast<uint2*>(dh + 8 * v) = make_uint2(oh[0], oh[1]);
         *reinterpret_cast<uint2*>(dl + 8 * v) = make_uint2(ol[0], ol[1]);
+      };
+      if (cached) {
+#pragma unroll
+        for (int k = 0; k < RC; ++k) {
+          const int v = lane + 32 * k;
+          if (v < nvec) convert_store(qc[k], v);
+        }
+      } else {
+#pragma unroll 4
+        for (int v = lane; v < nvec; v += 32) convert_store(__ldg(s4 + v), v);
       }
       for (int e = nvec * 8 + lane; e < d; e += 32) {
         const float y = __bfloat162float(src[e]) * up;
