@@ -170,3 +170,39 @@ def test_token_sharing_split_is_even(plan_check):
     # equal time per tile against 563 with head sharing)
     (a,) = run_cases(plan_check, [(294, 0, 0, 1024, 4096, QUAD_G, 594, 2, 1, 2, 4, 100)])
     assert a[0] == "ok" and int(a[7]) == 562
+
+
+def _fuzz_cases(n, seed):
+    import random
+
+    rnd = random.Random(seed)
+    cases = []
+    for _ in range(n):
+        kind = rnd.choice(["pair", "pair", "tc", "simt"])
+        n_rows = rnd.choice([0, 1, rnd.randint(1, 600), rnd.randint(1, 9000), rnd.randint(1, 60000)])
+        n_vt = rnd.choice([1, 2, 3, rnd.randint(1, 40), rnd.randint(1, 700)])
+        gm = rnd.choice([0, 0, 0, rnd.randint(1, 40)])
+        vt_kb, row_bytes = rnd.choice([(1024, 4096), (2048, 8192), (1280, 10240), (64, 1024)])
+        if kind == "pair":
+            layout = rnd.choice(["pairs", "head", "tokens"])
+            mc, vc = {"pairs": (1, 1), "head": (2, 1), "tokens": (1, 2)}[layout]
+            G = rnd.choice([rnd.randint(1, 40), 36, 76]) if layout == "pairs" else rnd.choice([rnd.randint(1, 40), 36])
+            G2 = rnd.choice([0, rnd.randint(1, 8)]) if layout != "pairs" else 0
+            cases.append((n_rows, 0, gm, vt_kb, row_bytes, G, n_vt, 2, mc, vc, G2, rnd.choice([50, 100, 110, 400])))
+        else:
+            bm = 128 if kind == "tc" else 32
+            G = rnd.choice([rnd.randint(1, 320), 152, 304])
+            cases.append((n_rows, bm, gm, vt_kb, row_bytes, G, n_vt, 1, 1, 1, 0, 100))
+    return cases
+
+
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_random_plans_cover_every_tile_once(plan_check, seed):
+    # seeded random shapes over every kernel's plan and both cluster layouts,
+    # with and without spill pairs: every (m-tile, v-tile) pair computed once,
+    # parts whole within rounds, partial slots within the merge's range
+    cases = _fuzz_cases(150, seed)
+    res = run_cases(plan_check, cases)
+    assert len(res) == len(cases)
+    for case, r in zip(cases, res):
+        assert r[0] == "ok", (case, r)
